@@ -1,0 +1,505 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Each check compares the oracle with something other than itself: a closed
+form, an identity of the definitions, a library routine (scipy's entropy,
+torch's scaled-dot-product attention, Triton's Philox), or a statistical law
+(the Gumbel-max theorem).  CPU only.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+from scipy import special, stats
+
+import oracle
+import workloads
+
+pytestmark = pytest.mark.usefixtures("oracle_lib")
+
+
+def _row(z):
+    return np.asarray(z, dtype=np.float32)
+
+
+def _ets(z, T=1.0, H_prev=None, tau=0.0, H_target=None, seed=0, offset=0, **ctrl):
+    z = np.atleast_2d(np.asarray(z, np.float32))
+    B, V = z.shape
+    H_prev = np.zeros(B) if H_prev is None else np.broadcast_to(H_prev, (B,))
+    H_target = np.full(B, 0.5 * math.log(max(V, 2))) if H_target is None else np.broadcast_to(H_target, (B,))
+    return oracle.entropy_temp_sample(z, np.full(B, T), H_prev, np.broadcast_to(tau, (B,)),
+                                      H_target, oracle.ctrl(**ctrl), seed=seed, offset=offset)
+
+
+# ----------------------------------------------------------------------------
+# Entropy H_t (Section 2.1)
+
+@pytest.mark.parametrize("V", [1, 2, 7, 4096, 128256])
+@pytest.mark.parametrize("c", [0.0, -3.5, 17.25])
+def test_uniform_logits_give_log_V(V, c):
+    r = _ets(np.full(V, c), T=0.7)
+    # sequential double summation of V terms: error below ~V * 2^-53 relative
+    assert abs(r["H"][0] - math.log(V)) < (1e-13 + 4 * V * 2.0 ** -53) * max(1.0, math.log(V))
+
+
+def test_single_finite_logit_gives_zero_entropy():
+    z = np.full(1000, -np.inf, np.float32)
+    z[417] = 2.5
+    r = _ets(z)
+    assert r["H"][0] == 0.0 and r["tok"][0] == 417 and r["err"][0] == 0
+    assert r["surprisal"][0] == 0.0
+
+
+@pytest.mark.parametrize("a,T", [(0.0, 1.0), (1.0, 1.0), (-2.3, 0.5), (9.0, 3.0), (30.0, 1.0)])
+def test_two_logits_give_binary_entropy(a, T):
+    r = _ets([a, 0.0], T=T)
+    p = special.expit(float(np.float32(a)) / T)   # the oracle reads fp32 logits
+    hb = -(p * math.log(p) + (1 - p) * math.log(1 - p)) if 0 < p < 1 else 0.0
+    assert abs(r["H"][0] - hb) < 1e-12
+
+
+def test_entropy_matches_scipy_on_random_rows():
+    rng = np.random.default_rng(5)
+    for V, s, T in [(10, 1.0, 1.0), (4096, 3.0, 0.8), (50000, 10.0, 1.7), (1000, 0.1, 0.05)]:
+        z = (rng.standard_normal(V) * s).astype(np.float32)
+        T = float(np.float32(T))          # T_in is an fp32 input
+        p = special.softmax(z.astype(np.float64) / T)
+        ref = stats.entropy(p)
+        r = _ets(z, T=T)
+        assert abs(r["H"][0] - ref) < 1e-10 * max(1.0, ref)
+        assert abs(oracle.entropy_row(z, T) - ref) < 1e-10 * max(1.0, ref)
+
+
+def test_entropy_derivative_in_T_is_variance_over_T_cubed():
+    """dH/dT = Var_p(z) / T^3 for p = softmax(z/T) (differentiate -sum p log p)."""
+    rng = np.random.default_rng(7)
+    z = (rng.standard_normal(300) * 2).astype(np.float32)
+    for T in (0.3, 1.0, 2.5):
+        h = 1e-5 * T
+        fd = (oracle.entropy_row(z, T + h) - oracle.entropy_row(z, T - h)) / (2 * h)
+        p = special.softmax(z.astype(np.float64) / T)
+        zz = z.astype(np.float64)
+        var = (p * zz ** 2).sum() - (p * zz).sum() ** 2
+        assert abs(fd - var / T ** 3) < 1e-6 * max(1.0, var / T ** 3)
+
+
+def test_entropy_increases_with_T_and_tends_to_log_V():
+    rng = np.random.default_rng(8)
+    z = (rng.standard_normal(512) * 4).astype(np.float32)
+    Ts = np.geomspace(0.05, 1e5, 40)
+    Hs = [oracle.entropy_row(z, T) for T in Ts]
+    assert all(b > a for a, b in zip(Hs, Hs[1:]))
+    assert abs(Hs[-1] - math.log(512)) < 1e-6
+
+
+def test_entropy_ignores_minus_inf_logits():
+    rng = np.random.default_rng(9)
+    z = rng.standard_normal(100).astype(np.float32)
+    zi = np.concatenate([z, np.full(37, -np.inf, np.float32)])
+    assert abs(_ets(zi)["H"][0] - stats.entropy(special.softmax(z.astype(np.float64)))) < 1e-12
+
+
+def test_nonfinite_rows_flag_errors():
+    z = np.zeros((3, 16), np.float32)
+    z[0, 3] = np.nan
+    z[1, 5] = np.inf
+    z[2, :] = -np.inf
+    r = _ets(z, T=1.0, tau=2.0)
+    assert list(r["err"]) == [oracle.ERR_NONFINITE, oracle.ERR_NONFINITE, oracle.ERR_ALL_NEG_INF]
+    assert (r["tok"] == -1).all() and np.isnan(r["H"]).all()
+    assert (r["tau"] == 2.0).all() and (r["T_out"] == 1.0).all() and (r["theta_next"] == 0.0).all()
+
+
+# ----------------------------------------------------------------------------
+# Entropy flow and entropic time (Section 2)
+
+def test_entropy_flow_and_entropic_time_hand_cases():
+    V = 64
+    z_flat = np.zeros(V, np.float32)                  # H = log 64
+    z_peak = np.zeros(V, np.float32); z_peak[0] = 50  # H ~ 0
+    H_flat = math.log(V)
+    Hp = np.array([H_flat + 1.0, H_flat - 1.0, H_flat], np.float32).astype(np.float64)  # fp32 inputs
+    r = _ets(np.stack([z_flat, z_flat, z_peak]), H_prev=Hp, tau=np.array([0.5, 0.5, 0.0]))
+    assert abs(r["dH"][0] - (Hp[0] - H_flat)) < 1e-12 and abs(r["tau"][0] - (0.5 + Hp[0] - H_flat)) < 1e-12
+    assert abs(r["dH"][1] - (Hp[1] - H_flat)) < 1e-12 and r["tau"][1] == 0.5   # increases do not count
+    assert abs(r["tau"][2] - (Hp[2] - r["H"][2])) < 1e-12
+
+
+def test_entropic_time_is_monotone_along_a_trajectory():
+    rng = np.random.default_rng(11)
+    tau, Hp = 0.0, 3.0
+    for t in range(200):
+        z = (rng.standard_normal(256) * rng.uniform(0.1, 5)).astype(np.float32)
+        r = _ets(z, H_prev=Hp, tau=tau, seed=1, offset=t)
+        assert r["tau"][0] >= tau and abs((r["tau"][0] - tau) - max(0.0, Hp - r["H"][0])) < 1e-12
+        # the state arrays are fp32; carry them as such
+        tau, Hp = float(np.float32(r["tau"][0])), float(np.float32(r["H"][0]))
+
+
+# ----------------------------------------------------------------------------
+# Temperature controller (Section 3.3, Section 7.2, Appendix A)
+
+def _bisect_T(z, Hstar, lo=1e-3, hi=1e3):
+    """T* with H(T*) = H*, by bisection on scipy's entropy (H increases with T)."""
+    zz = z.astype(np.float64)
+    H = lambda T: stats.entropy(special.softmax(zz / T))
+    for _ in range(200):
+        mid = math.sqrt(lo * hi)
+        if H(mid) < Hstar:
+            lo = mid
+        else:
+            hi = mid
+    return math.sqrt(lo * hi)
+
+
+def _run_ctrl(z, T0, Hstar_seq, steps, **kw):
+    T = T0
+    Ts = [T]
+    for t in range(steps):
+        r = _ets(z, T=T, H_target=Hstar_seq(t), **kw)
+        T = float(np.float32(r["T_out"][0]))
+        Ts.append(T)
+    return np.array(Ts)
+
+
+def test_controller_converges_to_bisected_fixed_point():
+    rng = np.random.default_rng(12)
+    z = (rng.standard_normal(200) * 2.0).astype(np.float32)
+    Hstar = 0.6 * math.log(200)
+    Tstar = _bisect_T(z, Hstar)
+    Ts = _run_ctrl(z, 1.0, lambda t: Hstar, 400, eta=0.2, T_min=0.01, T_max=100.0)
+    assert abs(math.log(Ts[-1]) - math.log(Tstar)) < 1e-5
+    for T0 in (0.02, 50.0):
+        Ts = _run_ctrl(z, T0, lambda t: Hstar, 400, eta=0.2, T_min=0.01, T_max=100.0)
+        assert abs(math.log(Ts[-1]) - math.log(Tstar)) < 1e-5
+
+
+def test_controller_saturates_at_clip_bounds():
+    rng = np.random.default_rng(13)
+    z = (rng.standard_normal(50) * 3).astype(np.float32)
+    # target above what T_max can reach -> pinned at T_max
+    Ts = _run_ctrl(z, 1.0, lambda t: math.log(50) + 1.0, 300, eta=0.5, T_min=0.05, T_max=5.0)
+    assert Ts[-1] == np.float32(5.0)
+    # target 0 is unreachable for T >= T_min -> pinned at T_min
+    Ts = _run_ctrl(z, 1.0, lambda t: 0.0, 300, eta=0.5, T_min=0.05, T_max=5.0)
+    assert Ts[-1] == np.float32(0.05)
+
+
+def test_printed_sign_runs_off_to_a_bound():
+    """With the formula exactly as printed (sigma = +1) the loop is positive feedback."""
+    rng = np.random.default_rng(14)
+    z = (rng.standard_normal(200) * 2).astype(np.float32)
+    Hstar = 0.6 * math.log(200)
+    Tstar = _bisect_T(z, Hstar)
+    for T0, bound in ((Tstar * 1.01, 100.0), (Tstar * 0.99, 0.01)):
+        Ts = _run_ctrl(z, T0, lambda t: Hstar, 2000, eta=0.2, sign=1.0, T_min=0.01, T_max=100.0)
+        assert Ts[-1] == np.float32(bound)
+
+
+def test_iss_bound_under_bounded_estimator_noise():
+    """Appendix A: |delta_t| <= a^t |delta_0| + eps_H / mu, a = 1 - eta mu, in log-temperature,
+    with the estimate H + e_t (|e_t| <= eps_H) fed to the restoring law."""
+    rng = np.random.default_rng(15)
+    z = (rng.standard_normal(300) * 1.5).astype(np.float32)
+    Hstar = 0.7 * math.log(300)
+    Tstar = _bisect_T(z, Hstar)
+    xs = math.log(Tstar)
+    zz = z.astype(np.float64)
+    Hx = lambda x: stats.entropy(special.softmax(zz / math.exp(x)))
+    r, eta, eps = 0.6, 0.3, 0.02
+    # restoring slope mu: the smallest secant slope of H(e^x) over the neighbourhood
+    grid = np.linspace(-r, r, 241)
+    grid = grid[grid != 0]
+    mu = min((Hx(xs + d) - Hstar) / d for d in grid)
+    slope_max = max((Hx(xs + d) - Hstar) / d for d in grid)
+    assert mu > 0 and eta * slope_max < 1.0
+    a = 1.0 - eta * mu
+    noise = rng.uniform(-eps, eps, size=500)
+    delta0 = 0.5
+    Ts = _run_ctrl(z, Tstar * math.exp(delta0), lambda t: Hstar - noise[t], 500,
+                   eta=eta, T_min=1e-3, T_max=1e3)
+    for t, T in enumerate(Ts):
+        d = abs(math.log(T) - xs)
+        assert d <= r
+        assert d <= a ** t * delta0 + eps / mu + 1e-6
+
+
+def test_threshold_floor():
+    """theta_next = min(theta_user, theta_hi * max(0, 1 - max(H - eps_H, H_min)/log V))."""
+    V = 1000
+    rng = np.random.default_rng(16)
+    z = (rng.standard_normal(V) * 2).astype(np.float32)
+    H = stats.entropy(special.softmax(z.astype(np.float64)))
+    for kw in [dict(), dict(eps_H=0.5), dict(H_min=0.9 * math.log(V)), dict(theta_user=0.2),
+               dict(theta_hi=2.0, eps_H=100.0)]:
+        c = oracle.ctrl(**kw)
+        Heff = max(H - c["eps_H"], c["H_min"])
+        want = min(c["theta_user"], c["theta_hi"] * max(0.0, 1 - Heff / math.log(V)))
+        assert abs(_ets(z, **kw)["theta_next"][0] - want) < 1e-12
+
+
+# ----------------------------------------------------------------------------
+# Sampler: Philox4x32-10 and the Gumbel-max draw
+
+def test_philox_matches_tritons_independent_implementation():
+    """Triton's Philox4x32-10 (run by its CPU interpreter) on random counters and 64-bit keys."""
+    pytest.importorskip("triton")
+    import subprocess, sys, json, os
+    rng = np.random.default_rng(0)
+    ctr = rng.integers(0, 2 ** 32, size=(64, 4), dtype=np.uint64).astype(np.uint32)
+    seeds = [0, 1, 0xFFFFFFFF, 0x123456789ABCDEF0, 2 ** 64 - 1]
+    prog = r'''
+import os, sys, json
+os.environ["TRITON_INTERPRET"] = "1"
+import numpy as np, torch, triton, triton.language as tl
+@triton.jit
+def k(out_ptr, c_ptr, seed, N: tl.constexpr):
+    o = tl.arange(0, N)
+    c0 = tl.load(c_ptr + o * 4 + 0); c1 = tl.load(c_ptr + o * 4 + 1)
+    c2 = tl.load(c_ptr + o * 4 + 2); c3 = tl.load(c_ptr + o * 4 + 3)
+    r0, r1, r2, r3 = tl.philox(seed, c0, c1, c2, c3, 10)
+    tl.store(out_ptr + o * 4 + 0, r0); tl.store(out_ptr + o * 4 + 1, r1)
+    tl.store(out_ptr + o * 4 + 2, r2); tl.store(out_ptr + o * 4 + 3, r3)
+inp = json.loads(sys.stdin.read())
+c = torch.tensor(np.array(inp["ctr"], dtype=np.uint32).view(np.int32))
+res = []
+for s in inp["seeds"]:
+    out = torch.zeros(c.numel(), dtype=torch.int32)
+    k[(1,)](out, c, s, c.shape[0] // 4)
+    res.append(out.numpy().view(np.uint32).tolist())
+print(json.dumps(res))
+'''
+    env = dict(os.environ, TRITON_INTERPRET="1")
+    p = subprocess.run([sys.executable, "-c", prog], input=json.dumps(
+        {"ctr": ctr.reshape(-1).tolist(), "seeds": seeds}), capture_output=True, text=True,
+        env=env, timeout=600)
+    if p.returncode != 0:
+        pytest.skip("triton interpreter unavailable: " + p.stderr[-300:])
+    res = json.loads(p.stdout.strip().splitlines()[-1])
+    for s, r in zip(seeds, res):
+        key = np.tile(np.array([s & 0xFFFFFFFF, s >> 32], np.uint32), (64, 1))
+        assert (oracle.philox4x32_10(ctr, key).reshape(-1) == np.array(r, np.uint32)).all(), hex(s)
+
+
+def test_uniforms_lie_on_the_open_lattice_and_are_uniform():
+    u = np.concatenate([oracle.uniforms(3, o, b, 0, 25000) for o in (0, 1 << 40) for b in (0, 7)])
+    j = u * 2 ** 24
+    assert np.all(u > 0) and np.all(u < 1)
+    assert np.all(np.abs(j - np.round(j)) == 0) and np.all(np.round(j) % 2 == 1)
+    assert stats.kstest(u, "uniform").pvalue > 1e-4
+    # distinct rows and offsets draw distinct streams
+    a, b2 = oracle.uniforms(3, 0, 0, 0, 1000), oracle.uniforms(3, 0, 1, 0, 1000)
+    c = oracle.uniforms(3, 1, 0, 0, 1000)
+    assert np.mean(a == b2) < 0.01 and np.mean(a == c) < 0.01
+
+
+@pytest.mark.parametrize("T", [1.0, 0.5, 2.0])
+def test_gumbel_max_frequencies_follow_softmax(T):
+    """Gumbel-max theorem: argmax(y + G) is a draw from softmax(y).  One row per draw."""
+    z = np.array([0.0, 1.0, -0.5, 2.0, 0.3, -np.inf, 1.5], np.float32)
+    N = 40000
+    r = _ets(np.tile(z, (N, 1)), T=T, seed=99)
+    p = special.softmax(np.where(np.isinf(z), -np.inf, z.astype(np.float64) / T))
+    counts = np.bincount(r["tok"], minlength=len(z))
+    assert counts[5] == 0
+    keep = p > 0
+    chi = stats.chisquare(counts[keep], N * p[keep])
+    assert chi.pvalue > 1e-4, (counts, N * p)
+
+
+def test_sample_is_reproducible_and_offset_dependent():
+    rng = np.random.default_rng(17)
+    z = rng.standard_normal((32, 500)).astype(np.float32)
+    a = _ets(z, seed=5, offset=9)["tok"]
+    assert (a == _ets(z, seed=5, offset=9)["tok"]).all()
+    assert np.mean(a == _ets(z, seed=5, offset=10)["tok"]) < 0.5
+    assert np.mean(a == _ets(z, seed=6, offset=9)["tok"]) < 0.5
+
+
+def test_sample_key_and_margin_are_consistent():
+    rng = np.random.default_rng(18)
+    z = rng.standard_normal((4, 300)).astype(np.float32)
+    T = float(np.float32(0.9))
+    r = _ets(z, T=T, seed=2, offset=3)
+    for b in range(4):
+        keys = np.array([oracle.sample_key(z[b], T, 2, 3, b, x) for x in range(300)])
+        assert keys.argmax() == r["tok"][b]
+        srt = np.sort(keys)
+        assert abs((srt[-1] - srt[-2]) - r["margin"][b]) < 1e-12
+        # surprisal = -log softmax(z/T)[tok]
+        p = special.softmax(z[b].astype(np.float64) / T)
+        assert abs(r["surprisal"][b] + math.log(p[r["tok"][b]])) < 1e-10
+
+
+# ----------------------------------------------------------------------------
+# Block scores, keep set (Section 3.2) and restricted attention
+
+def _small_kv(B=3, Hq=8, Hkv=2, D=32, P=16, lens=(37, 64, 5), seed=21, hi=0.2):
+    w = workloads.Workload("pin", B=B, Hq=Hq, Hkv=Hkv, D=D, P=P, V=16, ctx=("list", list(lens)),
+                           seed=seed, hi_frac=hi)
+    kv = workloads.make_kv(w, "cpu")
+    return w, kv, dict(q=workloads.bf16_bits(kv["q"]), k=workloads.bf16_bits(kv["k_cache"]),
+                       v=workloads.bf16_bits(kv["v_cache"]), bt=kv["block_table"].numpy(),
+                       L=kv["ctx_lens"].numpy(), scale=kv["scale"])
+
+
+def _dense(n, b, which="k"):
+    """K or V of sequence b as [Hkv, L, D] float64, gathered by page."""
+    L, P = int(n["L"][b]), n["k"].shape[2]
+    pages = n["bt"][b, :(L + P - 1) // P]
+    c = n[which][pages].astype(np.uint32) << 16
+    x = c.view(np.float32).astype(np.float64)             # [nb, Hkv, P, D]
+    return x.transpose(1, 0, 2, 3).reshape(x.shape[1], -1, x.shape[3])[:, :L]
+
+
+def _q(n):
+    return (n["q"].astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def test_block_scores_sum_to_attention_entropy():
+    """Reading R4: sum_b I_b^(h) is the entropy of head h's attention (scipy on torch logits)."""
+    w, kv, n = _small_kv()
+    r = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1, want_heads=True)
+    g = w.Hq // w.Hkv
+    qd = _q(n)
+    for b in range(w.B):
+        K = torch.from_numpy(_dense(n, b, "k"))
+        for h in range(w.Hq):
+            x = (K[h // g] @ torch.from_numpy(qd[b, h])) * n["scale"]
+            Ha = stats.entropy(torch.softmax(x, 0).numpy())
+            assert abs(r["head_H"][b, h] - Ha) < 1e-10
+            assert abs(r["head_I"][b, h].sum() - Ha) < 1e-10
+
+
+def test_uniform_attention_closed_form():
+    """q = 0: a_i = 1/L, so I_b = (t_b/L) log L and Ibar_b = n_b t_b / L."""
+    w, kv, n = _small_kv(lens=(37, 64, 5, 16), B=4)
+    q0 = np.zeros_like(n["q"])
+    r = oracle.score_prune(q0, n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1)
+    for b in range(w.B):
+        L = int(n["L"][b]); nb = -(-L // w.P)
+        t = np.array([min(w.P, L - j * w.P) for j in range(nb)])
+        want = nb * t / L if L > 1 else np.ones(nb)
+        for kvh in range(w.Hkv):
+            assert np.allclose(r["block_score"][b, kvh, :nb], want, rtol=0, atol=1e-12)
+
+
+def test_keep_set_rules():
+    w, kv, n = _small_kv(B=3, lens=(200, 129, 48), seed=22)
+    args = (n["q"], n["k"], n["bt"], n["L"], n["scale"])
+    nbs = [-(-int(L) // w.P) for L in n["L"]]
+    allk = oracle.score_prune(*args, np.zeros(w.B), 1)
+    for b, nb in enumerate(nbs):
+        assert (allk["kept_cnt"][b] == nb).all()
+        assert (allk["keep_mask"][b, :, :nb] == 1).all() and (allk["keep_mask"][b, :, nb:] == 0).all()
+        assert (allk["kept_idx"][b, :, :nb] == np.arange(nb)).all()
+    inf = np.full(w.B, np.inf)
+    big = oracle.score_prune(*args, inf, 10 ** 6)
+    assert (big["kept_cnt"] == np.array(nbs)[:, None]).all()
+    for k in (0, 1, 3, 7):
+        r = oracle.score_prune(*args, inf, k)
+        assert (r["kept_cnt"] == np.minimum(k, np.array(nbs))[:, None]).all()
+        for b, nb in enumerate(nbs):
+            for kvh in range(w.Hkv):
+                s = allk["block_score"][b, kvh, :nb]
+                order = sorted(range(nb), key=lambda j: (-s[j], j))[:min(k, nb)]
+                assert set(np.nonzero(r["keep_mask"][b, kvh])[0]) == set(order)
+                kept = r["kept_idx"][b, kvh, :r["kept_cnt"][b, kvh]]
+                assert (np.diff(kept) > 0).all()
+    # monotone in theta; the score threshold applies with >=
+    prev = None
+    for th in (0.0, 0.5, 0.9, 1.0, 1.3, 2.0, 5.0):
+        r = oracle.score_prune(*args, np.full(w.B, th), 1)
+        s = allk["block_score"]
+        for b, nb in enumerate(nbs):
+            for kvh in range(w.Hkv):
+                m = r["keep_mask"][b, kvh, :nb].astype(bool)
+                assert (m[s[b, kvh, :nb] >= th]).all()
+        if prev is not None:
+            assert (r["keep_mask"] <= prev).all()
+        prev = r["keep_mask"]
+
+
+def test_block_of_equally_attended_tokens_ranks_first():
+    """A block whose keys all equal c*q takes nearly all of the attention, spread evenly over
+    its tokens, so its share of the attention entropy (and its score) is the largest."""
+    w, kv, n = _small_kv(B=1, Hq=1, Hkv=1, lens=(160,), seed=23, hi=0.0)
+    qd = _q(n)[0, 0]
+    k = n["k"].copy()
+    page = n["bt"][0, 6]
+    aligned = (qd * 2.0).astype(np.float32).view(np.uint32) >> 16
+    k[page, 0, :, :] = aligned.astype(np.uint16)
+    r = oracle.score_prune(n["q"], k, n["bt"], n["L"], n["scale"], np.full(1, np.inf), 1)
+    assert r["kept_cnt"][0, 0] == 1 and r["kept_idx"][0, 0, 0] == 6
+
+
+def _sdpa(qd, K, V, scale, g):
+    q = torch.from_numpy(qd)[:, None, :]                  # [Hq, 1, D]
+    Kx = torch.from_numpy(K).repeat_interleave(g, 0)      # [Hq, L, D]
+    Vx = torch.from_numpy(V).repeat_interleave(g, 0)
+    return torch.nn.functional.scaled_dot_product_attention(q, Kx, Vx, scale=scale)[:, 0].numpy()
+
+
+def test_keep_all_attention_equals_library_dense_attention():
+    w, kv, n = _small_kv(B=3, Hq=8, Hkv=2, D=32, lens=(37, 64, 5))
+    out, err = oracle.paged_attention(n["q"], n["k"], n["v"], n["bt"], n["L"], n["scale"])
+    assert (err == 0).all()
+    qd = _q(n)
+    for b in range(w.B):
+        ref = _sdpa(qd[b], _dense(n, b, "k"), _dense(n, b, "v"), n["scale"], w.Hq // w.Hkv)
+        assert np.abs(out[b] - ref).max() < 1e-12
+    ones = np.ones((w.B, w.Hkv, w.max_blocks), np.uint8)
+    out2, _ = oracle.paged_attention(n["q"], n["k"], n["v"], n["bt"], n["L"], n["scale"], ones)
+    assert np.array_equal(out, out2)
+
+
+def test_restricted_attention_equals_dense_attention_over_kept_tokens():
+    w, kv, n = _small_kv(B=2, Hq=4, Hkv=2, D=32, lens=(150, 90), seed=24)
+    rng = np.random.default_rng(0)
+    mask = (rng.random((w.B, w.Hkv, w.max_blocks)) < 0.5).astype(np.uint8)
+    out, _ = oracle.paged_attention(n["q"], n["k"], n["v"], n["bt"], n["L"], n["scale"], mask)
+    qd = _q(n)
+    g = w.Hq // w.Hkv
+    for b in range(w.B):
+        K, V = _dense(n, b, "k"), _dense(n, b, "v")
+        L = int(n["L"][b])
+        for kvh in range(w.Hkv):
+            tok = [i for i in range(L) if mask[b, kvh, i // w.P]]
+            for hh in range(g):
+                h = kvh * g + hh
+                if not tok:
+                    assert (out[b, h] == 0).all()
+                    continue
+                ref = _sdpa(qd[b, h:h + 1], K[kvh:kvh + 1, tok], V[kvh:kvh + 1, tok], n["scale"], 1)
+                assert np.abs(out[b, h] - ref[0]).max() < 1e-12
+
+
+def test_attention_and_scores_invariant_under_page_permutation():
+    w, kv, n = _small_kv(B=3, lens=(100, 33, 64), seed=25)
+    rng = np.random.default_rng(1)
+    perm = rng.permutation(n["k"].shape[0])            # new page id of old page p: inv[p]
+    inv = np.empty_like(perm); inv[perm] = np.arange(len(perm))
+    k2, v2 = n["k"][perm], n["v"][perm]
+    bt2 = np.where(n["bt"] >= 0, inv[np.maximum(n["bt"], 0)], -1).astype(np.int32)
+    o1, _ = oracle.paged_attention(n["q"], n["k"], n["v"], n["bt"], n["L"], n["scale"])
+    o2, _ = oracle.paged_attention(n["q"], k2, v2, bt2, n["L"], n["scale"])
+    assert np.array_equal(o1, o2)
+    s1 = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], np.full(w.B, 0.8), 2)
+    s2 = oracle.score_prune(n["q"], k2, bt2, n["L"], n["scale"], np.full(w.B, 0.8), 2)
+    assert np.array_equal(s1["block_score"], s2["block_score"])
+    assert np.array_equal(s1["keep_mask"], s2["keep_mask"])
+
+
+def test_empty_sequences_and_bad_inputs():
+    w, kv, n = _small_kv(B=3, lens=(0, 40, 40), seed=26)
+    bt = n["bt"].copy()
+    bt[2, 1] = n["k"].shape[0] + 5                       # page id past the pool
+    L = n["L"].copy()
+    out, err = oracle.paged_attention(n["q"], n["k"], n["v"], bt, L, n["scale"])
+    assert list(err) == [0, 0, oracle.ERR_BAD_PAGE]
+    assert (out[0] == 0).all() and (out[2] == 0).all() and np.abs(out[1]).sum() > 0
+    r = oracle.score_prune(n["q"], n["k"], bt, L, n["scale"], np.zeros(3), 1)
+    assert (r["kept_cnt"][0] == 0).all() and (r["kept_cnt"][2] == 0).all()
+    L[1] = w.max_blocks * w.P + 1
+    _, err = oracle.paged_attention(n["q"], n["k"], n["v"], bt, L, n["scale"])
+    assert err[1] == oracle.ERR_BAD_CTX
