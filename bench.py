@@ -1,0 +1,454 @@
+"""Benchmark of the entropic-time batched decode step on GB300.
+
+One step = one pass of the whole hot path over one batch:
+  score every key page (eti_score_blocks) -> keep set, budget, compaction and
+  kept-token normaliser (eti_prune_blocks) -> GQA paged decode over the kept
+  blocks (eti_paged_decode) -> entropy / entropic time / temperature /
+  threshold / sample (eti_entropy_temp_sample).
+The workload is the Llama-3-8B-shaped layer step (64 sequences, 32 query /
+8 kv heads, head_dim 128, page 16, context lengths uniform in [1024, 8192],
+vocabulary 128,256) with seeded synthetic inputs.
+
+Prints ONE JSON line (rank 0).  Timing: W warm-up steps, then K timed steps;
+before every step a buffer of twice the L2 size is written (L2 flush); each
+kernel call is bracketed by CUDA events on the launching stream and the step
+time is the sum of its calls.  `value` = sequences decoded per second per
+layer step over all ranks (each rank decodes its own batch: weak scaling).
+
+--impl reference times the fp64 CPU oracle on a bounded sample of the same
+workload (the paper has no reference implementation).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np
+import torch
+
+import workloads
+
+METRIC = "paged-decode tokens/s per layer-step"
+UNIT = "tokens/s"
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return rank, world, local
+
+
+def shard_workload(w: workloads.Workload, rank: int) -> workloads.Workload:
+    """Each rank decodes its own batch of the same shape (independent sequences)."""
+    return w.scaled(seed=w.seed + 7919 * rank) if rank else w
+
+
+def aggregate(per_rank_step_s: list[float], B: int) -> tuple[float, float]:
+    """Whole-job throughput from every rank's step time: all ranks' sequences
+    over the slowest rank's time."""
+    slowest = max(per_rank_step_s)
+    return B * len(per_rank_step_s) / slowest, slowest
+
+
+def max_over_ranks(x: float, world: int, device) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while it runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int, log_path: str | None = None):
+        self.index, self.log_path, self.proc, self.lines = index, log_path, None, []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.index), "-lms", "100"], stdout=subprocess.PIPE,
+                stderr=subprocess.DEVNULL, text=True)
+            self._t = threading.Thread(target=self._read, daemon=True)
+            self._t.start()
+            t0 = time.time()
+            while not self.lines and time.time() - t0 < 10 and self.proc.poll() is None:
+                time.sleep(0.02)           # the timed region starts once sampling runs
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self._t.join(timeout=2)
+        if self.log_path and self.lines:
+            with open(self.log_path, "w") as f:
+                f.write("\n".join(self.lines) + "\n")
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx = float(parts[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+def algorithmic_bytes(w, L: np.ndarray, kept_blocks: int) -> dict:
+    """Compulsory DRAM bytes per call of each kernel (see the design notes)."""
+    g = w.Hq // w.Hkv
+    nb = -(-L // w.P)
+    tokens_slots = int(nb.sum()) * w.P                   # token slots of all blocks
+    k_bytes = int(L.sum()) * w.Hkv * w.D * 2             # every key read once
+    q_bytes = w.B * w.Hq * w.D * 2
+    score_bytes = tokens_slots * w.Hq * 4                # x_i written for every slot
+    stats_bytes = int(nb.sum()) * w.Hq * 16
+    kept_slots = kept_blocks * w.P
+    return {
+        "score": k_bytes + q_bytes + score_bytes + stats_bytes,
+        "prune": stats_bytes + int(nb.sum()) * w.Hkv * 5,
+        # kept V pages + their scores + the bf16 output
+        "decode": kept_slots * w.D * 2 + kept_slots * g * 4 + w.B * w.Hq * w.D * 2,
+        "sample": w.B * w.V * 4,
+    }
+
+
+def run_gpu(args):
+    import paper_2603_03310_gb300 as eti
+
+    rank, world, local = dist_env()
+    device = torch.device(f"cuda:{local}")
+    torch.cuda.set_device(device)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=device)
+    eti.load()
+    w = shard_workload(workloads.WORKLOADS[args.workload], rank)
+    kv = workloads.make_kv(w, device)
+    lg = workloads.make_logits(w, device)
+    g = w.Hq // w.Hkv
+    step = eti.DecodeStep(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, w.V, device=device)
+    stats = torch.empty((w.B, w.Hkv, w.max_blocks, g, 4), dtype=torch.float32, device=device)
+    shape = (w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks)
+    prm = eti.ctrl_params()
+    # threshold of this step: theta_next of the previous step's entropy (same logits)
+    tau0 = lg["tau"].clone()
+    step.sample(lg["logits"], lg["T_in"], lg["H_prev"], tau0, lg["H_target"], params=prm,
+                seed=w.seed)
+    theta = step.theta_next.clone()
+    B_min = 1
+    stream = torch.cuda.current_stream()
+    L2 = torch.cuda.get_device_properties(device).L2_cache_size
+    flush = torch.empty(max(2 * L2, 256 << 20), dtype=torch.uint8, device=device)
+
+    def one_step(ev=None, offset=0):
+        if ev is not None:
+            ev[0].record(stream)
+        eti.eti_score_blocks(kv["q"], kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
+                             stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
+        if ev is not None:
+            ev[1].record(stream)
+        eti.eti_prune_blocks(stats, kv["block_table"], kv["ctx_lens"], shape, theta, B_min,
+                             step.keep_mask, step.kept_idx, step.kept_cnt, step.err_attn,
+                             kept_norm=step.kept_norm, num_pages=kv["num_pages"])
+        if ev is not None:
+            ev[2].record(stream)
+        eti.eti_paged_decode(kv["q"], kv["k_cache"], kv["v_cache"], kv["block_table"],
+                             kv["ctx_lens"], kv["scale"], step.out, step.err_dec, step.ws_dec,
+                             kept_idx=step.kept_idx, kept_cnt=step.kept_cnt,
+                             token_scores=step.token_scores, kept_norm=step.kept_norm,
+                             num_pages=kv["num_pages"])
+        if ev is not None:
+            ev[3].record(stream)
+        step.sample(lg["logits"], lg["T_in"], lg["H_prev"], lg["tau"], lg["H_target"], params=prm,
+                    seed=w.seed, offset=offset)
+        if ev is not None:
+            ev[4].record(stream)
+
+    for i in range(args.warmup):
+        flush.zero_()
+        one_step(offset=i)
+    torch.cuda.synchronize()
+    kept = int(step.kept_cnt.sum().item())
+    L = kv["ctx_lens"].cpu().numpy()
+    total_blocks = int((-(-L // w.P)).sum()) * w.Hkv
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    torch.cuda.synchronize()
+    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+    clock_log = os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
+    with ClockSampler(local, clock_log) as clk:
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            flush.zero_()
+            one_step(evs[i], offset=args.warmup + i)
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    if world > 1:
+        dist.barrier()
+    names = ["score", "prune", "decode", "sample"]
+    per = {n: [evs[i][j].elapsed_time(evs[i][j + 1]) for i in range(args.steps)]
+           for j, n in enumerate(names)}
+    step_ms = [sum(per[n][i] for n in names) for i in range(args.steps)]
+    ms_local = statistics.mean(step_ms)
+    ms = max_over_ranks(ms_local, world, device)
+    value, _ = aggregate([ms / 1e3] * world, w.B)
+    mean_ms = {n: statistics.mean(v) for n, v in per.items()}
+    abytes = algorithmic_bytes(w, L, kept)
+    dom = max(mean_ms, key=mean_ms.get)
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+        peak, peak_src = float(peaks["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        peak, peak_src = 6800.0, "fallback"
+    achieved = {n: abytes[n] / (mean_ms[n] / 1e3) / 1e9 for n in names}
+    roof = {"kernel": {"score": "score_blocks", "prune": "prune_finalize",
+                       "decode": "paged_decode (plan + decode + combine)",
+                       "sample": "entropy_temp_sample"}[dom],
+            "bound": "hbm", "achieved": round(achieved[dom], 1), "peak": peak, "unit": "GB/s",
+            "frac": round(achieved[dom] / peak, 4), "peak_source": peak_src,
+            "bytes_per_launch": abytes[dom], "ms_per_launch": round(mean_ms[dom], 5),
+            "traffic": args.traffic}
+
+    # end to end through the public API: host (pinned) inputs -> device -> step -> host results
+    e2e = None if args.no_e2e else run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm,
+                                           args, device)
+
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16/fp32",
+        "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
+        "config": {"workload": f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} D={w.D} P={w.P} "
+                               f"ctx U[{w.ctx[1]},{w.ctx[2]}] V={w.V}",
+                   "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write)",
+                   "parallelism": f"replicas x{world} (independent batches)", "B_min": B_min,
+                   "theta": "theta_next of the step's own entropy (defaults)",
+                   "kept_fraction": round(kept / total_blocks, 4)},
+        "roofline": roof,
+        "kernels_ms": {n: round(v, 5) for n, v in mean_ms.items()},
+        "kernels_gbs": {n: round(v, 1) for n, v in achieved.items()},
+        "entropy_sample_gbs": round(achieved["sample"], 1),
+        "attention_tbs": round((abytes["score"] + abytes["decode"]) /
+                               ((mean_ms["score"] + mean_ms["prune"] + mean_ms["decode"]) / 1e3) / 1e12, 3),
+        "gpu_launches": 6 * args.steps,
+        "launches_per_step": {"score_blocks": 1, "prune_finalize": 1, "decode_plan": 1,
+                              "paged_decode": 1, "decode_combine": 1, "entropy_temp_sample": 1},
+        "e2e": e2e,
+        "wall_s_timed_region": round(wall, 4),
+        "clocks": clk.summary(),
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(w, kv, lg, theta, B_min, budget_s=args.cpu_budget)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device):
+    """Same metric through the public API from pinned host buffers: per step the
+    step's inputs (q, logits, per-sequence state, threshold) go host -> device and
+    its results (attention output, token, entropy, temperature, threshold) come back."""
+    h_q = kv["q"].cpu().pin_memory()
+    h_logits = lg["logits"].cpu().pin_memory()
+    h_state = torch.stack([lg["T_in"], lg["H_prev"], lg["H_target"], lg["tau"], theta]).cpu().pin_memory()
+    d_q = torch.empty_like(kv["q"])
+    d_logits = torch.empty_like(lg["logits"])
+    d_state = torch.empty_like(h_state, device=device)
+    h_out = torch.empty(step.out.shape, dtype=step.out.dtype).pin_memory()
+    h_res = torch.empty((4, w.B), dtype=torch.float32).pin_memory()
+    h_tok = torch.empty(w.B, dtype=torch.int32).pin_memory()
+
+    def e2e_step(i):
+        d_q.copy_(h_q, non_blocking=True)
+        d_logits.copy_(h_logits, non_blocking=True)
+        d_state.copy_(h_state, non_blocking=True)
+        T_in, H_prev, H_tgt, tau, th = d_state[0], d_state[1], d_state[2], d_state[3], d_state[4]
+        eti.eti_score_blocks(d_q, kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
+                             stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
+        eti.eti_prune_blocks(stats, kv["block_table"], kv["ctx_lens"], shape, th.contiguous(), B_min,
+                             step.keep_mask, step.kept_idx, step.kept_cnt, step.err_attn,
+                             kept_norm=step.kept_norm, num_pages=kv["num_pages"])
+        eti.eti_paged_decode(d_q, kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
+                             kv["scale"], step.out, step.err_dec, step.ws_dec,
+                             kept_idx=step.kept_idx, kept_cnt=step.kept_cnt,
+                             token_scores=step.token_scores, kept_norm=step.kept_norm,
+                             num_pages=kv["num_pages"])
+        step.sample(d_logits, T_in.contiguous(), H_prev.contiguous(), tau.contiguous(),
+                    H_tgt.contiguous(), params=prm, seed=w.seed, offset=i)
+        h_out.copy_(step.out, non_blocking=True)
+        h_tok.copy_(step.tok, non_blocking=True)
+        h_res[0].copy_(step.H, non_blocking=True)
+        h_res[1].copy_(step.T_out, non_blocking=True)
+        h_res[2].copy_(step.theta_next, non_blocking=True)
+        h_res[3].copy_(step.surprisal, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+
+    for i in range(args.warmup):
+        e2e_step(i)
+    times = []
+    for i in range(args.steps):
+        t0 = time.perf_counter()
+        e2e_step(i)
+        times.append(time.perf_counter() - t0)
+    s = statistics.mean(times)
+    bi = h_q.numel() * 2 + h_logits.numel() * 4 + h_state.numel() * 4
+    bo = h_out.numel() * 2 + h_tok.numel() * 4 + h_res.numel() * 4
+    return {"value": round(w.B / s, 1), "unit": UNIT, "ms_per_step": round(s * 1e3, 4),
+            "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo)}
+
+
+# ---------------------------------------------------------------------------
+def oracle_step(w, sub, lg_np, theta_np, B_min, seqs, seed):
+    """One decode step of the oracle on the given sequences (host arrays)."""
+    import oracle
+    r = oracle.score_prune(sub["q"], sub["k_cache"], sub["block_table"], sub["ctx_lens"],
+                           sub["scale"], theta_np[seqs], B_min)
+    oracle.paged_attention(sub["q"], sub["k_cache"], sub["v_cache"], sub["block_table"],
+                           sub["ctx_lens"], sub["scale"], r["keep_mask"])
+    oracle.entropy_temp_sample(lg_np["logits"][seqs], lg_np["T_in"][seqs], lg_np["H_prev"][seqs],
+                               lg_np["tau"][seqs], lg_np["H_target"][seqs], seed=seed)
+
+
+def _oracle_sample(w, kv, lg, theta, budget_s):
+    """Pick a sample of sequences so one oracle step takes about budget_s seconds."""
+    import oracle
+    oracle.build()
+    lg_np = {k: (v.cpu().numpy() if torch.is_tensor(v) else v) for k, v in lg.items()}
+    theta_np = theta.cpu().numpy() if torch.is_tensor(theta) else theta
+    n = 1
+    while True:
+        seqs = list(range(n))
+        sub = workloads.gather_sequences(kv, seqs)
+        t0 = time.perf_counter()
+        oracle_step(w, sub, lg_np, theta_np, 1, seqs, w.seed)
+        dt = time.perf_counter() - t0
+        if n >= w.B or dt > budget_s / 4:
+            break
+        n = min(w.B, max(n + 1, int(n * min(8.0, budget_s / 2 / max(dt, 1e-3)))))
+    return seqs, sub, lg_np, theta_np, dt
+
+
+def cpu_baseline(w, kv, lg, theta, B_min, budget_s=15.0):
+    import oracle
+    seqs, sub, lg_np, theta_np, dt = _oracle_sample(w, kv, lg, theta, budget_s)
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        oracle_step(w, sub, lg_np, theta_np, B_min, seqs, w.seed)
+        reps += 1
+        if time.perf_counter() - t0 > budget_s / 2:
+            break
+    s = (time.perf_counter() - t0) / reps
+    return {"value": round(len(seqs) / s, 3), "unit": UNIT, "cores": oracle.num_threads(),
+            "kind": "oracle",
+            "sample": f"{len(seqs)} of {w.B} sequences of the same workload, full step "
+                      f"(scores + keep set + attention + entropy/sample), {reps} rep(s), fp64 C + OpenMP"}
+
+
+def run_reference(args):
+    """The oracle as the reference arm, on this host's cores, rank 0 only."""
+    rank, world, local = dist_env()
+    if rank != 0:
+        return
+    import oracle
+    oracle.build()
+    w = workloads.WORKLOADS[args.workload]
+    kv = workloads.make_kv(w, "cpu")
+    lg = workloads.make_logits(w, "cpu")
+    r = oracle.entropy_temp_sample(lg["logits"].numpy(), lg["T_in"].numpy(), lg["H_prev"].numpy(),
+                                   lg["tau"].numpy(), lg["H_target"].numpy(), seed=w.seed)
+    theta = r["theta_next"].astype(np.float32)
+    budget = max(1.0, args.cpu_budget / max(1, args.steps + args.warmup))
+    seqs, sub, lg_np, theta_np, _ = _oracle_sample(w, kv, lg, theta, budget)
+    for _ in range(args.warmup):
+        oracle_step(w, sub, lg_np, theta_np, 1, seqs, w.seed)
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        oracle_step(w, sub, lg_np, theta_np, 1, seqs, w.seed)
+        times.append(time.perf_counter() - t0)
+    s = statistics.mean(times)
+    v = round(len(seqs) / s, 3)
+    sample = (f"{len(seqs)} of {w.B} sequences per step, full step (scores + keep set + "
+              f"attention + entropy/sample), fp64 C + OpenMP")
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(s * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
+        "config": {"workload": f"{w.name} (oracle sample)", "global_batch": len(seqs)},
+        "cpu_baseline": {"value": v, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=3000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", choices=("eti", "reference"), default="eti")
+    ap.add_argument("--workload", default="llama3_8b", choices=sorted(workloads.WORKLOADS))
+    ap.add_argument("--cpu-budget", type=float, default=15.0,
+                    help="seconds of oracle work for the CPU baseline")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--traffic", type=float, default=None,
+                    help="ncu dram bytes per launch of the dominant kernel, if measured")
+    args = ap.parse_args(argv)
+    if args.warmup < 3 and args.impl == "eti":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_gpu(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,240 @@
+/*
+ * eti.h -- C ABI of libeti, the GB300 (sm_103a) kernels of the entropic-time
+ * batched decode step (Kiruluta, "Entropic-Time Inference: Self-Organizing
+ * Large Language Model Decoding Beyond Attention", arXiv 2603.03310).
+ *
+ * The step has two halves:
+ *   (a) per sequence: softmax and Shannon entropy H_t of the vocabulary
+ *       logits at the current temperature T_t (Section 2.1), the entropy
+ *       flow dH_t and entropic time tau (Section 2), the next temperature
+ *       (Section 3.3), the next pruning threshold (Section 3.2,
+ *       "Conservative pruning", and Section 5, entropy floor) and a token
+ *       drawn from p_t;
+ *   (b) per sequence and kv head: entropic scores of the paged KV blocks
+ *       (Section 3.2, I_b), the keep set B_t = {b : I_b >= theta_t} with the
+ *       minimum block budget B_min (Section 3.2), and GQA paged decode
+ *       attention restricted to B_t.
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every tensor argument is a DEVICE pointer owned by the caller, row-major
+ *    and contiguous unless a leading dimension is given; outputs are
+ *    preallocated by the caller.  bf16 data is passed as uint16_t bit
+ *    patterns (eti_bf16).  Small parameter structs are HOST pointers and are
+ *    read before the call returns.
+ *  - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls only
+ *    enqueue work: they never synchronise, never allocate device memory and
+ *    keep no state between calls.  Scratch comes from the caller's `ws`
+ *    buffer, sized by the matching *_workspace_size() function.
+ *  - Return value: ETI_OK or a negative ETI_ERR_* status for argument errors
+ *    detected on the host (nothing is enqueued then) or a failed launch.
+ *  - Problems found in the DATA on the device never trap: each call writes
+ *    one word of ETI_ERRF_* bits per sequence into `err_flags` (uint32 [B],
+ *    overwritten, 0 = fine) and gives that sequence a defined fallback
+ *    result, documented per call.
+ *  - Supported shapes: head_dim D in {64, 128}; page size P in {16, 32};
+ *    Hq % Hkv == 0 with group size g = Hq / Hkv <= 8; 1 <= max_blocks <= 32768;
+ *    B <= 65535 (entropy/sample) or 8192 (attention calls); 1 <= V.
+ *    q, k_cache, v_cache must be 16-byte aligned.
+ *
+ * Layouts
+ *  - q          bf16  [B][Hq][D]
+ *  - k_cache    bf16  [num_pages][Hkv][P][D]   (one (page, kv head) chunk is
+ *    v_cache    bf16  [num_pages][Hkv][P][D]    P*D*2 contiguous bytes)
+ *  - block_table int32 [B][max_blocks]: physical page of logical block j of
+ *    sequence b; only entries j < ceil(ctx_lens[b] / P) are read.
+ *  - ctx_lens   int32 [B]: tokens of sequence b (0 allowed).
+ *  - keep_mask  uint8 [B][Hkv][max_blocks]; kept_idx int32 [B][Hkv][max_blocks]
+ *    (kept block indices ascending, -1 after kept_cnt); kept_cnt int32 [B][Hkv].
+ *  - token_scores fp32 [B][Hkv][max_blocks][P][g]: x_i = scale * q_h . k_i
+ *    for every token slot (-inf past the sequence end).
+ *  - kept_norm  fp32 [B][Hq][2]: (max, sum of exp(x - max)) of the softmax
+ *    over the kept tokens of each query head.
+ */
+#ifndef ETI_H_
+#define ETI_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t eti_bf16;
+
+/* status codes */
+#define ETI_OK               0
+#define ETI_ERR_NULL        (-1)  /* a required pointer is NULL */
+#define ETI_ERR_SHAPE       (-2)  /* a size is out of range or inconsistent */
+#define ETI_ERR_UNSUPPORTED (-3)  /* a valid shape this build does not implement */
+#define ETI_ERR_WORKSPACE   (-4)  /* ws is NULL or smaller than *_workspace_size() */
+#define ETI_ERR_CUDA        (-5)  /* a kernel launch failed (cudaGetLastError) */
+#define ETI_ERR_ALIGN       (-6)  /* a bf16 tensor is not 16-byte aligned */
+
+/* per-sequence data error bits written to err_flags */
+#define ETI_ERRF_BAD_PAGE     0x1u  /* a block_table entry is outside [0, num_pages) */
+#define ETI_ERRF_BAD_CTX      0x2u  /* ctx_len < 0 or > max_blocks * P */
+#define ETI_ERRF_NONFINITE    0x4u  /* a logit is NaN or +inf */
+#define ETI_ERRF_ALL_NEG_INF  0x8u  /* every logit of the row is -inf */
+#define ETI_ERRF_BAD_TEMP     0x10u /* T_in is not a positive finite number */
+
+/*
+ * Controller parameters (Section 3.3 temperature law, Section 3.2 safety
+ * floor, Section 5 guards).  The paper gives no values; eti_ctrl_defaults()
+ * fills the defaults this library documents.
+ *   eta         gain of the temperature law                       (default 0.1)
+ *   sign        -1: T' = T exp(eta (H* - H)), which restores H toward H*
+ *               because H grows with T; +1: the law exactly as printed in
+ *               Section 3.3, which is positive feedback          (default -1)
+ *   T_min,T_max clip range of the temperature               (0.05, 5.0)
+ *   eps_H       bound on the entropy-estimate error, subtracted before the
+ *               threshold floor (Section 3.2)                     (0)
+ *   H_min       entropy floor for pruning decisions (Section 5)   (0)
+ *   theta_user  threshold before the safety floor                 (+inf)
+ *   theta_hi    scale of theta_max(H) = theta_hi * max(0, 1 - H / log V) (1)
+ */
+typedef struct {
+    float eta;
+    float sign;
+    float T_min;
+    float T_max;
+    float eps_H;
+    float H_min;
+    float theta_user;
+    float theta_hi;
+} eti_ctrl_params;
+
+void eti_ctrl_defaults(eti_ctrl_params* p);
+
+/*
+ * eti_entropy_temp_sample -- half (a) of the step, one fused pass per row.
+ *
+ * For each sequence b, with y = z / T_in[b] over the first V entries of row
+ * b of `logits` (fp32, row stride ld >= V elements):
+ *   H[b]       = -sum_x p(x) log p(x),  p = softmax(y)          (Section 2.1)
+ *   dH[b]      = H_prev[b] - H[b]                                (Section 2)
+ *   tau[b]    += max(0, dH[b])         (entropic time, in place; Section 2)
+ *   T_out[b]   = clip(T_in[b] exp(sign eta (H[b] - H_target[b])), T_min, T_max)
+ *                                                                (Section 3.3)
+ *   theta_next[b] = min(theta_user, theta_hi max(0, 1 - max(H - eps_H, H_min) / log V))
+ *                  (threshold floor of Section 3.2 with the Section 5 floor;
+ *                   theta_hi when V == 1)
+ *   tok[b]     = argmax_x y_x - log(-log u_x): a draw from p by the Gumbel-max
+ *                rule, u_x from Philox4x32-10 with counter
+ *                (x / 4, b, lo32(offset), hi32(offset)), key (lo32(seed),
+ *                hi32(seed)), word x mod 4, u = (2 (word >> 9) + 1) / 2^24;
+ *                ties go to the lowest token id; -inf logits are never drawn
+ *   tok_surprisal[b] = -log p(tok)
+ * H, dH, T_out, theta_next, tok_surprisal: fp32 [B]; tok: int32 [B];
+ * dH, theta_next, tok_surprisal may be NULL.  T_in, H_prev, H_target: fp32
+ * [B].  T_out may alias T_in.
+ * Row errors (NaN/+inf logit, all -inf, bad T_in) give tok = -1, H = dH =
+ * surprisal = NaN, T_out = T_in, theta_next = 0 (prune nothing), tau unchanged.
+ * Uses no workspace.
+ */
+int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
+                            const float* T_in, const float* H_prev, float* tau,
+                            const float* H_target, const eti_ctrl_params* params,
+                            uint64_t seed, uint64_t offset,
+                            int32_t* tok, float* H, float* T_out,
+                            float* dH, float* theta_next, float* tok_surprisal,
+                            uint32_t* err_flags, void* stream);
+
+/*
+ * eti_score_prune_blocks -- the entropic keep set of half (b).
+ *
+ * For each sequence b, query head h and token i < ctx_lens[b]:
+ *   x_i = scale * q[b,h,:] . k_i,   a_i = softmax_i(x_i) over all tokens,
+ *   I_b^(h) = sum_{i in block} a_i (-log a_i)
+ * (Section 3.2 with the surprisal of value i read as -log a_i, so that the
+ * block scores add up to the attention entropy), normalised to
+ *   Ibar_b^(h) = n_b I_b^(h) / sum_b' I_b'^(h)   (1 when the sum is 0),
+ * grouped per kv head as Ibar_b = max over the g query heads of the group.
+ * Block b of (sequence, kv head) is kept iff Ibar_b >= theta[b_seq] (Section
+ * 3.2) or b is among the first min(B_min, n_b) blocks ordered by (Ibar
+ * descending, block index ascending) (minimum budget, Section 3.2).
+ *
+ * Outputs: keep_mask, kept_idx, kept_cnt (layouts above); block_score fp32
+ * [B][Hkv][max_blocks] = Ibar (0 past n_b), nullable; token_scores and
+ * kept_norm (layouts above), nullable together -- when given,
+ * eti_paged_decode reuses them and reads no key page again.
+ * theta: fp32 [B] (typically theta_next of the previous step; <= 0 keeps
+ * every block, +inf keeps only the B_min budget).
+ * A sequence with a bad page id or context length keeps nothing
+ * (kept_cnt = 0) and gets its error bit.
+ * Workspace: eti_score_prune_workspace_size(...) bytes.
+ */
+size_t eti_score_prune_workspace_size(int B, int Hq, int Hkv, int D, int P, int max_blocks);
+
+int eti_score_prune_blocks(const eti_bf16* q, const eti_bf16* k_cache,
+                           const int32_t* block_table, const int32_t* ctx_lens,
+                           int B, int Hq, int Hkv, int D, int P, int max_blocks,
+                           int64_t num_pages, float scale,
+                           const float* theta, int B_min,
+                           uint8_t* keep_mask, int32_t* kept_idx, int32_t* kept_cnt,
+                           float* block_score, float* token_scores, float* kept_norm,
+                           uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * The two steps of eti_score_prune_blocks, callable separately (same
+ * arguments and semantics; block_stats is the caller's buffer in place of the
+ * workspace):
+ *   eti_score_blocks  -- the scoring pass over every key page: token_scores
+ *                        (nullable) and block_stats fp32 [B][Hkv][max_blocks][g][4]
+ *                        = (m = max x, sum e^{x - m} - 1, sum e^{x - m}(x - m), 0)
+ *                        per block and query head (the second entry excludes one
+ *                        token at the max, which contributes exactly 1, so it
+ *                        keeps full relative precision; garbage past n_b).
+ *   eti_prune_blocks  -- the keep set, budget, compaction and kept-token
+ *                        normaliser from block_stats; writes err_flags.
+ */
+int eti_score_blocks(const eti_bf16* q, const eti_bf16* k_cache,
+                     const int32_t* block_table, const int32_t* ctx_lens,
+                     int B, int Hq, int Hkv, int D, int P, int max_blocks,
+                     int64_t num_pages, float scale,
+                     float* token_scores, float* block_stats, void* stream);
+
+int eti_prune_blocks(const float* block_stats, const int32_t* block_table,
+                     const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
+                     int max_blocks, int64_t num_pages, const float* theta, int B_min,
+                     uint8_t* keep_mask, int32_t* kept_idx, int32_t* kept_cnt,
+                     float* block_score, float* kept_norm, uint32_t* err_flags, void* stream);
+
+/*
+ * eti_paged_decode -- GQA paged decode attention restricted to the kept
+ * blocks (Section 3.2: attention computation is restricted to B_t; the
+ * softmax is renormalised over the kept tokens):
+ *   out[b,h,:] = sum_{i kept} softmax_kept(x_i) v_i,   x_i = scale q_h . k_i
+ * out: bf16 [B][Hq][D].
+ * The keep set comes from, in order of precedence: kept_idx + kept_cnt,
+ * else keep_mask, else every block (dense decode).
+ * When token_scores and kept_norm from eti_score_prune_blocks are given
+ * (with kept_idx + kept_cnt from the same call), only the kept V pages and
+ * kept scores are read; otherwise the keys of every block are scored first.
+ * A sequence with no kept token, a bad page id or a bad context length gets
+ * a zero output (and its error bit for the last two).
+ * Workspace: eti_paged_decode_workspace_size(..., have_scores) bytes, where
+ * have_scores says whether token_scores/kept_norm will be passed.
+ */
+size_t eti_paged_decode_workspace_size(int B, int Hq, int Hkv, int D, int P, int max_blocks,
+                                       int have_scores);
+
+int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16* v_cache,
+                     const int32_t* block_table, const int32_t* ctx_lens,
+                     int B, int Hq, int Hkv, int D, int P, int max_blocks,
+                     int64_t num_pages, float scale,
+                     const uint8_t* keep_mask, const int32_t* kept_idx, const int32_t* kept_cnt,
+                     const float* token_scores, const float* kept_norm,
+                     eti_bf16* out, uint32_t* err_flags,
+                     void* ws, size_t ws_bytes, void* stream);
+
+/* Version string and a readable name for a status code. */
+const char* eti_version(void);
+const char* eti_status_string(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ETI_H_ */

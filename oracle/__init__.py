@@ -30,6 +30,7 @@ ERR_BAD_PAGE = 0x1
 ERR_BAD_CTX = 0x2
 ERR_NONFINITE = 0x4
 ERR_ALL_NEG_INF = 0x8
+ERR_BAD_TEMP = 0x10
 
 
 def build(force: bool = False) -> str:

@@ -43,6 +43,7 @@
 #define ORC_ERR_BAD_CTX       0x2u
 #define ORC_ERR_NONFINITE     0x4u
 #define ORC_ERR_ALL_NEG_INF   0x8u
+#define ORC_ERR_BAD_TEMP      0x10u
 
 int oracle_num_threads(void) {
 #ifdef _OPENMP
@@ -149,7 +150,8 @@ typedef struct {
  *  surprisal = -log p(tok)
  *
  * Outputs are double.  margin[b] = best key minus second-best key.  Rows with
- * a NaN or +inf logit, or with every logit -inf, set an error bit and return
+ * a NaN or +inf logit, with every logit -inf, or with a temperature that is
+ * not a positive finite number, set an error bit and return
  * H = NaN, tok = -1, T_out = T_in, theta_next = 0 (prune nothing), tau unchanged.
  */
 void oracle_entropy_temp_sample(const float *logits, int B, int64_t V, int64_t ld,
@@ -164,9 +166,9 @@ void oracle_entropy_temp_sample(const float *logits, int B, int64_t V, int64_t l
     for (int b = 0; b < B; ++b) {
         const float *z = logits + (int64_t)b * ld;
         const double T = (double)T_in[b];
-        uint32_t e = 0;
+        uint32_t e = (T > 0.0 && !isinf(T)) ? 0u : ORC_ERR_BAD_TEMP;
         double m = -INFINITY;
-        for (int64_t x = 0; x < V; ++x) {
+        for (int64_t x = 0; x < V && !e; ++x) {
             double zx = (double)z[x];
             if (isnan(zx) || (isinf(zx) && zx > 0)) e |= ORC_ERR_NONFINITE;
             else if (zx / T > m) m = zx / T;

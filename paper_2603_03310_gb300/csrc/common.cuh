@@ -1,0 +1,119 @@
+// common.cuh -- device helpers shared by the libeti kernels (sm_103a).
+//
+// Thin wrappers around single PTX instructions: streaming 128-bit loads, the
+// MUFU exp2 / log2 approximations, the legacy bf16 tensor-core tile
+// (mma.sync m16n8k16) and warp shuffles.  No math routine is re-derived here:
+// ex2/lg2 are the hardware approximations, used where the callers' error
+// analysis allows them, and the accurate libdevice functions are called where
+// it does not.
+#pragma once
+
+#include <cstdint>
+#include <type_traits>
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include "../../include/eti.h"
+
+namespace eti {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr float kInf = __builtin_huge_valf();
+
+// 16-byte read-only load that does not allocate in L1 (data read once).
+__device__ __forceinline__ uint4 ldg_stream_u4(const void* p) {
+    uint4 r;
+    asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+        : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+        : "l"(p));
+    return r;
+}
+
+__device__ __forceinline__ float4 ldg_stream_f4(const float* p) {
+    float4 r;
+    asm("ld.global.nc.L1::no_allocate.v4.f32 {%0,%1,%2,%3}, [%4];"
+        : "=f"(r.x), "=f"(r.y), "=f"(r.z), "=f"(r.w)
+        : "l"(p));
+    return r;
+}
+
+__device__ __forceinline__ uint2 ldg_stream_u2(const void* p) {
+    uint2 r;
+    asm("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];"
+        : "=r"(r.x), "=r"(r.y)
+        : "l"(p));
+    return r;
+}
+
+// 2^x, hardware approximation (MUFU.EX2), denormal results flushed to zero.
+__device__ __forceinline__ float fast_ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// log2(x), hardware approximation (MUFU.LG2).
+__device__ __forceinline__ float fast_lg2(float x) {
+    float y;
+    asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// D += A * B on one m16n8k16 bf16 tile with fp32 accumulators.
+// Fragment ownership (lane = 4 * grp + t):
+//   A (16x16, row-major): a0 = A[grp][2t..2t+1], a1 = A[grp+8][2t..2t+1],
+//                         a2 = A[grp][2t+8..2t+9], a3 = A[grp+8][2t+8..2t+9]
+//   B (16x8, col-major):  b0 = B[2t..2t+1][grp], b1 = B[2t+8..2t+9][grp]
+//   D (16x8):             d0,d1 = D[grp][2t..2t+1], d2,d3 = D[grp+8][2t..2t+1]
+__device__ __forceinline__ void mma_bf16_16x8x16(float (&d)[4], uint32_t a0, uint32_t a1,
+                                                 uint32_t a2, uint32_t a3, uint32_t b0,
+                                                 uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 "
+        "{%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%0,%1,%2,%3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Pack two fp32 values into a bf16x2 register (round to nearest even);
+// `lo` lands in the low half.
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+// Low / high bf16 halves of two registers combined into one register.
+__device__ __forceinline__ uint32_t lo_halves(uint32_t a, uint32_t b) { return __byte_perm(a, b, 0x5410); }
+__device__ __forceinline__ uint32_t hi_halves(uint32_t a, uint32_t b) { return __byte_perm(a, b, 0x7632); }
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__device__ __forceinline__ int warp_sum_i(int v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+__host__ __device__ __forceinline__ int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+// Blocks of a sequence with context length L (0 for an invalid length, which
+// the finalizing kernels report).
+__device__ __forceinline__ int seq_blocks(int L, int P, int max_blocks) {
+    if (L <= 0 || L > max_blocks * P) return 0;
+    return (L + P - 1) / P;
+}
+
+}  // namespace eti

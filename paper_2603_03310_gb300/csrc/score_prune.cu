@@ -1,0 +1,667 @@
+// score_prune.cu -- entropic block scores and the keep set (Section 3.2).
+//
+// score_blocks (the HBM-bound pass): every key page chunk (page, kv head) is
+// read exactly once.  Warps walk a flattened list of (sequence, kv head,
+// block) units, each warp taking an equal contiguous share (no idle tail);
+// a unit is P/16 tiles of 16 tokens x D.  Each tile is loaded straight into
+// registers with 128-bit streaming loads in the A-fragment order of a bf16
+// m16n8k16 tensor-core tile (tokens = M, query heads of the GQA group = N,
+// head_dim = K; the K index is permuted identically in the key and query
+// fragments, so a thread's 16-byte load feeds two MMAs), and the next tile's
+// loads are issued before the current tile is consumed.  Per block and query
+// head it emits the stats (m_b, l_b, u_b) = (max x, sum e^{x-m_b},
+// sum e^{x-m_b}(x-m_b)) and, optionally, the scaled scores x_i themselves so
+// the decode pass never reads a key page again.
+//
+// prune_finalize (one CTA per (sequence, kv head)): with M = max_b m_b and
+// Z = sum_b l_b e^{m_b - M}, the block term of the attention entropy is
+//   I_b = e^{m_b - M} [ l_b (log Z + M - m_b) - u_b ] / Z,
+// which is sum_{i in b} a_i (-log a_i) with a_i = e^{x_i - M} / Z written
+// over the block stats (both bracket terms are >= 0, so no cancellation).
+// Then the normalised group score, the threshold, the B_min budget (radix
+// select, ties to the lower block index), compaction, and the kept-token
+// softmax normaliser (max, sum) that the decode pass uses.
+#include "common.cuh"
+
+namespace eti {
+
+constexpr int kScoreThreads = 256;
+constexpr int kScoreWarps = kScoreThreads / 32;
+constexpr int kFinThreads = 256;
+
+struct ScoreArgs {
+    const uint16_t* q;
+    const uint16_t* k_cache;
+    const int32_t* block_table;
+    const int32_t* ctx_lens;
+    int B, Hq, Hkv, g, max_blocks;
+    long long num_pages;
+    float scale;
+    float* token_scores;   // [B][Hkv][max_blocks][P][g] or null
+    float4* stats;         // [B][Hkv][max_blocks][g]: (m, l, u, 0)
+};
+
+// Exclusive prefix over sequences of (blocks * Hkv) into shared memory;
+// returns the total.  cum has B + 1 entries.
+__device__ int units_prefix(const int32_t* ctx_lens, int B, int P, int max_blocks, int Hkv,
+                            int* cum, int* warp_tot) {
+    const int tid = threadIdx.x, nt = blockDim.x;
+    int carry = 0;
+    for (int base = 0; base < B; base += nt) {
+        const int b = base + tid;
+        const int v = b < B ? seq_blocks(ctx_lens[b], P, max_blocks) * Hkv : 0;
+        // block-wide inclusive scan
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if ((tid & 31) >= o) x += y;
+        }
+        if ((tid & 31) == 31) warp_tot[tid >> 5] = x;
+        __syncthreads();
+        int wofs = 0, tot = 0;
+        for (int w = 0; w < (nt >> 5); ++w) {
+            if (w < (tid >> 5)) wofs += warp_tot[w];
+            tot += warp_tot[w];
+        }
+        if (b < B) cum[b] = carry + wofs + x - v;
+        carry += tot;
+        __syncthreads();
+    }
+    if (tid == 0) cum[B] = carry;
+    __syncthreads();
+    return carry;
+}
+
+template <int D>
+struct KTile {
+    static constexpr int kChunks = D / 32;   // 16-byte loads per token row per thread
+    uint4 lo[kChunks];                        // token grp
+    uint4 hi[kChunks];                        // token grp + 8
+};
+
+template <int D>
+__device__ __forceinline__ void load_k_tile(KTile<D>& t, const uint16_t* tile, int grp, int tq,
+                                            bool valid) {
+#pragma unroll
+    for (int c = 0; c < KTile<D>::kChunks; ++c) {
+        if (valid) {
+            t.lo[c] = ldg_stream_u4(tile + grp * D + 32 * c + 8 * tq);
+            t.hi[c] = ldg_stream_u4(tile + (grp + 8) * D + 32 * c + 8 * tq);
+        } else {
+            t.lo[c] = make_uint4(0, 0, 0, 0);
+            t.hi[c] = make_uint4(0, 0, 0, 0);
+        }
+    }
+}
+
+// Cursor over a warp's units (sequence, kv head, block, tile).
+struct UnitCursor {
+    int b, kvh, blk, tile, nb;
+};
+
+__device__ __forceinline__ void cursor_advance(UnitCursor& u, const int32_t* ctx_lens, int P,
+                                               int max_blocks, int Hkv, int tiles) {
+    if (++u.tile < tiles) return;
+    u.tile = 0;
+    if (++u.blk < u.nb) return;
+    u.blk = 0;
+    if (++u.kvh < Hkv) return;
+    u.kvh = 0;
+    do {
+        ++u.b;
+        u.nb = seq_blocks(ctx_lens[u.b], P, max_blocks);
+    } while (u.nb == 0);
+}
+
+template <int D, int P>
+__global__ void __launch_bounds__(kScoreThreads, 2)
+score_blocks_kernel(const ScoreArgs a) {
+    extern __shared__ int smem_cum[];
+    __shared__ int warp_tot[kScoreWarps];
+    constexpr int kTiles = P / 16;
+    const int total = units_prefix(a.ctx_lens, a.B, P, a.max_blocks, a.Hkv, smem_cum, warp_tot);
+    const int lane = threadIdx.x & 31, grp = lane >> 2, tq = lane & 3;
+    const int gwarp = blockIdx.x * kScoreWarps + (threadIdx.x >> 5);
+    const int nwarps = gridDim.x * kScoreWarps;
+    const int share = (total + nwarps - 1) / nwarps;
+    const int u0 = gwarp * share;
+    const int u1 = min(u0 + share, total);
+    if (u0 >= u1) return;
+
+    // locate the first unit: largest b with cum[b] <= u0 (and blocks > 0)
+    int lo = 0, hi = a.B - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (smem_cum[mid] <= u0) lo = mid; else hi = mid - 1;
+    }
+    UnitCursor cur;
+    cur.b = lo;
+    cur.nb = seq_blocks(a.ctx_lens[lo], P, a.max_blocks);
+    {
+        const int r = u0 - smem_cum[lo];
+        cur.kvh = r / cur.nb;
+        cur.blk = r - cur.kvh * cur.nb;
+        cur.tile = 0;
+    }
+    const int ntiles = (u1 - u0) * kTiles;
+
+    auto tile_ptr = [&](const UnitCursor& u, bool& valid) -> const uint16_t* {
+        const int page = a.block_table[(long long)u.b * a.max_blocks + u.blk];
+        valid = page >= 0 && (long long)page < a.num_pages;
+        const long long chunk = ((long long)(valid ? page : 0) * a.Hkv + u.kvh) * P;
+        return a.k_cache + (chunk + u.tile * 16) * D;
+    };
+
+    KTile<D> buf0, buf1;
+    bool v0 = false, v1 = false;
+    {
+        const uint16_t* p0 = tile_ptr(cur, v0);
+        load_k_tile<D>(buf0, p0, grp, tq, v0);
+    }
+    UnitCursor nxt = cur;
+    uint4 qf[KTile<D>::kChunks];
+    int q_b = -1, q_kvh = -1;
+    float xs[kTiles][4];
+
+    // one tile: prefetch the next tile into `nb`, then consume `cb`
+    auto step = [&](const KTile<D>& cbuf, bool cvalid, KTile<D>& nbuf, bool& nvalid, int i) {
+        if (i + 1 < ntiles) {
+            cursor_advance(nxt, a.ctx_lens, P, a.max_blocks, a.Hkv, kTiles);
+            const uint16_t* p = tile_ptr(nxt, nvalid);
+            load_k_tile<D>(nbuf, p, grp, tq, nvalid);
+        }
+        if (cur.b != q_b || cur.kvh != q_kvh) {
+            q_b = cur.b;
+            q_kvh = cur.kvh;
+            const int h = cur.kvh * a.g + grp;
+#pragma unroll
+            for (int c = 0; c < KTile<D>::kChunks; ++c)
+                qf[c] = grp < a.g ? __ldg(reinterpret_cast<const uint4*>(
+                                        a.q + ((long long)cur.b * a.Hq + h) * D + 32 * c + 8 * tq))
+                                  : make_uint4(0, 0, 0, 0);
+        }
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < KTile<D>::kChunks; ++c) {
+            mma_bf16_16x8x16(acc, cbuf.lo[c].x, cbuf.hi[c].x, cbuf.lo[c].y, cbuf.hi[c].y, qf[c].x, qf[c].y);
+            mma_bf16_16x8x16(acc, cbuf.lo[c].z, cbuf.hi[c].z, cbuf.lo[c].w, cbuf.hi[c].w, qf[c].z, qf[c].w);
+        }
+        // token slots grp, grp+8 of this tile; heads 2tq, 2tq+1
+        const int L = a.ctx_lens[cur.b];
+        const int valid_tok = min(P, L - cur.blk * P) - cur.tile * 16;
+        float x4[4];
+        x4[0] = (cvalid && grp < valid_tok) ? acc[0] * a.scale : -kInf;
+        x4[1] = (cvalid && grp < valid_tok) ? acc[1] * a.scale : -kInf;
+        x4[2] = (cvalid && grp + 8 < valid_tok) ? acc[2] * a.scale : -kInf;
+        x4[3] = (cvalid && grp + 8 < valid_tok) ? acc[3] * a.scale : -kInf;
+#pragma unroll
+        for (int tt = 0; tt < kTiles; ++tt)      // static indices keep xs in registers
+            if (tt == cur.tile)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) xs[tt][e] = x4[e];
+        const long long unit = ((long long)cur.b * a.Hkv + cur.kvh) * a.max_blocks + cur.blk;
+        if (a.token_scores) {
+            float* ts = a.token_scores + (unit * P + cur.tile * 16) * a.g;
+            const int h0 = 2 * tq, h1 = 2 * tq + 1;
+            if (h0 < a.g) {
+                ts[grp * a.g + h0] = x4[0];
+                ts[(grp + 8) * a.g + h0] = x4[2];
+            }
+            if (h1 < a.g) {
+                ts[grp * a.g + h1] = x4[1];
+                ts[(grp + 8) * a.g + h1] = x4[3];
+            }
+        }
+        if (cur.tile == kTiles - 1) {
+            // block stats for heads 2tq (j = 0) and 2tq + 1 (j = 1)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                float m = -kInf;
+#pragma unroll
+                for (int tt = 0; tt < kTiles; ++tt) m = fmaxf(m, fmaxf(xs[tt][j], xs[tt][j + 2]));
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 4));
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 8));
+                m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 16));
+                // l1 = (sum e^{x-m}) - 1, kept exact: the tokens below the max are
+                // summed and every further token AT the max adds exactly 1, so a
+                // block dominated by one token keeps its small remainder.
+                float l1 = 0.f, u = 0.f, neq = 0.f;
+                if (m != -kInf) {
+#pragma unroll
+                    for (int tt = 0; tt < kTiles; ++tt) {
+#pragma unroll
+                        for (int e = 0; e < 2; ++e) {
+                            const float d = xs[tt][j + 2 * e] - m;
+                            const float w = fast_ex2(d * kLog2e);
+                            l1 += d < 0.f ? w : 0.f;
+                            neq += d == 0.f ? 1.f : 0.f;
+                            u = fmaf(w, fmaxf(d, -1e30f), u);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int o = 4; o <= 16; o <<= 1) {
+                    l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+                    u += __shfl_xor_sync(0xffffffffu, u, o);
+                    neq += __shfl_xor_sync(0xffffffffu, neq, o);
+                }
+                l1 += neq - 1.f;
+                const int h = 2 * tq + j;
+                if (grp == 0 && h < a.g) a.stats[unit * a.g + h] = make_float4(m, l1, u, 0.f);
+            }
+        }
+        cur = nxt;
+    };
+
+    for (int i = 0; i < ntiles; i += 2) {
+        step(buf0, v0, buf1, v1, i);
+        if (i + 1 < ntiles) step(buf1, v1, buf0, v0, i + 1);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// prune_finalize
+
+struct FinArgs {
+    const float4* stats;
+    const int32_t* ctx_lens;
+    const int32_t* block_table;
+    long long num_pages;
+    int B, Hq, Hkv, g, P, max_blocks;
+    // rule mode (given == 0)
+    const float* theta;
+    int B_min;
+    // given mode: keep set from a list or a mask (or every block)
+    int given;
+    const uint8_t* given_mask;
+    const int32_t* given_idx;
+    const int32_t* given_cnt;
+    // outputs
+    uint8_t* keep_mask;     // nullable
+    int32_t* kept_idx;
+    int32_t* kept_cnt;
+    float* block_score;     // nullable
+    float* kept_norm;       // nullable: [B][Hq][2]
+    uint32_t* err;          // nullable
+};
+
+template <int N>
+__device__ __forceinline__ void block_reduce_max(float (&v)[N], float* red) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int k = 0; k < N; ++k) v[k] = warp_max(v[k]);
+    if (lane == 0)
+        for (int k = 0; k < N; ++k) red[w * N + k] = v[k];
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < N; ++k) {
+        float r = -kInf;
+        for (int i = 0; i < nw; ++i) r = fmaxf(r, red[i * N + k]);
+        v[k] = r;
+    }
+    __syncthreads();
+}
+
+template <int N>
+__device__ __forceinline__ void block_reduce_sum(float (&v)[N], float* red) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int k = 0; k < N; ++k) v[k] = warp_sum(v[k]);
+    if (lane == 0)
+        for (int k = 0; k < N; ++k) red[w * N + k] = v[k];
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < N; ++k) {
+        float r = 0.f;
+        for (int i = 0; i < nw; ++i) r += red[i * N + k];
+        v[k] = r;
+    }
+    __syncthreads();
+}
+
+// exclusive block scan of one int per thread; returns the total in *tot
+__device__ __forceinline__ int block_excl_scan(int v, int* red, int* tot) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int x = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, x, o);
+        if (lane >= o) x += y;
+    }
+    if (lane == 31) red[w] = x;
+    __syncthreads();
+    int ofs = 0, t = 0;
+    for (int i = 0; i < nw; ++i) {
+        if (i < w) ofs += red[i];
+        t += red[i];
+    }
+    __syncthreads();
+    *tot = t;
+    return ofs + x - v;
+}
+
+__device__ __forceinline__ uint32_t order_key(float f) {
+    if (f != f) return 0u;
+    const uint32_t b = __float_as_uint(f);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+template <int G>
+__global__ void __launch_bounds__(kFinThreads)
+prune_finalize_kernel(const FinArgs a) {
+    extern __shared__ float sh_score[];          // [max_blocks] scores, then flags
+    __shared__ float red[(kFinThreads / 32) * 16];
+    __shared__ int ired[kFinThreads / 32];
+    __shared__ int hist[256];
+    __shared__ int sel_digit, sel_rem;
+    const int seg = blockIdx.x;
+    const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
+    const int tid = threadIdx.x, nt = blockDim.x;
+    const int L = a.ctx_lens[b];
+    const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
+    const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
+    const long long segbase = (long long)seg * a.max_blocks;
+
+    // page ids of the sequence
+    int bad = 0;
+    for (int j = tid; j < nb; j += nt) {
+        const int pg = a.block_table[(long long)b * a.max_blocks + j];
+        bad |= (pg < 0 || (long long)pg >= a.num_pages);
+    }
+    const bool bad_page = __syncthreads_or(bad) != 0;
+    if (a.err && kvh == 0 && tid == 0)
+        a.err[b] = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page && !bad_ctx ? ETI_ERRF_BAD_PAGE : 0u);
+    const int n = (bad_ctx || bad_page) ? 0 : nb;
+    const int per = (n + nt - 1) / nt;          // contiguous block range per thread
+    const int j0 = min(tid * per, n), j1 = min(j0 + per, n);
+    const float4* st = a.stats + segbase * G;
+
+    float M[G], Z[G];
+    if (n > 0) {
+#pragma unroll
+        for (int h = 0; h < G; ++h) M[h] = -kInf;
+        for (int j = j0; j < j1; ++j)
+#pragma unroll
+            for (int h = 0; h < G; ++h) M[h] = fmaxf(M[h], st[j * G + h].x);
+        block_reduce_max<G>(M, red);
+    }
+
+    if (!a.given) {
+        if (n > 0) {
+#pragma unroll
+            // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
+            // c_b = e^{m_b - M}: exact around Z ~ 1, so log Z = log1p(Z - 1) keeps
+            // its relative precision when one token takes nearly all attention.
+            float Zs[2 * G];   // [h]: the part below 1; [G + h]: number of top blocks
+#pragma unroll
+            for (int h = 0; h < 2 * G; ++h) Zs[h] = 0.f;
+            for (int j = j0; j < j1; ++j)
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    const float4 s = st[j * G + h];
+                    const float cb = expf(s.x - M[h]);
+                    Zs[h] += cb * s.y + (s.x < M[h] ? cb : 0.f);
+                    Zs[G + h] += s.x < M[h] ? 0.f : 1.f;
+                }
+            block_reduce_sum<2 * G>(Zs, red);
+            float lZ[G], Hs[G];
+#pragma unroll
+            for (int h = 0; h < G; ++h) {
+                const float zm1 = Zs[h] + (Zs[G + h] - 1.f);
+                lZ[h] = log1pf(zm1);
+                Z[h] = 1.f + zm1;
+                Hs[h] = 0.f;
+            }
+            // I_b per head; sum = attention entropy of the head
+            for (int j = j0; j < j1; ++j)
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    const float4 s = st[j * G + h];
+                    const float I = expf(s.x - M[h]) * ((1.f + s.y) * (lZ[h] + M[h] - s.x) - s.z) / Z[h];
+                    Hs[h] += I;
+                }
+            block_reduce_sum<G>(Hs, red);
+            for (int j = j0; j < j1; ++j) {
+                float best = -kInf;
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    const float4 s = st[j * G + h];
+                    const float I = expf(s.x - M[h]) * ((1.f + s.y) * (lZ[h] + M[h] - s.x) - s.z) / Z[h];
+                    const float nrm = Hs[h] > 0.f ? (float)n * I / Hs[h] : 1.f;
+                    best = fmaxf(best, nrm);
+                }
+                sh_score[j] = best;
+            }
+        }
+        __syncthreads();
+        if (a.block_score) {
+            for (int j = tid; j < a.max_blocks; j += nt)
+                a.block_score[segbase + j] = j < n ? sh_score[j] : 0.f;
+        }
+        // B_min budget: the first k blocks by (score desc, index asc)
+        const int k = min(max(a.B_min, 0), n);
+        uint32_t kth = 0xffffffffu;   // keys > kth are selected; `rem` of those == kth
+        int rem = 0;
+        int arg = -1;                 // B_min == 1: the first block of highest score
+        if (k == n && n > 0) {
+            kth = 0u; rem = 0;        // every block
+        } else if (k == 1) {
+            float bs = -kInf;
+            int bj = 0x7fffffff;
+            for (int j = j0; j < j1; ++j) {
+                const float v = sh_score[j];
+                if (v > bs || (bj == 0x7fffffff)) { bs = v; bj = j; }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float ov = __shfl_xor_sync(0xffffffffu, bs, o);
+                const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+                if (ov > bs || (ov == bs && oj < bj)) { bs = ov; bj = oj; }
+            }
+            if ((tid & 31) == 0) { red[tid >> 5] = bs; ired[tid >> 5] = bj; }
+            __syncthreads();
+            if (tid == 0) {
+                for (int w = 1; w < nt / 32; ++w)
+                    if (red[w] > bs || (red[w] == bs && ired[w] < bj)) { bs = red[w]; bj = ired[w]; }
+                sel_digit = bj;
+            }
+            __syncthreads();
+            arg = sel_digit;
+            __syncthreads();
+        } else if (k > 0) {
+            uint32_t prefix = 0, mask = 0;
+            int need = k;
+            for (int digit = 3; digit >= 0; --digit) {
+                const int sh = digit * 8;
+                for (int i = tid; i < 256; i += nt) hist[i] = 0;
+                __syncthreads();
+                for (int j = j0; j < j1; ++j) {
+                    const uint32_t key = order_key(sh_score[j]);
+                    if ((key & mask) == prefix) atomicAdd(&hist[(key >> sh) & 255], 1);
+                }
+                __syncthreads();
+                // bucket where the count from the top reaches `need`
+                if (tid < 32) {
+                    int cnt8[8], s8 = 0;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) { cnt8[e] = hist[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
+                    int incl = s8;
+#pragma unroll
+                    for (int o = 1; o < 32; o <<= 1) {
+                        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                        if (tid >= o) incl += y;
+                    }
+                    int above = incl - s8;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        if (above < need && need <= above + cnt8[e]) {
+                            sel_digit = 255 - (tid * 8 + e);
+                            sel_rem = need - above;
+                        }
+                        above += cnt8[e];
+                    }
+                }
+                __syncthreads();
+                prefix |= (uint32_t)sel_digit << sh;
+                mask |= 255u << sh;
+                need = sel_rem;
+                __syncthreads();
+            }
+            kth = prefix;
+            rem = need;
+        }
+        // flags: threshold or budget (ties at the k-th key go to the lower index)
+        const float th = a.theta[b];
+        int eq = 0;
+        for (int j = j0; j < j1; ++j) eq += (k > 1 && k < n && order_key(sh_score[j]) == kth);
+        int eq_tot;
+        int eq_rank = block_excl_scan(eq, ired, &eq_tot);
+        for (int j = j0; j < j1; ++j) {
+            const float s = sh_score[j];
+            const uint32_t key = order_key(s);
+            bool keep = s >= th;
+            if (k == n) keep = true;
+            else if (k == 1) keep |= (j == arg);
+            else if (k > 1) {
+                if (key > kth) keep = true;
+                else if (key == kth) { keep |= eq_rank < rem; ++eq_rank; }
+            }
+            sh_score[j] = keep ? 1.f : 0.f;   // scores are no longer needed
+        }
+        __syncthreads();
+    } else {
+        // given keep set
+        for (int j = j0; j < j1; ++j) sh_score[j] = 0.f;
+        __syncthreads();
+        if (a.given_idx) {
+            const int c = min(max(a.given_cnt[seg], 0), a.max_blocks);
+            for (int i = tid; i < c; i += nt) {
+                const int j = a.given_idx[segbase + i];
+                if (j >= 0 && j < n) sh_score[j] = 1.f;
+            }
+        } else {
+            for (int j = j0; j < j1; ++j) sh_score[j] = a.given_mask ? (a.given_mask[segbase + j] ? 1.f : 0.f) : 1.f;
+        }
+        __syncthreads();
+    }
+
+    // compaction (ascending block index)
+    int cnt = 0;
+    for (int j = j0; j < j1; ++j) cnt += sh_score[j] != 0.f;
+    int total;
+    int pos = block_excl_scan(cnt, ired, &total);
+    for (int j = j0; j < j1; ++j)
+        if (sh_score[j] != 0.f) a.kept_idx[segbase + pos++] = j;
+    for (int i = total + tid; i < a.max_blocks; i += nt) a.kept_idx[segbase + i] = -1;
+    if (a.keep_mask)
+        for (int j = tid; j < a.max_blocks; j += nt)
+            a.keep_mask[segbase + j] = (j < n && sh_score[j] != 0.f) ? 1 : 0;
+    if (tid == 0) a.kept_cnt[seg] = total;
+
+    // softmax normaliser over the kept tokens of each query head
+    if (a.kept_norm) {
+        float Mk[G], Lk[G];
+#pragma unroll
+        for (int h = 0; h < G; ++h) Mk[h] = -kInf;
+        for (int j = j0; j < j1; ++j)
+            if (sh_score[j] != 0.f)
+#pragma unroll
+                for (int h = 0; h < G; ++h) Mk[h] = fmaxf(Mk[h], st[j * G + h].x);
+        block_reduce_max<G>(Mk, red);
+#pragma unroll
+        for (int h = 0; h < G; ++h) Lk[h] = 0.f;
+        for (int j = j0; j < j1; ++j)
+            if (sh_score[j] != 0.f)
+#pragma unroll
+                for (int h = 0; h < G; ++h) {
+                    const float4 s = st[j * G + h];
+                    Lk[h] += (1.f + s.y) * expf(s.x - Mk[h]);
+                }
+        block_reduce_sum<G>(Lk, red);
+        if (tid < a.g) {
+            float mm = 0.f, ll = 0.f;
+#pragma unroll
+            for (int h = 0; h < G; ++h)
+                if (h == tid) { mm = Mk[h]; ll = Lk[h]; }
+            float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + tid) * 2;
+            kn[0] = mm;
+            kn[1] = ll;
+        }
+    }
+}
+
+}  // namespace eti
+
+using namespace eti;
+
+int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const int32_t* block_table,
+                            const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
+                            int max_blocks, long long num_pages, float scale, float* token_scores,
+                            float4* stats, cudaStream_t stream) {
+    if (B == 0) return ETI_OK;
+    ScoreArgs a;
+    a.q = q; a.k_cache = k_cache; a.block_table = block_table; a.ctx_lens = ctx_lens;
+    a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.g = Hq / Hkv; a.max_blocks = max_blocks;
+    a.num_pages = num_pages; a.scale = scale; a.token_scores = token_scores; a.stats = stats;
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int grid = 2 * sms;
+    const size_t smem = (size_t)(B + 1) * sizeof(int);
+    cudaError_t e;
+#define ETI_SCORE_CASE(DD, PP)                                                              \
+    if (D == DD && P == PP) {                                                               \
+        auto k = score_blocks_kernel<DD, PP>;                                               \
+        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        k<<<grid, kScoreThreads, smem, stream>>>(a);                                        \
+        e = cudaGetLastError();                                                             \
+        return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;                                    \
+    }
+    ETI_SCORE_CASE(128, 16)
+    ETI_SCORE_CASE(128, 32)
+    ETI_SCORE_CASE(64, 16)
+    ETI_SCORE_CASE(64, 32)
+#undef ETI_SCORE_CASE
+    return ETI_ERR_UNSUPPORTED;
+}
+
+int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, const int32_t* block_table,
+                              long long num_pages, int B, int Hq, int Hkv, int P, int max_blocks,
+                              const float* theta, int B_min, int given, const uint8_t* given_mask,
+                              const int32_t* given_idx, const int32_t* given_cnt, uint8_t* keep_mask,
+                              int32_t* kept_idx, int32_t* kept_cnt, float* block_score,
+                              float* kept_norm, uint32_t* err, cudaStream_t stream) {
+    if (B == 0) return ETI_OK;
+    FinArgs a;
+    a.stats = stats; a.ctx_lens = ctx_lens; a.block_table = block_table; a.num_pages = num_pages;
+    a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.g = Hq / Hkv; a.P = P; a.max_blocks = max_blocks;
+    a.theta = theta; a.B_min = B_min; a.given = given; a.given_mask = given_mask;
+    a.given_idx = given_idx; a.given_cnt = given_cnt; a.keep_mask = keep_mask;
+    a.kept_idx = kept_idx; a.kept_cnt = kept_cnt; a.block_score = block_score;
+    a.kept_norm = kept_norm; a.err = err;
+    const size_t smem = (size_t)max_blocks * sizeof(float);
+    const int grid = B * Hkv;
+    cudaError_t e = cudaSuccess;
+#define ETI_FIN_CASE(GG)                                                                    \
+    case GG: {                                                                              \
+        auto k = prune_finalize_kernel<GG>;                                                 \
+        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        k<<<grid, kFinThreads, smem, stream>>>(a);                                          \
+        e = cudaGetLastError();                                                             \
+        break;                                                                              \
+    }
+    switch (a.g) {
+        ETI_FIN_CASE(1)
+        ETI_FIN_CASE(2)
+        ETI_FIN_CASE(3)
+        ETI_FIN_CASE(4)
+        ETI_FIN_CASE(5)
+        ETI_FIN_CASE(6)
+        ETI_FIN_CASE(7)
+        ETI_FIN_CASE(8)
+        default: return ETI_ERR_UNSUPPORTED;
+    }
+#undef ETI_FIN_CASE
+    return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
+}

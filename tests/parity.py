@@ -1,0 +1,157 @@
+"""Shared comparison logic for the GPU-vs-oracle parity tests.
+
+Tolerances (stated here once, used by every parity test):
+  * entropy H: 1e-4 relative, or 1e-6 nats absolute when H < 1e-2;
+  * temperature T_out, entropy flow dH, tau: 1e-4 relative (dH and tau also
+    1e-5 absolute, since dH can cancel to ~0);
+  * theta_next: 2e-4 absolute (it is 1 - H / log V, an O(1) quantity whose
+    error is the H error divided by log V);
+  * surprisal: 1e-4 relative or 1e-5 absolute;
+  * sampled token: exact, unless the oracle's Gumbel-max key of the GPU's
+    token is within 1e-5 of the best key (counted as a tie and reported);
+  * keep mask / kept lists: exact, unless the oracle's block score is within
+    1e-5 * max(1, theta) of theta, or within 1e-5 * max(1, s_k) of the k-th
+    best score at the B_min boundary (counted as ties);
+  * attention output (bf16 from fp32 accumulation over bf16 K/V): 2e-2
+    absolute.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+import workloads
+
+H_REL, H_ABS_SMALL = 1e-4, 1e-6
+KEY_TIE = 1e-5
+MASK_TIE = 1e-5
+ATTN_ABS = 2e-2
+
+
+def run_ets(eti, lg: dict, params=None, seed=0, offset=0, V=None):
+    """Run eti_entropy_temp_sample on the workload's logits; numpy results."""
+    B = lg["logits"].shape[0]
+    dev = lg["logits"].device
+    f32, i32 = torch.float32, torch.int32
+    tau = lg["tau"].clone()
+    out = dict(tok=torch.empty(B, dtype=i32, device=dev), H=torch.empty(B, dtype=f32, device=dev),
+               T_out=torch.empty(B, dtype=f32, device=dev), dH=torch.empty(B, dtype=f32, device=dev),
+               theta_next=torch.empty(B, dtype=f32, device=dev),
+               surprisal=torch.empty(B, dtype=f32, device=dev),
+               err=torch.empty(B, dtype=i32, device=dev))
+    eti.eti_entropy_temp_sample(lg["logits"], lg["T_in"], lg["H_prev"], tau, lg["H_target"],
+                                out["tok"], out["H"], out["T_out"], out["err"], params=params,
+                                seed=seed, offset=offset, dH=out["dH"],
+                                theta_next=out["theta_next"], tok_surprisal=out["surprisal"], V=V)
+    torch.cuda.synchronize()
+    res = {k: v.cpu().numpy() for k, v in out.items()}
+    res["tau"] = tau.cpu().numpy()
+    res["err"] = res["err"].view(np.uint32)
+    return res
+
+
+def oracle_ets(lg: dict, ctrl=None, seed=0, offset=0, V=None):
+    return oracle.entropy_temp_sample(lg["logits"].cpu().numpy(), lg["T_in"].cpu().numpy(),
+                                      lg["H_prev"].cpu().numpy(), lg["tau"].cpu().numpy(),
+                                      lg["H_target"].cpu().numpy(), ctrl, seed=seed, offset=offset,
+                                      V=V)
+
+
+def _close(a, b, rel, abs_=0.0):
+    a = np.asarray(a, np.float64)
+    b = np.asarray(b, np.float64)
+    return np.abs(a - b) <= np.maximum(rel * np.abs(b), abs_)
+
+
+def compare_ets(gpu: dict, ref: dict, lg: dict, seed=0, offset=0, V=None) -> dict:
+    """Assert parity of every output of the entropy/sample call; return tie stats."""
+    ok_rows = ref["err"] == 0
+    assert np.array_equal(gpu["err"], ref["err"]), (gpu["err"], ref["err"])
+    bad = ~ok_rows
+    assert (gpu["tok"][bad] == -1).all() and np.isnan(gpu["H"][bad]).all()
+    Hr, Hg = ref["H"][ok_rows], gpu["H"][ok_rows].astype(np.float64)
+    small = Hr < 1e-2
+    okH = np.where(small, np.abs(Hg - Hr) <= H_ABS_SMALL, np.abs(Hg - Hr) <= H_REL * Hr)
+    assert okH.all(), f"H mismatch: worst rel {np.max(np.abs(Hg - Hr) / np.maximum(Hr, 1e-12))}"
+    assert _close(gpu["T_out"][ok_rows], ref["T_out"][ok_rows], 1e-4).all()
+    assert _close(gpu["dH"][ok_rows], ref["dH"][ok_rows], 1e-4, 1e-5).all()
+    assert _close(gpu["tau"][ok_rows], ref["tau"][ok_rows], 1e-4, 1e-5).all()
+    assert _close(gpu["theta_next"][ok_rows], ref["theta_next"][ok_rows], 0.0, 2e-4).all()
+    assert (gpu["tau"][bad] == lg["tau"].cpu().numpy()[bad]).all()
+    # sampled tokens: exact except Gumbel near-ties
+    z = lg["logits"].cpu().numpy()
+    T = lg["T_in"].cpu().numpy()
+    ties, worst = 0, 0.0
+    for b in np.nonzero(ok_rows)[0]:
+        if gpu["tok"][b] == ref["tok"][b]:
+            continue
+        Vb = z.shape[1] if V is None else V
+        kg = oracle.sample_key(z[b, :Vb], float(T[b]), seed, offset, int(b), int(gpu["tok"][b]))
+        kb = oracle.sample_key(z[b, :Vb], float(T[b]), seed, offset, int(b), int(ref["tok"][b]))
+        gap = kb - kg
+        worst = max(worst, gap)
+        assert gap < KEY_TIE, f"row {b}: GPU token {gpu['tok'][b]} vs oracle {ref['tok'][b]}, key gap {gap}"
+        ties += 1
+    sr, sg = ref["surprisal"][ok_rows], gpu["surprisal"][ok_rows]
+    same = gpu["tok"][ok_rows] == ref["tok"][ok_rows]
+    assert _close(sg[same], sr[same], 1e-4, 1e-5).all()
+    return dict(rows=int(ok_rows.sum()), token_ties=ties, worst_tie_gap=worst)
+
+
+# ---------------------------------------------------------------------------
+def host_kv(kv: dict) -> dict:
+    return dict(q=workloads.bf16_bits(kv["q"]), k=workloads.bf16_bits(kv["k_cache"]),
+                v=workloads.bf16_bits(kv["v_cache"]), bt=kv["block_table"].cpu().numpy(),
+                L=kv["ctx_lens"].cpu().numpy(), scale=kv["scale"], num_pages=kv["num_pages"])
+
+
+def compare_masks(gpu_mask, gpu_idx, gpu_cnt, ref: dict, theta, B_min, P, L) -> dict:
+    """Keep sets equal except for near-threshold / near-budget-boundary ties."""
+    B, Hkv, mb = ref["keep_mask"].shape
+    ties = 0
+    for b in range(B):
+        n = -(-int(L[b]) // P) if L[b] > 0 else 0
+        th = float(theta[b])
+        for h in range(Hkv):
+            gm, rm = gpu_mask[b, h, :n].astype(bool), ref["keep_mask"][b, h, :n].astype(bool)
+            assert not gpu_mask[b, h, n:].any()
+            c = int(gpu_cnt[b, h])
+            assert c == int(gm.sum())
+            assert np.array_equal(gpu_idx[b, h, :c], np.nonzero(gm)[0])
+            assert (gpu_idx[b, h, c:] == -1).all()
+            diff = np.nonzero(gm != rm)[0]
+            if len(diff) == 0:
+                continue
+            s = ref["block_score"][b, h, :n]
+            k = min(max(B_min, 0), n)
+            sk = np.sort(s)[::-1][k - 1] if 0 < k < n else None
+            for j in diff:
+                near_th = abs(s[j] - th) <= MASK_TIE * max(1.0, abs(th)) if np.isfinite(th) else False
+                near_k = sk is not None and abs(s[j] - sk) <= MASK_TIE * max(1.0, abs(sk))
+                assert near_th or near_k, (f"seq {b} kvh {h} block {j}: gpu {gm[j]} oracle {rm[j]} "
+                                           f"score {s[j]} theta {th} s_k {sk}")
+                ties += 1
+    return dict(mask_ties=ties)
+
+
+def compare_scores(gpu_score, ref_score, P, L):
+    """Block scores (normalised Ibar) within 1e-4 relative (reported, for the tie analysis)."""
+    B, Hkv, mb = ref_score.shape
+    worst = 0.0
+    for b in range(B):
+        n = -(-int(L[b]) // P) if L[b] > 0 else 0
+        g, r = gpu_score[b, :, :n].astype(np.float64), ref_score[b, :, :n]
+        if n:
+            worst = max(worst, float(np.max(np.abs(g - r) / np.maximum(1.0, np.abs(r)))))
+    assert worst < 1e-4, worst
+    return worst
+
+
+def compare_attention(gpu_out, ref_out, rows=None):
+    g = gpu_out.astype(np.float64)
+    err = np.abs(g - ref_out)
+    assert np.isfinite(g).all()
+    worst = float(err.max()) if err.size else 0.0
+    assert worst < ATTN_ABS, worst
+    return worst

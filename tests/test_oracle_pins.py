@@ -110,6 +110,13 @@ def test_nonfinite_rows_flag_errors():
     assert (r["tau"] == 2.0).all() and (r["T_out"] == 1.0).all() and (r["theta_next"] == 0.0).all()
 
 
+def test_bad_temperature_flags_error():
+    z = np.zeros((3, 8), np.float32)
+    for T in (0.0, -1.0, np.inf):
+        r = _ets(z, T=T)
+        assert (r["err"] == oracle.ERR_BAD_TEMP).all() and (r["tok"] == -1).all()
+
+
 # ----------------------------------------------------------------------------
 # Entropy flow and entropic time (Section 2)
 

@@ -115,7 +115,7 @@ def make_logits(w: Workload, device="cpu", ld: int | None = None) -> dict:
         if w.even_row_spike is not None and b % 2 == 0:
             z[b, int(rng.integers(0, V))] += w.even_row_spike
         else:
-            n = int(rng.integers(0, 4))
+            n = min(int(rng.integers(0, 4)), V)
             for x in rng.choice(V, size=n, replace=False):
                 z[b, int(x)] += w.spike
     logV = math.log(V)
