@@ -75,7 +75,7 @@ def _load():
             lib.oracle_entropy_temp_sample.argtypes = (
                 [P, i32, i64, i64, P, P, P, P, P, u64, u64] + [P] * 9)
             lib.oracle_score_prune.argtypes = (
-                [P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, i32] + [P] * 7)
+                [P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, i32] + [P] * 8)
             lib.oracle_paged_attention.argtypes = (
                 [P, P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, P, P])
             _lib = lib
@@ -184,14 +184,17 @@ def score_prune(q, k_cache, block_table, ctx_lens, scale: float, theta, B_min: i
     kcnt = np.empty((B, Hkv), np.int32)
     score = np.empty((B, Hkv, mb), np.float64)
     head_I = np.empty((B, Hq, mb), np.float64) if want_heads else None
+    head_A = np.empty((B, Hq, mb), np.float64) if want_heads else None
     head_H = np.empty((B, Hq), np.float64) if want_heads else None
     err = np.empty(B, np.uint32)
     lib.oracle_score_prune(_ptr(q), _ptr(k_cache), _ptr(bt), _ptr(cl), B, Hq, Hkv, D, P, mb,
                            num_pages, float(scale), _ptr(th), int(B_min), _ptr(keep), _ptr(kidx),
-                           _ptr(kcnt), _ptr(score), _ptr(head_I), _ptr(head_H), _ptr(err))
+                           _ptr(kcnt), _ptr(score), _ptr(head_I), _ptr(head_A), _ptr(head_H),
+                           _ptr(err))
     res = dict(keep_mask=keep, kept_idx=kidx, kept_cnt=kcnt, block_score=score, err=err)
     if want_heads:
         res["head_I"] = head_I
+        res["head_A"] = head_A
         res["head_H"] = head_H
     return res
 

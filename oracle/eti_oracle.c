@@ -293,8 +293,9 @@ static int rank_cmp(const void *pa, const void *pb) {
  *
  * Outputs: keep_mask [B][Hkv][max_blocks] (0/1), kept_idx [B][Hkv][max_blocks]
  * (ascending, -1 padded), kept_cnt [B][Hkv], block_score [B][Hkv][max_blocks]
- * (Ibar, 0 padded), head_I [B][Hq][max_blocks] (raw I_b^(h)) and
- * head_H [B][Hq] (attention entropy) -- the last two may be NULL.
+ * (Ibar, 0 padded), head_I [B][Hq][max_blocks] (raw I_b^(h)),
+ * head_A [B][Hq][max_blocks] (block attention mass sum_{i in block} a_i) and
+ * head_H [B][Hq] (attention entropy) -- the last three may be NULL.
  * A sequence with a bad page id or context length keeps nothing.
  */
 void oracle_score_prune(const uint16_t *q, const uint16_t *k_cache, const int32_t *block_table,
@@ -302,7 +303,8 @@ void oracle_score_prune(const uint16_t *q, const uint16_t *k_cache, const int32_
                         int max_blocks, int64_t num_pages, double scale,
                         const float *theta, int B_min,
                         uint8_t *keep_mask, int32_t *kept_idx, int32_t *kept_cnt,
-                        double *block_score, double *head_I, double *head_H, uint32_t *err) {
+                        double *block_score, double *head_I, double *head_A, double *head_H,
+                        uint32_t *err) {
     const int g = Hq / Hkv;
     for (int b = 0; b < B; ++b) err[b] = seq_check(block_table, ctx_lens, b, P, max_blocks, num_pages);
 #pragma omp parallel for collapse(2) schedule(dynamic, 1)
@@ -314,14 +316,19 @@ void oracle_score_prune(const uint16_t *q, const uint16_t *k_cache, const int32_
             double *bs = block_score + seg * max_blocks;
             for (int j = 0; j < max_blocks; ++j) { km[j] = 0; ki[j] = -1; bs[j] = 0.0; }
             kept_cnt[seg] = 0;
-            if (head_I) for (int hh = 0; hh < g; ++hh)
-                for (int j = 0; j < max_blocks; ++j) head_I[((int64_t)b * Hq + kvh * g + hh) * max_blocks + j] = 0.0;
+            for (int hh = 0; hh < g; ++hh)
+                for (int j = 0; j < max_blocks; ++j) {
+                    int64_t o = ((int64_t)b * Hq + kvh * g + hh) * max_blocks + j;
+                    if (head_I) head_I[o] = 0.0;
+                    if (head_A) head_A[o] = 0.0;
+                }
             if (head_H) for (int hh = 0; hh < g; ++hh) head_H[(int64_t)b * Hq + kvh * g + hh] = 0.0;
             int L = ctx_lens[b];
             if (err[b] || L == 0) continue;
             int nb = (L + P - 1) / P;
             double *x = (double *)malloc(sizeof(double) * (size_t)L);
             double *Ih = (double *)malloc(sizeof(double) * (size_t)nb);
+            double *Ah = (double *)malloc(sizeof(double) * (size_t)nb);
             double *score = (double *)malloc(sizeof(double) * (size_t)nb);
             for (int j = 0; j < nb; ++j) score[j] = -INFINITY;
             for (int hh = 0; hh < g; ++hh) {
@@ -333,19 +340,22 @@ void oracle_score_prune(const uint16_t *q, const uint16_t *k_cache, const int32_
                 for (int i = 0; i < L; ++i) Z += exp(x[i] - M);
                 double total = 0.0;
                 for (int j = 0; j < nb; ++j) {
-                    double s = 0.0;
+                    double s = 0.0, mass = 0.0;
                     int i1 = (j + 1) * P < L ? (j + 1) * P : L;
                     for (int i = j * P; i < i1; ++i) {
                         double a = exp(x[i] - M) / Z;
+                        mass += a;
                         if (a > 0.0) s += a * (-log(a));
                     }
                     Ih[j] = s;
+                    Ah[j] = mass;
                     total += s;
                 }
                 for (int j = 0; j < nb; ++j) {
                     double nrm = total > 0.0 ? (double)nb * Ih[j] / total : 1.0;
                     if (nrm > score[j]) score[j] = nrm;
                     if (head_I) head_I[((int64_t)b * Hq + h) * max_blocks + j] = Ih[j];
+                    if (head_A) head_A[((int64_t)b * Hq + h) * max_blocks + j] = Ah[j];
                 }
                 if (head_H) head_H[(int64_t)b * Hq + h] = total;
             }
@@ -368,7 +378,7 @@ void oracle_score_prune(const uint16_t *q, const uint16_t *k_cache, const int32_
                 if (keep) ki[cnt++] = j;
             }
             kept_cnt[seg] = cnt;
-            free(taken); free(score); free(Ih); free(x);
+            free(taken); free(score); free(Ah); free(Ih); free(x);
         }
     }
 }

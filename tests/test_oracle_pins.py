@@ -376,6 +376,12 @@ def test_block_scores_sum_to_attention_entropy():
             Ha = stats.entropy(torch.softmax(x, 0).numpy())
             assert abs(r["head_H"][b, h] - Ha) < 1e-10
             assert abs(r["head_I"][b, h].sum() - Ha) < 1e-10
+            # block masses partition the attention: they add to 1 and match torch
+            a = torch.softmax(x, 0).numpy()
+            nb = -(-int(n["L"][b]) // w.P)
+            mass = [a[j * w.P:(j + 1) * w.P].sum() for j in range(nb)]
+            assert np.allclose(r["head_A"][b, h, :nb], mass, atol=1e-12)
+            assert abs(r["head_A"][b, h].sum() - 1.0) < 1e-12
 
 
 def test_uniform_attention_closed_form():
