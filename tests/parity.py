@@ -106,9 +106,66 @@ def host_kv(kv: dict) -> dict:
                 L=kv["ctx_lens"].cpu().numpy(), scale=kv["scale"], num_pages=kv["num_pages"])
 
 
-def compare_masks(gpu_mask, gpu_idx, gpu_cnt, ref: dict, theta, B_min, P, L) -> dict:
-    """Keep sets equal except for near-threshold / near-budget-boundary ties."""
+def host_from_gather(sub: dict) -> dict:
+    """workloads.gather_sequences output in the host_kv layout."""
+    return dict(q=sub["q"], k=sub["k_cache"], v=sub["v_cache"], bt=sub["block_table"],
+                L=sub["ctx_lens"], scale=sub["scale"], num_pages=sub["num_pages"])
+
+
+def score_bands(ref: dict, n: dict) -> np.ndarray:
+    """Per (sequence, kv head, block) bound on |Ibar_gpu - Ibar_exact| from fp32 scores.
+
+    The kernel forms x_i = s q.k_i as an fp32 dot product of D bf16 products,
+    error |dx| <= c sqrt(D) 2^-24 s |q| |k_i| with c = 4 (the root-D growth of
+    rounding errors with a margin; the worst-case D 2^-24 bound is far looser).
+    Then |da_i / a_i| <= 2 |dx| and, from I_b = sum a_i (-log a_i) and
+    H = sum_b I_b,  |dIbar_b| / Ibar_b <= 2 |dx| ((I_b + A_b) / I_b + (H + 1) / H),
+    A_b the block's attention mass: the bound is large exactly where one token
+    takes nearly all of a block's attention (I_b << A_b).
+    """
+    q = (n["q"].astype(np.uint32) << 16).view(np.float32)           # [B, Hq, D]
+    k = (n["k"].astype(np.uint32) << 16).view(np.float32)           # [pages, Hkv, P, D]
+    B, Hq, D = q.shape
+    _, Hkv, P, _ = k.shape
+    g = Hq // Hkv
+    mb = n["bt"].shape[1]
+    band = np.zeros((B, Hkv, mb))
+    with np.errstate(invalid="ignore", over="ignore"):
+        knorm = np.sqrt((k.astype(np.float64) ** 2).sum(-1))        # [pages, Hkv, P]
+    for b in range(B):
+        L = int(n["L"][b])
+        nb = -(-L // P) if L > 0 else 0
+        if nb == 0:
+            continue
+        pages = n["bt"][b, :nb]
+        if (pages < 0).any() or (pages >= k.shape[0]).any():
+            continue
+        valid = np.arange(nb * P).reshape(nb, P) < L
+        for kvh in range(Hkv):
+            kn = np.where(valid, knorm[pages, kvh], 0.0).max()
+            qn = np.linalg.norm(q[b, kvh * g:(kvh + 1) * g].astype(np.float64), axis=-1).max()
+            dx = 4.0 * np.sqrt(D) * 2.0 ** -24 * n["scale"] * qn * kn
+            for hh in range(g):
+                h = kvh * g + hh
+                I = ref["head_I"][b, h, :nb]
+                A = ref["head_A"][b, h, :nb]
+                H = ref["head_H"][b, h]
+                if H <= 0:
+                    continue
+                kappa = (I + A) / np.maximum(I, 1e-300) + (H + 1.0) / H
+                nrm = nb * I / H
+                band[b, kvh, :nb] = np.maximum(band[b, kvh, :nb], 2.0 * dx * kappa * nrm)
+    return band
+
+
+def compare_masks(gpu_mask, gpu_idx, gpu_cnt, ref: dict, theta, B_min, P, L, band=None) -> dict:
+    """Keep sets equal except for near-threshold / near-budget-boundary ties.
+
+    A block may differ only if its oracle score is within max(1e-5 max(1, theta),
+    band) of theta, or within max(1e-5 max(1, s_k), band) of the k-th best score
+    s_k at the B_min boundary (band: score_bands, the fp32 evaluation bound)."""
     B, Hkv, mb = ref["keep_mask"].shape
+    band = np.zeros((B, Hkv, mb)) if band is None else band
     ties = 0
     for b in range(B):
         n = -(-int(L[b]) // P) if L[b] > 0 else 0
@@ -125,26 +182,35 @@ def compare_masks(gpu_mask, gpu_idx, gpu_cnt, ref: dict, theta, B_min, P, L) -> 
                 continue
             s = ref["block_score"][b, h, :n]
             k = min(max(B_min, 0), n)
-            sk = np.sort(s)[::-1][k - 1] if 0 < k < n else None
+            order = np.argsort(-s, kind="stable")
+            sk = s[order[k - 1]] if 0 < k < n else None
+            bk = band[b, h, order[k - 1]] if 0 < k < n else 0.0
             for j in diff:
-                near_th = abs(s[j] - th) <= MASK_TIE * max(1.0, abs(th)) if np.isfinite(th) else False
-                near_k = sk is not None and abs(s[j] - sk) <= MASK_TIE * max(1.0, abs(sk))
+                tol = max(MASK_TIE * max(1.0, abs(th)) if np.isfinite(th) else 0.0, band[b, h, j])
+                near_th = np.isfinite(th) and abs(s[j] - th) <= tol
+                near_k = sk is not None and abs(s[j] - sk) <= max(MASK_TIE * max(1.0, abs(sk)),
+                                                                   band[b, h, j] + bk)
                 assert near_th or near_k, (f"seq {b} kvh {h} block {j}: gpu {gm[j]} oracle {rm[j]} "
-                                           f"score {s[j]} theta {th} s_k {sk}")
+                                           f"score {s[j]} theta {th} s_k {sk} band {band[b, h, j]}")
                 ties += 1
     return dict(mask_ties=ties)
 
 
-def compare_scores(gpu_score, ref_score, P, L):
-    """Block scores (normalised Ibar) within 1e-4 relative (reported, for the tie analysis)."""
+def compare_scores(gpu_score, ref_score, P, L, band=None):
+    """Block scores within 2e-5 relative plus the fp32 evaluation band."""
     B, Hkv, mb = ref_score.shape
+    band = np.zeros((B, Hkv, mb)) if band is None else band
     worst = 0.0
     for b in range(B):
         n = -(-int(L[b]) // P) if L[b] > 0 else 0
+        if not n:
+            continue
         g, r = gpu_score[b, :, :n].astype(np.float64), ref_score[b, :, :n]
-        if n:
-            worst = max(worst, float(np.max(np.abs(g - r) / np.maximum(1.0, np.abs(r)))))
-    assert worst < 1e-4, worst
+        err = np.abs(g - r)
+        tol = 2e-5 * np.maximum(1.0, np.abs(r)) + band[b, :, :n]
+        assert (err <= tol).all(), (b, np.unravel_index(np.argmax(err - tol), err.shape),
+                                    float((err - tol).max()))
+        worst = max(worst, float(np.max(err / np.maximum(1.0, np.abs(r)))))
     return worst
 
 

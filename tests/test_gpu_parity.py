@@ -160,13 +160,14 @@ def _check_step(st, n, theta_np, B_min, P, seqs=None):
     """Compare a DecodeStep's keep set and output with the oracle (on `seqs`)."""
     rng = slice(None) if seqs is None else seqs
     ref = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], theta_np, B_min,
-                             num_pages=n.get("num_pages"))
+                             num_pages=n.get("num_pages"), want_heads=True)
+    band = parity.score_bands(ref, n)
     gm = st.keep_mask.cpu().numpy()[rng]
     gi = st.kept_idx.cpu().numpy()[rng]
     gc = st.kept_cnt.cpu().numpy()[rng]
     gs = st.block_score.cpu().numpy()[rng]
-    worst_s = parity.compare_scores(gs, ref["block_score"], P, n["L"])
-    mt = parity.compare_masks(gm, gi, gc, ref, theta_np, B_min, P, n["L"])
+    worst_s = parity.compare_scores(gs, ref["block_score"], P, n["L"], band)
+    mt = parity.compare_masks(gm, gi, gc, ref, theta_np, B_min, P, n["L"], band)
     out_ref, err = oracle.paged_attention(n["q"], n["k"], n["v"], n["bt"], n["L"], n["scale"], gm,
                                           num_pages=n.get("num_pages"))
     worst_o = parity.compare_attention(st.out.float().cpu().numpy()[rng], out_ref)
@@ -302,7 +303,7 @@ def test_attention_full_workloads(eti, name, nsample):
     st = _step(eti, w, kv, theta, B_min)
     rng = np.random.default_rng(w.seed)
     seqs = sorted(rng.choice(w.B, size=min(nsample, w.B), replace=False).tolist())
-    sub = workloads.gather_sequences(kv, seqs)
+    sub = parity.host_from_gather(workloads.gather_sequences(kv, seqs))
     s = _check_step(st, sub, theta.cpu().numpy()[seqs], B_min, w.P, seqs=seqs)
     kept = st.kept_cnt.sum().item()
     total = sum(-(-int(L) // w.P) for L in kv["ctx_lens"].cpu().numpy()) * w.Hkv
@@ -316,7 +317,7 @@ def test_long_context_keep_fraction_sweep(eti):
     kv = workloads.make_kv(w, DEV)
     th = torch.full((w.B,), float("inf"), device=DEV)
     seqs = [0, 2]
-    sub = workloads.gather_sequences(kv, seqs)
+    sub = parity.host_from_gather(workloads.gather_sequences(kv, seqs))
     L = kv["ctx_lens"].cpu().numpy()
     for f in (0.1, 0.5, 1.0):
         # one B_min for the batch: the fraction of the longest sequence
