@@ -35,7 +35,7 @@
  *  - Supported shapes: head_dim D in {64, 128}; page size P in {16, 32};
  *    Hq % Hkv == 0 with group size g = Hq / Hkv <= 8; 1 <= max_blocks <= 32768;
  *    B <= 65535 (entropy/sample) or 8192 (attention calls); 1 <= V.
- *    q, k_cache, v_cache must be 16-byte aligned.
+ *    q, k_cache, v_cache and the decode output must be 16-byte aligned.
  *
  * Layouts
  *  - q          bf16  [B][Hq][D]
@@ -123,7 +123,7 @@ void eti_ctrl_defaults(eti_ctrl_params* p);
  *   tok[b]     = argmax_x y_x - log(-log u_x): a draw from p by the Gumbel-max
  *                rule, u_x from Philox4x32-10 with counter
  *                (x / 4, b, lo32(offset), hi32(offset)), key (lo32(seed),
- *                hi32(seed)), word x mod 4, u = (2 (word >> 9) + 1) / 2^24;
+ *                hi32(seed)), word x mod 4, u = (2 (word & 0x7FFFFF) + 1) / 2^24;
  *                ties go to the lowest token id; -inf logits are never drawn
  *   tok_surprisal[b] = -log p(tok)
  * H, dH, T_out, theta_next, tok_surprisal: fp32 [B]; tok: int32 [B];

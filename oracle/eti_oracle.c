@@ -95,9 +95,9 @@ static uint32_t token_word(uint64_t seed, uint64_t offset, int64_t b, int64_t x)
     return out[x & 3];
 }
 
-/* Uniform in (0,1) from the top 23 bits of the word: u = (2j + 1) / 2^24. */
+/* Uniform in (0,1) from the low 23 bits of the word: u = (2j + 1) / 2^24. */
 static double word_to_uniform(uint32_t w) {
-    uint32_t j = w >> 9;
+    uint32_t j = w & 0x7FFFFFu;
     return ((double)(2u * j + 1u)) / 16777216.0;
 }
 
