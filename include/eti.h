@@ -131,15 +131,18 @@ void eti_ctrl_defaults(eti_ctrl_params* p);
  * [B].  T_out may alias T_in.
  * Row errors (NaN/+inf logit, all -inf, bad T_in) give tok = -1, H = dH =
  * surprisal = NaN, T_out = T_in, theta_next = 0 (prune nothing), tau unchanged.
- * Uses no workspace.
+ * Workspace: eti_entropy_temp_sample_workspace_size(B, V) bytes (partial
+ * reductions of the row pieces; no initial contents required).
  */
+size_t eti_entropy_temp_sample_workspace_size(int B, int V);
+
 int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
                             const float* T_in, const float* H_prev, float* tau,
                             const float* H_target, const eti_ctrl_params* params,
                             uint64_t seed, uint64_t offset,
                             int32_t* tok, float* H, float* T_out,
                             float* dH, float* theta_next, float* tok_surprisal,
-                            uint32_t* err_flags, void* stream);
+                            uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * eti_score_prune_blocks -- the entropic keep set of half (b).

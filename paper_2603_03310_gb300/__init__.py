@@ -26,7 +26,8 @@ STATUS = {0: "ok", -1: "null pointer", -2: "bad shape", -3: "unsupported shape",
 ERRF_BAD_PAGE, ERRF_BAD_CTX, ERRF_NONFINITE, ERRF_ALL_NEG_INF, ERRF_BAD_TEMP = 1, 2, 4, 8, 16
 
 # C-ABI symbols declared in include/eti.h
-SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_score_prune_workspace_size",
+SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_entropy_temp_sample_workspace_size",
+           "eti_score_prune_workspace_size",
            "eti_score_prune_blocks", "eti_score_blocks", "eti_prune_blocks",
            "eti_paged_decode_workspace_size", "eti_paged_decode", "eti_version",
            "eti_status_string")
@@ -64,8 +65,10 @@ def load(path: str | None = None):
         lib.eti_version.restype = ctypes.c_char_p
         lib.eti_status_string.argtypes = [i32]
         lib.eti_status_string.restype = ctypes.c_char_p
+        lib.eti_entropy_temp_sample_workspace_size.argtypes = [i32, i32]
+        lib.eti_entropy_temp_sample_workspace_size.restype = sz
         lib.eti_entropy_temp_sample.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64,
-                                                P, P, P, P, P, P, P, P]
+                                                P, P, P, P, P, P, P, P, sz, P]
         lib.eti_entropy_temp_sample.restype = i32
         lib.eti_score_prune_workspace_size.argtypes = [i32] * 6
         lib.eti_score_prune_workspace_size.restype = sz
@@ -124,7 +127,11 @@ def _stream(stream) -> ctypes.c_void_p:
 
 
 # ---------------------------------------------------------------------------
-def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, err_flags,
+def entropy_temp_sample_workspace_size(B: int, V: int) -> int:
+    return int(load().eti_entropy_temp_sample_workspace_size(B, V))
+
+
+def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, err_flags, ws,
                             params: CtrlParams | None = None, seed: int = 0, offset: int = 0,
                             dH=None, theta_next=None, tok_surprisal=None, V: int | None = None,
                             stream=None):
@@ -142,7 +149,7 @@ def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, 
         _dev(tok, "tok", i32, B), _dev(H, "H", f32, B), _dev(T_out, "T_out", f32, B),
         _dev(dH, "dH", f32, B), _dev(theta_next, "theta_next", f32, B),
         _dev(tok_surprisal, "tok_surprisal", f32, B), _dev(err_flags, "err_flags", torch.int32, B),
-        _stream(stream))
+        _dev(ws, "ws", torch.uint8), ws.numel() if ws is not None else 0, _stream(stream))
     _check(st, "eti_entropy_temp_sample")
 
 
@@ -271,6 +278,7 @@ class DecodeStep:
                                     dtype=u8, device=dev)
         self.ws_dec = torch.empty(paged_decode_workspace_size(B, Hq, Hkv, D, P, max_blocks, True),
                                   dtype=u8, device=dev)
+        self.ws_ets = torch.empty(entropy_temp_sample_workspace_size(B, V), dtype=u8, device=dev)
 
     def attention(self, q, k_cache, v_cache, block_table, ctx_lens, scale, theta, B_min,
                   num_pages=None, stream=None):
@@ -287,7 +295,8 @@ class DecodeStep:
     def sample(self, logits, T_in, H_prev, tau, H_target, params=None, seed=0, offset=0, V=None,
                stream=None):
         eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, self.tok, self.H, self.T_out,
-                                self.err_ets, params=params, seed=seed, offset=offset, dH=self.dH,
+                                self.err_ets, self.ws_ets, params=params, seed=seed, offset=offset,
+                                dH=self.dH,
                                 theta_next=self.theta_next, tok_surprisal=self.surprisal,
                                 V=V, stream=stream)
 

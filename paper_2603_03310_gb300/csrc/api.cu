@@ -11,7 +11,8 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
                                    const float* H_target, const eti_ctrl_params* p,
                                    uint64_t seed, uint64_t offset, int32_t* tok, float* H,
                                    float* T_out, float* dH, float* theta_next, float* surprisal,
-                                   uint32_t* err, cudaStream_t stream, int cluster_override);
+                                   uint32_t* err, void* part, cudaStream_t stream);
+size_t eti_entropy_partial_bytes(int B);
 int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const int32_t* block_table,
                             const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
                             int max_blocks, long long num_pages, float scale, float* token_scores,
@@ -26,9 +27,9 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
                       const int32_t* kept_idx, const int32_t* kept_cnt, const float* token_scores,
                       const float* kept_norm, int B, int Hq, int Hkv, int D, int P, int max_blocks,
                       long long num_pages, uint16_t* out, uint32_t* err, int* plan_cum,
-                      int* plan_info, int* plan_cta_seg, float* partial, int ncta,
+                      int* plan_info, int* plan_warp_seg, float* partial, int nwarps,
                       cudaStream_t stream);
-int eti_decode_ncta();
+int eti_decode_nwarps();
 
 namespace {
 
@@ -63,11 +64,11 @@ struct Carver {
 
 struct DecodeWs {
     float* scores; float4* stats; int32_t* kidx; int32_t* kcnt; float* knorm;
-    int* cum; int* info; int* cta_seg; float* partial;
+    int* cum; int* info; int* warp_seg; float* partial;
 };
 
 DecodeWs carve_decode(void* ws, int B, int Hq, int Hkv, int D, int P, int max_blocks,
-                      int have_scores, int ncta, size_t* bytes) {
+                      int have_scores, int nwarps, size_t* bytes) {
     Carver c(ws);
     DecodeWs w{};
     const size_t g = Hq / Hkv, nseg = (size_t)B * Hkv;
@@ -80,8 +81,8 @@ DecodeWs carve_decode(void* ws, int B, int Hq, int Hkv, int D, int P, int max_bl
     }
     w.cum = c.take<int>(nseg + 1);
     w.info = c.take<int>(4);
-    w.cta_seg = c.take<int>(ncta);
-    w.partial = c.take<float>(((size_t)ncta + nseg) * g * D);
+    w.warp_seg = c.take<int>(nwarps);
+    w.partial = c.take<float>(((size_t)nwarps + nseg) * g * D);
     *bytes = c.off;
     return w;
 }
@@ -117,21 +118,27 @@ const char* eti_status_string(int s) {
     }
 }
 
+size_t eti_entropy_temp_sample_workspace_size(int B, int V) {
+    if (B < 0 || B > 65535 || V < 1) return 0;
+    return align256(eti_entropy_partial_bytes(B));
+}
+
 int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
                             const float* T_in, const float* H_prev, float* tau,
                             const float* H_target, const eti_ctrl_params* params,
                             uint64_t seed, uint64_t offset,
                             int32_t* tok, float* H, float* T_out,
                             float* dH, float* theta_next, float* tok_surprisal,
-                            uint32_t* err_flags, void* stream) {
+                            uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream) {
     if (B < 0 || B > 65535 || V < 1 || ld < V) return ETI_ERR_SHAPE;
     if (B == 0) return ETI_OK;
     if (!logits || !T_in || !H_prev || !tau || !H_target || !params || !tok || !H || !T_out ||
         !err_flags)
         return ETI_ERR_NULL;
+    if (!ws || ws_bytes < eti_entropy_temp_sample_workspace_size(B, V)) return ETI_ERR_WORKSPACE;
     return eti_launch_entropy_temp_sample(logits, B, V, (long long)ld, T_in, H_prev, tau, H_target,
                                           params, seed, offset, tok, H, T_out, dH, theta_next,
-                                          tok_surprisal, err_flags, (cudaStream_t)stream, 0);
+                                          tok_surprisal, err_flags, ws, (cudaStream_t)stream);
 }
 
 size_t eti_score_prune_workspace_size(int B, int Hq, int Hkv, int D, int P, int max_blocks) {
@@ -207,7 +214,7 @@ size_t eti_paged_decode_workspace_size(int B, int Hq, int Hkv, int D, int P, int
                                        int have_scores) {
     if (check_attn_shape(B, Hq, Hkv, D, P, max_blocks, 0) != ETI_OK) return 0;
     size_t bytes = 0;
-    carve_decode(nullptr, B, Hq, Hkv, D, P, max_blocks, have_scores, eti_decode_ncta(), &bytes);
+    carve_decode(nullptr, B, Hq, Hkv, D, P, max_blocks, have_scores, eti_decode_nwarps(), &bytes);
     return bytes;
 }
 
@@ -226,13 +233,14 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
     const bool have_scores = token_scores && kept_norm && have_lists;
     if (!v_cache || !block_table || !ctx_lens || !out || !err_flags) return ETI_ERR_NULL;
     if (!have_scores && (!q || !k_cache)) return ETI_ERR_NULL;
-    if (!aligned16(v_cache) || (!have_scores && (!aligned16(q) || !aligned16(k_cache))))
+    if (!aligned16(v_cache) || !aligned16(out) ||
+        (!have_scores && (!aligned16(q) || !aligned16(k_cache))))
         return ETI_ERR_ALIGN;
-    const int ncta = eti_decode_ncta();
+    const int nwarps = eti_decode_nwarps();
     size_t need = 0;
-    carve_decode(nullptr, B, Hq, Hkv, D, P, max_blocks, have_scores, ncta, &need);
+    carve_decode(nullptr, B, Hq, Hkv, D, P, max_blocks, have_scores, nwarps, &need);
     if (!ws || ws_bytes < need) return ETI_ERR_WORKSPACE;
-    DecodeWs w = carve_decode(ws, B, Hq, Hkv, D, P, max_blocks, have_scores, ncta, &need);
+    DecodeWs w = carve_decode(ws, B, Hq, Hkv, D, P, max_blocks, have_scores, nwarps, &need);
     cudaStream_t s = (cudaStream_t)stream;
     if (!have_scores) {
         st = eti_launch_score_blocks(q, k_cache, block_table, ctx_lens, B, Hq, Hkv, D, P,
@@ -251,7 +259,7 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
     }
     return eti_launch_decode(v_cache, block_table, ctx_lens, kept_idx, kept_cnt, token_scores,
                              kept_norm, B, Hq, Hkv, D, P, max_blocks, (long long)num_pages, out,
-                             err_flags, w.cum, w.info, w.cta_seg, w.partial, ncta, s);
+                             err_flags, w.cum, w.info, w.warp_seg, w.partial, nwarps, s);
 }
 
 }  // extern "C"

@@ -4,56 +4,55 @@
 // threshold (Section 3.2 safety floor, Section 5 entropy floor) and a
 // Gumbel-max draw from p_t, in ONE pass over the fp32 logits.
 //
-// Decomposition: a thread-block cluster of S CTAs per row; each CTA streams a
-// contiguous chunk of the row with 128-bit loads and keeps, per thread, the
-// online state
-//     m  = running max of z          (raw logit units)
-//     S  = sum 2^{t},  t = (z - m) * log2(e) / T
+// Decomposition: a persistent grid (4 CTAs per SM) in which every CTA takes an
+// equal contiguous share of the row-major list of all rows' 4-token groups,
+// so every SM finishes at the same time whatever B and V are.  Each CTA
+// streams its share with 128-bit loads (the next pair of groups is in flight
+// while the current pair is processed) and keeps, per thread, the online state
+//     m  = running max of z (raw logit units), mc = m * c,  c = log2(e) / T
+//     S  = sum 2^{t},  t = z c - mc
 //     U  = sum 2^{t} * t
-//     race best (w, E, index)  for the exponential race below.
-// The CTA partials are merged through distributed shared memory by cluster
-// rank 0, which writes the per-row outputs.  H = ln2 * (log2 S - U / S).
+//     race best (r = w / E, index)  for the exponential race below.
+// t is formed with one fma against the rounded mc; that rounding shifts every
+// t of a state by the same amount and cancels exactly in H = ln2 (log2 S - U/S).
+// A CTA writes one partial state per row piece it covered to scratch slot
+// (cta + row); a finalize kernel merges each row's slots in CTA order (a fixed
+// order: results do not depend on timing) and writes the per-row outputs.
 //
 // Sampling.  argmax_x y_x - log(-log u_x) is argmax_x w_x / E_x with
 // w_x = exp(y_x - m) and the exponential variate E_x = -log u_x, so the
-// exp() already needed for S is reused and one log per token remains.
-// Candidates are compared by cross-multiplication (w_a E_b > w_b E_a).
+// exp() already needed for S is reused and one log per token remains.  The
+// race keeps the best ratio r = w / E and a candidate wins when w > r E.
 // E is computed in log2 units (the common factor cancels in the race):
 //   u <= 15/16 : E2 = -lg2(u) with the MUFU approximation (|lg2 u| >= 0.093,
 //                so its absolute error stays a small relative error);
 //   u >  15/16 : v = 1 - u (exact), E2 = log2(e) * v * (1 + v/2 + ... + v^5/6),
 //                the Taylor series of -log(1 - v), whose remainder is below
 //                v^6/7 < 2^-24 / 7 relative.
-// u = (2 (word >> 9) + 1) / 2^24 is formed exactly as (1.m - (1 - 2^-24)).
-#include <cooperative_groups.h>
-
+// u = (2 (word & 0x7FFFFF) + 1) / 2^24 is formed exactly as 1.m - (1 - 2^-24).
 #include "common.cuh"
-
-namespace cg = cooperative_groups;
 
 namespace eti {
 
 // Philox4x32-10 (Salmon et al., SC'11): ten rounds of two 32x32->64-bit
-// multiplies; the key is bumped by the Weyl constants between rounds.
-__device__ __forceinline__ uint4 philox4x32_10(uint4 c, uint32_t k0, uint32_t k1) {
+// multiplies; round r uses the key bumped r times by the Weyl constants.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 c, const uint32_t (&k0)[10], const uint32_t (&k1)[10]) {
 #pragma unroll
     for (int r = 0; r < 10; ++r) {
         const unsigned long long p0 = (unsigned long long)0xD2511F53u * c.x;
         const unsigned long long p1 = (unsigned long long)0xCD9E8D57u * c.z;
         const uint32_t hi0 = (uint32_t)(p0 >> 32), lo0 = (uint32_t)p0;
         const uint32_t hi1 = (uint32_t)(p1 >> 32), lo1 = (uint32_t)p1;
-        c = make_uint4(hi1 ^ c.y ^ k0, lo1, hi0 ^ c.w ^ k1, lo0);
-        k0 += 0x9E3779B9u;
-        k1 += 0xBB67AE85u;
+        c = make_uint4(hi1 ^ c.y ^ k0[r], lo1, hi0 ^ c.w ^ k1[r], lo0);
     }
     return c;
 }
 
 // Exponential variate E / ln 2 from one 32-bit word (see the file comment).
 __device__ __forceinline__ float exp_variate_log2(uint32_t word) {
-    const float one_m = __uint_as_float((word >> 9) | 0x3F800000u);   // 1 + j 2^-23
-    const float u = one_m - __uint_as_float(0x3F7FFFFFu);             // (2j + 1) 2^-24, exact
-    const float v = 1.0f - u;                                         // exact for u > 1/2
+    const float one_m = __uint_as_float((word & 0x7FFFFFu) | 0x3F800000u);   // 1 + j 2^-23
+    const float u = one_m - __uint_as_float(0x3F7FFFFFu);                    // (2j + 1) 2^-24, exact
+    const float v = 1.0f - u;                                                // exact for u > 1/2
     // log2(e) / (k + 1), k = 0..5
     float s = fmaf(v, 0.24044917348149393f, 0.28853900817779268f);
     s = fmaf(v, s, 0.36067376022224085f);
@@ -67,67 +66,79 @@ __device__ __forceinline__ float exp_variate_log2(uint32_t word) {
 
 struct RowState {
     float m;    // max logit seen (raw units)
+    float mc;   // m * c, rounded once
     float S;    // sum 2^t
     float U;    // sum 2^t * t
-    float bw;   // race best: w relative to m
-    float bE;   // race best: E / ln 2
+    float r;    // race best: w / E relative to m (0 = none)
     int bi;     // race best: token index (INT_MAX = none)
 };
 
 __device__ __forceinline__ void state_init(RowState& s) {
-    s.m = -kInf; s.S = 0.f; s.U = 0.f; s.bw = 0.f; s.bE = 1.f; s.bi = 0x7fffffff;
+    s.m = -kInf; s.mc = -kInf; s.S = 0.f; s.U = 0.f; s.r = 0.f; s.bi = 0x7fffffff;
 }
 
 // Move the state to a new, larger reference max `nm`.
 __device__ __forceinline__ void state_rebase(RowState& s, float nm, float c) {
+    const float nmc = nm * c;
     float a = 0.f, d = 0.f;
     if (s.m != -kInf) {
-        d = (s.m - nm) * c;
+        d = s.mc - nmc;              // t_new = t_old + d for every term of the state
         a = fast_ex2(d);
     }
     s.U = a * fmaf(d, s.S, s.U);
     s.S *= a;
-    s.bw *= a;
+    s.r *= a;
     s.m = nm;
+    s.mc = nmc;
 }
 
 // Merge partial `o` into `s` (both may be empty).
 __device__ __forceinline__ void state_merge(RowState& s, RowState o, float c) {
-    const float nm = fmaxf(s.m, o.m);
-    if (nm == -kInf) return;
-    state_rebase(s, nm, c);
-    state_rebase(o, nm, c);
+    if (o.m == -kInf) return;
+    if (s.m == -kInf) { s = o; return; }
+    if (o.m > s.m) {
+        state_rebase(s, o.m, c);
+        // align o to the same rounded reference
+        const float d = o.mc - s.mc;
+        const float a = fast_ex2(d);
+        o.U = a * fmaf(d, o.S, o.U); o.S *= a; o.r *= a;
+    } else {
+        const float d = o.mc - s.mc;
+        const float a = fast_ex2(d);
+        o.U = a * fmaf(d, o.S, o.U); o.S *= a; o.r *= a;
+    }
     s.S += o.S;
     s.U += o.U;
-    const float lhs = o.bw * s.bE, rhs = s.bw * o.bE;
-    if (lhs > rhs || (lhs == rhs && o.bi < s.bi)) {
-        s.bw = o.bw; s.bE = o.bE; s.bi = o.bi;
-    }
+    if (o.r > s.r || (o.r == s.r && o.bi < s.bi)) { s.r = o.r; s.bi = o.bi; }
 }
 
 __device__ __forceinline__ RowState state_shfl_xor(const RowState& s, int o) {
     RowState r;
     r.m = __shfl_xor_sync(0xffffffffu, s.m, o);
+    r.mc = __shfl_xor_sync(0xffffffffu, s.mc, o);
     r.S = __shfl_xor_sync(0xffffffffu, s.S, o);
     r.U = __shfl_xor_sync(0xffffffffu, s.U, o);
-    r.bw = __shfl_xor_sync(0xffffffffu, s.bw, o);
-    r.bE = __shfl_xor_sync(0xffffffffu, s.bE, o);
+    r.r = __shfl_xor_sync(0xffffffffu, s.r, o);
     r.bi = __shfl_xor_sync(0xffffffffu, s.bi, o);
     return r;
 }
 
 // One token: entropy sums and the race.
 __device__ __forceinline__ void consume(RowState& s, float z, uint32_t word, int x, float c) {
-    const float t = (z - s.m) * c;
+    const float t = fmaf(z, c, -s.mc);
     const float w = fast_ex2(t);
     s.S += w;
     s.U = fmaf(w, fmaxf(t, -250.f), s.U);   // -inf logits add 0 (w = 0); NaN still reaches S
     const float E = exp_variate_log2(word);
-    if (w * s.bE > s.bw * E) { s.bw = w; s.bE = E; s.bi = x; }
+    if (w > s.r * E) {                        // rare after the first few tokens
+        s.r = __fdividef(w, E);
+        s.bi = x;
+    }
 }
 
 constexpr int kEtsThreads = 256;
-constexpr int kEtsBatch = 4;    // groups of 4 tokens loaded per thread per step
+constexpr int kEtsPair = 2;     // 4-token groups per thread per pipeline step
+constexpr int kEtsCtasPerSm = 4;
 
 struct EtsArgs {
     const float* logits;
@@ -146,156 +157,204 @@ struct EtsArgs {
     float* theta_next;
     float* surprisal;
     uint32_t* err;
-    int groups_per_cta;   // groups of 4 tokens per cluster rank
+    int ngroups;          // 4-token groups per row
+    long long share;      // groups per CTA of the persistent grid
+    RowState* part;       // [nCTA + B] partial states, slot (cta + row)
 };
 
 template <bool kVec>
-__global__ void __launch_bounds__(kEtsThreads)
-entropy_temp_sample_kernel(const EtsArgs a) {
-    cg::cluster_group cluster = cg::this_cluster();
-    const int rank = (int)cluster.block_rank();
-    const int nrank = (int)cluster.num_blocks();
-    const int b = blockIdx.y;
-    const int tid = threadIdx.x;
-    __shared__ RowState warp_part[kEtsThreads / 32];
-    __shared__ RowState cta_part;
+__device__ __forceinline__ void load_group(float (&z)[4], const float* row, int g, int g1, int full_groups,
+                                           int V) {
+    if (g < g1 && kVec && g < full_groups) {
+        const float4 v = ldg_stream_f4(row + 4 * (long long)g);
+        z[0] = v.x; z[1] = v.y; z[2] = v.z; z[3] = v.w;
+    } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int x = 4 * g + e;
+            z[e] = (g < g1 && x < V) ? __ldg(row + x) : -kInf;
+        }
+    }
+}
 
+// Persistent pass: CTA c takes groups [c*share, (c+1)*share) of the
+// row-major list of all rows' 4-token groups, one row piece at a time.
+template <bool kVec>
+__global__ void __launch_bounds__(kEtsThreads, kEtsCtasPerSm)
+entropy_sample_partial_kernel(const EtsArgs a) {
+    __shared__ RowState warp_part[kEtsThreads / 32];
+    const int tid = threadIdx.x;
+    const long long total = (long long)a.B * a.ngroups;
+    long long q0 = (long long)blockIdx.x * a.share;
+    const long long q1 = min(q0 + a.share, total);
+    const int full_groups = a.V >> 2;
+    uint32_t k0[10], k1[10];
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        k0[r] = a.seed_lo + (uint32_t)r * 0x9E3779B9u;
+        k1[r] = a.seed_hi + (uint32_t)r * 0xBB67AE85u;
+    }
+    while (q0 < q1) {
+        const int b = (int)(q0 / a.ngroups);
+        const int g0 = (int)(q0 - (long long)b * a.ngroups);
+        const int g1 = (int)min((long long)a.ngroups, q1 - (long long)b * a.ngroups);
+        const float T = a.T_in[b];
+        const bool bad_T = !(T > 0.f && T < kInf);
+        const float c = bad_T ? 0.f : kLog2e / T;
+        const float* row = a.logits + (long long)b * a.ld;
+        RowState s;
+        state_init(s);
+        if (!bad_T && g0 + tid < g1) {
+            constexpr int step = kEtsPair * kEtsThreads;
+            float cur[kEtsPair][4], nxt[kEtsPair][4];
+#pragma unroll
+            for (int k = 0; k < kEtsPair; ++k) load_group<kVec>(cur[k], row, g0 + k * kEtsThreads + tid, g1, full_groups, a.V);
+            for (int base = g0; base < g1; base += step) {
+                const bool more = base + step < g1;
+                if (more) {
+#pragma unroll
+                    for (int k = 0; k < kEtsPair; ++k)
+                        load_group<kVec>(nxt[k], row, base + step + k * kEtsThreads + tid, g1, full_groups, a.V);
+                }
+                float bm = -kInf;
+#pragma unroll
+                for (int k = 0; k < kEtsPair; ++k)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) bm = fmaxf(bm, cur[k][e]);
+                if (bm == -kInf) {
+                    // every token of the pair is -inf (or NaN): nothing to add and
+                    // nothing to draw, but a NaN must still poison the row
+                    bool nan = false;
+#pragma unroll
+                    for (int k = 0; k < kEtsPair; ++k)
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) nan |= (cur[k][e] != cur[k][e]);
+                    if (nan) s.S = __int_as_float(0x7fc00000);
+                } else {
+                    if (bm > s.m) state_rebase(s, bm, c);
+#pragma unroll
+                    for (int k = 0; k < kEtsPair; ++k) {
+                        const int g = base + k * kEtsThreads + tid;
+                        if (g < g1) {
+                            const uint4 r = philox4x32_10(make_uint4((uint32_t)g, (uint32_t)b, a.off_lo, a.off_hi), k0, k1);
+                            consume(s, cur[k][0], r.x, 4 * g + 0, c);
+                            consume(s, cur[k][1], r.y, 4 * g + 1, c);
+                            consume(s, cur[k][2], r.z, 4 * g + 2, c);
+                            consume(s, cur[k][3], r.w, 4 * g + 3, c);
+                        }
+                    }
+                }
+                if (!more) break;
+#pragma unroll
+                for (int k = 0; k < kEtsPair; ++k)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) cur[k][e] = nxt[k][e];
+            }
+        }
+        // CTA reduction of the piece into slot (cta + row)
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) state_merge(s, state_shfl_xor(s, o), c);
+        if ((tid & 31) == 0) warp_part[tid >> 5] = s;
+        __syncthreads();
+        if (tid == 0) {
+            RowState t = warp_part[0];
+            for (int w = 1; w < kEtsThreads / 32; ++w) state_merge(t, warp_part[w], c);
+            a.part[blockIdx.x + b] = t;
+        }
+        __syncthreads();
+        q0 = (long long)b * a.ngroups + g1;
+    }
+}
+
+// Per row: merge the partial slots in CTA order, then the scalar epilogue.
+__global__ void __launch_bounds__(128)
+entropy_sample_finalize_kernel(const EtsArgs a) {
+    const int lane = threadIdx.x & 31;
+    const int b = blockIdx.x * 4 + (threadIdx.x >> 5);
+    if (b >= a.B) return;
     const float T = a.T_in[b];
     const bool bad_T = !(T > 0.f && T < kInf);
     const float c = bad_T ? 0.f : kLog2e / T;
-    const float* row = a.logits + (long long)b * a.ld;
-    const int ngroups = (a.V + 3) >> 2;
-    const int g0 = min(rank * a.groups_per_cta, ngroups);
-    const int g1 = min(g0 + a.groups_per_cta, ngroups);
-    const int full_groups = a.V >> 2;   // groups with 4 in-range tokens
-
+    const long long lo = (long long)b * a.ngroups, hi = lo + a.ngroups - 1;
+    const int c0 = (int)(lo / a.share), c1 = (int)(hi / a.share);
+    // lane l merges slots c0 + l, c0 + l + 32, ... in order, then the lanes merge
+    // in a fixed tree: the result does not depend on timing
     RowState s;
     state_init(s);
-    if (!bad_T) {
-        for (int base = g0; base < g1; base += kEtsBatch * kEtsThreads) {
-            float z[kEtsBatch][4];
+    for (int cc = c0 + lane; cc <= c1; cc += 32) state_merge(s, a.part[cc + b], c);
 #pragma unroll
-            for (int k = 0; k < kEtsBatch; ++k) {
-                const int g = base + k * kEtsThreads + tid;
-                if (g < g1 && kVec && g < full_groups) {
-                    const float4 v = ldg_stream_f4(row + 4 * (long long)g);
-                    z[k][0] = v.x; z[k][1] = v.y; z[k][2] = v.z; z[k][3] = v.w;
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int x = 4 * g + e;
-                        z[k][e] = (g < g1 && x < a.V) ? __ldg(row + x) : -kInf;
-                    }
-                }
-            }
-            float bm = -kInf;
-#pragma unroll
-            for (int k = 0; k < kEtsBatch; ++k)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) bm = fmaxf(bm, z[k][e]);
-            if (bm == -kInf) {
-                // every token of the batch is -inf (or NaN): nothing to add and
-                // nothing to draw, but a NaN must still poison the row
-                bool nan = false;
-#pragma unroll
-                for (int k = 0; k < kEtsBatch; ++k)
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) nan |= (z[k][e] != z[k][e]);
-                if (nan) s.S = __int_as_float(0x7fc00000);
-                continue;
-            }
-            if (bm > s.m) state_rebase(s, bm, c);
-#pragma unroll
-            for (int k = 0; k < kEtsBatch; ++k) {
-                const int g = base + k * kEtsThreads + tid;
-                if (g < g1) {
-                    const uint4 r = philox4x32_10(make_uint4((uint32_t)g, (uint32_t)b, a.off_lo, a.off_hi),
-                                                  a.seed_lo, a.seed_hi);
-                    consume(s, z[k][0], r.x, 4 * g + 0, c);
-                    consume(s, z[k][1], r.y, 4 * g + 1, c);
-                    consume(s, z[k][2], r.z, 4 * g + 2, c);
-                    consume(s, z[k][3], r.w, 4 * g + 3, c);
-                }
-            }
+    for (int o = 1; o < 32; o <<= 1) {
+        RowState o2 = state_shfl_xor(s, o);
+        // keep the lower-lane state first so ties resolve to the lower index
+        if (lane & o) { RowState t = o2; o2 = s; s = t; }
+        state_merge(s, o2, c);
+    }
+    if (lane != 0) return;
+    const RowState& t = s;
+    const float* row = a.logits + (long long)b * a.ld;
+    uint32_t err = bad_T ? ETI_ERRF_BAD_TEMP : 0u;
+    if (!err) {
+        if (t.m == -kInf) err = ETI_ERRF_ALL_NEG_INF;
+        else if (t.m == kInf || isnan(t.S) || isnan(t.U)) err = ETI_ERRF_NONFINITE;
+    }
+    const float tau_in = a.tau[b];
+    if (err) {
+        a.tok[b] = -1;
+        a.H[b] = __int_as_float(0x7fc00000);
+        a.T_out[b] = T;
+        if (a.dH) a.dH[b] = __int_as_float(0x7fc00000);
+        if (a.theta_next) a.theta_next[b] = 0.f;
+        if (a.surprisal) a.surprisal[b] = __int_as_float(0x7fc00000);
+    } else {
+        const float l2S = log2f(t.S);
+        const float H = fmaxf(kLn2 * (l2S - t.U / t.S), 0.f);
+        const float dH = a.H_prev[b] - H;
+        a.tau[b] = tau_in + fmaxf(dH, 0.f);
+        float Tn = T * expf(a.p.sign * a.p.eta * (H - a.H_target[b]));
+        Tn = fminf(a.p.T_max, fmaxf(a.p.T_min, Tn));
+        a.tok[b] = t.bi;
+        a.H[b] = H;
+        a.T_out[b] = Tn;
+        if (a.dH) a.dH[b] = dH;
+        if (a.theta_next) {
+            const float Heff = fmaxf(H - a.p.eps_H, a.p.H_min);
+            const float tmax = a.V > 1 ? a.p.theta_hi * fmaxf(0.f, 1.f - Heff / logf((float)a.V))
+                                       : a.p.theta_hi;
+            a.theta_next[b] = fminf(a.p.theta_user, tmax);
+        }
+        if (a.surprisal) {
+            const float tt = fmaf(row[t.bi], c, -t.mc);
+            a.surprisal[b] = kLn2 * (l2S - tt);
         }
     }
-    // CTA reduction: warp shuffles, then one warp over the warp partials.
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) state_merge(s, state_shfl_xor(s, o), c);
-    if ((tid & 31) == 0) warp_part[tid >> 5] = s;
-    __syncthreads();
-    if (tid == 0) {
-        RowState t = warp_part[0];
-        for (int w = 1; w < kEtsThreads / 32; ++w) state_merge(t, warp_part[w], c);
-        cta_part = t;
-    }
-    cluster.sync();
-    if (rank == 0 && tid == 0) {
-        RowState t = cta_part;
-        for (int r = 1; r < nrank; ++r) state_merge(t, *cluster.map_shared_rank(&cta_part, r), c);
-        uint32_t err = bad_T ? ETI_ERRF_BAD_TEMP : 0u;
-        if (!err) {
-            if (t.m == -kInf) err = ETI_ERRF_ALL_NEG_INF;
-            else if (t.m == kInf || isnan(t.S) || isnan(t.U)) err = ETI_ERRF_NONFINITE;
-        }
-        const float tau_in = a.tau[b];
-        if (err) {
-            a.tok[b] = -1;
-            a.H[b] = __int_as_float(0x7fc00000);
-            a.T_out[b] = T;
-            if (a.dH) a.dH[b] = __int_as_float(0x7fc00000);
-            if (a.theta_next) a.theta_next[b] = 0.f;
-            if (a.surprisal) a.surprisal[b] = __int_as_float(0x7fc00000);
-        } else {
-            const float l2S = log2f(t.S);
-            const float H = fmaxf(kLn2 * (l2S - t.U / t.S), 0.f);
-            const float dH = a.H_prev[b] - H;
-            a.tau[b] = tau_in + fmaxf(dH, 0.f);
-            float Tn = T * expf(a.p.sign * a.p.eta * (H - a.H_target[b]));
-            Tn = fminf(a.p.T_max, fmaxf(a.p.T_min, Tn));
-            a.tok[b] = t.bi;
-            a.H[b] = H;
-            a.T_out[b] = Tn;
-            if (a.dH) a.dH[b] = dH;
-            if (a.theta_next) {
-                const float Heff = fmaxf(H - a.p.eps_H, a.p.H_min);
-                const float tmax = a.V > 1 ? a.p.theta_hi * fmaxf(0.f, 1.f - Heff / logf((float)a.V))
-                                           : a.p.theta_hi;
-                a.theta_next[b] = fminf(a.p.theta_user, tmax);
-            }
-            if (a.surprisal) {
-                const float tt = (row[t.bi] - t.m) * c;
-                a.surprisal[b] = kLn2 * (l2S - tt);
-            }
-        }
-        a.err[b] = err;
-    }
-    // keep every CTA's shared memory alive until rank 0 has read it
-    cluster.sync();
+    a.err[b] = err;
 }
 
 }  // namespace eti
 
-// Host launcher (called from the C ABI after argument validation).
+// CTAs of the persistent sampling grid on the current device
+int eti_entropy_ncta() {
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return eti::kEtsCtasPerSm * sms;
+}
+
+size_t eti_entropy_partial_bytes(int B) {
+    return (size_t)(eti_entropy_ncta() + B) * sizeof(eti::RowState);
+}
+
+// Host launcher (called from the C ABI after argument validation); `part`
+// holds eti_entropy_partial_bytes(B) bytes of scratch.
 int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long ld,
                                    const float* T_in, const float* H_prev, float* tau,
                                    const float* H_target, const eti_ctrl_params* p,
                                    uint64_t seed, uint64_t offset, int32_t* tok, float* H,
                                    float* T_out, float* dH, float* theta_next, float* surprisal,
-                                   uint32_t* err, cudaStream_t stream, int cluster_override) {
+                                   uint32_t* err, void* part, cudaStream_t stream) {
     using namespace eti;
     if (B == 0) return ETI_OK;
-    const int ngroups = (V + 3) / 4;
-    int dev = 0, sms = 148;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    // aim for ~4 CTAs per SM in one wave, at least one group per thread
-    int S = cluster_override > 0 ? cluster_override : 1;
-    if (cluster_override <= 0) {
-        const int want = ceil_div(4 * sms, B);
-        const int cap = max(1, ceil_div(ngroups, kEtsThreads));
-        while (S < 8 && S < want && S < cap) S <<= 1;
-    }
+    const int ncta = eti_entropy_ncta();
     EtsArgs a;
     a.logits = logits; a.B = B; a.V = V; a.ld = ld; a.T_in = T_in; a.H_prev = H_prev;
     a.tau = tau; a.H_target = H_target; a.p = *p;
@@ -303,22 +362,14 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
     a.off_lo = (uint32_t)offset; a.off_hi = (uint32_t)(offset >> 32);
     a.tok = tok; a.H = H; a.T_out = T_out; a.dH = dH; a.theta_next = theta_next;
     a.surprisal = surprisal; a.err = err;
-    a.groups_per_cta = ceil_div(ngroups, S);
+    a.ngroups = (V + 3) / 4;
+    const long long total = (long long)B * a.ngroups;
+    a.share = (total + ncta - 1) / ncta;
+    a.part = static_cast<RowState*>(part);
     const bool vec = (ld % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
-
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(S, B, 1);
-    cfg.blockDim = dim3(kEtsThreads, 1, 1);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = S;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cudaError_t e = vec ? cudaLaunchKernelEx(&cfg, entropy_temp_sample_kernel<true>, a)
-                        : cudaLaunchKernelEx(&cfg, entropy_temp_sample_kernel<false>, a);
-    return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
+    if (vec) entropy_sample_partial_kernel<true><<<ncta, kEtsThreads, 0, stream>>>(a);
+    else entropy_sample_partial_kernel<false><<<ncta, kEtsThreads, 0, stream>>>(a);
+    if (cudaGetLastError() != cudaSuccess) return ETI_ERR_CUDA;
+    entropy_sample_finalize_kernel<<<(B + 3) / 4, 128, 0, stream>>>(a);
+    return cudaGetLastError() == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
 }

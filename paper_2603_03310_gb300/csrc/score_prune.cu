@@ -73,6 +73,8 @@ __device__ int units_prefix(const int32_t* ctx_lens, int B, int P, int max_block
     return carry;
 }
 
+constexpr int kScorePrefetch = 6;   // blocks prefetched into L2 ahead of the loads
+
 template <int D>
 struct KTile {
     static constexpr int kChunks = D / 32;   // 16-byte loads per token row per thread
@@ -95,31 +97,18 @@ __device__ __forceinline__ void load_k_tile(KTile<D>& t, const uint16_t* tile, i
     }
 }
 
-// Cursor over a warp's units (sequence, kv head, block, tile).
-struct UnitCursor {
-    int b, kvh, blk, tile, nb;
+// one unit of a warp's range, resolved by one lane
+struct UnitInfo {
+    int b, kvh, blk, page;
 };
-
-__device__ __forceinline__ void cursor_advance(UnitCursor& u, const int32_t* ctx_lens, int P,
-                                               int max_blocks, int Hkv, int tiles) {
-    if (++u.tile < tiles) return;
-    u.tile = 0;
-    if (++u.blk < u.nb) return;
-    u.blk = 0;
-    if (++u.kvh < Hkv) return;
-    u.kvh = 0;
-    do {
-        ++u.b;
-        u.nb = seq_blocks(ctx_lens[u.b], P, max_blocks);
-    } while (u.nb == 0);
-}
 
 template <int D, int P>
 __global__ void __launch_bounds__(kScoreThreads, 2)
 score_blocks_kernel(const ScoreArgs a) {
+    constexpr int kTiles = P / 16;
+    constexpr int C = KTile<D>::kChunks;
     extern __shared__ int smem_cum[];
     __shared__ int warp_tot[kScoreWarps];
-    constexpr int kTiles = P / 16;
     const int total = units_prefix(a.ctx_lens, a.B, P, a.max_blocks, a.Hkv, smem_cum, warp_tot);
     const int lane = threadIdx.x & 31, grp = lane >> 2, tq = lane & 3;
     const int gwarp = blockIdx.x * kScoreWarps + (threadIdx.x >> 5);
@@ -128,92 +117,129 @@ score_blocks_kernel(const ScoreArgs a) {
     const int u0 = gwarp * share;
     const int u1 = min(u0 + share, total);
     if (u0 >= u1) return;
-
-    // locate the first unit: largest b with cum[b] <= u0 (and blocks > 0)
-    int lo = 0, hi = a.B - 1;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (smem_cum[mid] <= u0) lo = mid; else hi = mid - 1;
-    }
-    UnitCursor cur;
-    cur.b = lo;
-    cur.nb = seq_blocks(a.ctx_lens[lo], P, a.max_blocks);
-    {
-        const int r = u0 - smem_cum[lo];
-        cur.kvh = r / cur.nb;
-        cur.blk = r - cur.kvh * cur.nb;
-        cur.tile = 0;
-    }
     const int ntiles = (u1 - u0) * kTiles;
 
-    auto tile_ptr = [&](const UnitCursor& u, bool& valid) -> const uint16_t* {
-        const int page = a.block_table[(long long)u.b * a.max_blocks + u.blk];
-        valid = page >= 0 && (long long)page < a.num_pages;
-        const long long chunk = ((long long)(valid ? page : 0) * a.Hkv + u.kvh) * P;
-        return a.k_cache + (chunk + u.tile * 16) * D;
+    // unit u -> (sequence, kv head, block, page); one lane per unit, 32 at a time
+    auto resolve = [&](int base) -> UnitInfo {
+        UnitInfo it{0, 0, 0, -1};
+        const int u = base + lane;
+        if (u < u1) {
+            int lo = 0, hi = a.B - 1;   // largest b with cum[b] <= u
+            while (lo < hi) {
+                const int mid = (lo + hi + 1) >> 1;
+                if (smem_cum[mid] <= u) lo = mid; else hi = mid - 1;
+            }
+            const int nb = seq_blocks(__ldg(a.ctx_lens + lo), P, a.max_blocks);
+            const int r = u - smem_cum[lo];
+            it.b = lo;
+            it.kvh = r / nb;
+            it.blk = r - it.kvh * nb;
+            const int pg = __ldg(a.block_table + (long long)lo * a.max_blocks + it.blk);
+            it.page = (pg >= 0 && (long long)pg < a.num_pages) ? pg : -1;
+        }
+        return it;
     };
+    UnitInfo cur = resolve(u0);
+    int cbase = u0;
+    UnitInfo nxt = resolve(u0 + 32);
+    // unit at offset off (0..63) from cbase
+    auto unit_at = [&](int off) -> UnitInfo {
+        const int l = off & 31;
+        UnitInfo a0, a1;
+        a0.b = __shfl_sync(0xffffffffu, cur.b, l);     a1.b = __shfl_sync(0xffffffffu, nxt.b, l);
+        a0.kvh = __shfl_sync(0xffffffffu, cur.kvh, l); a1.kvh = __shfl_sync(0xffffffffu, nxt.kvh, l);
+        a0.blk = __shfl_sync(0xffffffffu, cur.blk, l); a1.blk = __shfl_sync(0xffffffffu, nxt.blk, l);
+        a0.page = __shfl_sync(0xffffffffu, cur.page, l); a1.page = __shfl_sync(0xffffffffu, nxt.page, l);
+        return off < 32 ? a0 : a1;
+    };
+    auto chunk_ptr = [&](const UnitInfo& it) {
+        return a.k_cache + ((long long)(it.page >= 0 ? it.page : 0) * a.Hkv + it.kvh) * P * D;
+    };
+    // warm the L2 with the first blocks of the range (shuffles on every lane,
+    // one prefetch instruction from lane 0)
+    for (int k = 0; k < kScorePrefetch && u0 + k < u1; ++k) {
+        const UnitInfo it = unit_at(k);
+        if (lane == 0 && it.page >= 0) prefetch_l2_bulk(chunk_ptr(it), P * D * 2);
+    }
 
     KTile<D> buf0, buf1;
-    bool v0 = false, v1 = false;
-    {
-        const uint16_t* p0 = tile_ptr(cur, v0);
-        load_k_tile<D>(buf0, p0, grp, tq, v0);
-    }
-    UnitCursor nxt = cur;
-    uint4 qf[KTile<D>::kChunks];
+    UnitInfo ucur = unit_at(0);
+    load_k_tile<D>(buf0, chunk_ptr(ucur), grp, tq, ucur.page >= 0);
+    int cur_tile = 0;
+    uint4 qf[C];
     int q_b = -1, q_kvh = -1;
     float xs[kTiles][4];
 
-    // one tile: prefetch the next tile into `nb`, then consume `cb`
-    auto step = [&](const KTile<D>& cbuf, bool cvalid, KTile<D>& nbuf, bool& nvalid, int i) {
+    // one tile: load the next tile into `nbuf` (and prefetch further ahead),
+    // then consume `cbuf`
+    auto step = [&](const KTile<D>& cbuf, KTile<D>& nbuf, int i) {
+        const UnitInfo me = ucur;
+        const int tile = cur_tile;
         if (i + 1 < ntiles) {
-            cursor_advance(nxt, a.ctx_lens, P, a.max_blocks, a.Hkv, kTiles);
-            const uint16_t* p = tile_ptr(nxt, nvalid);
-            load_k_tile<D>(nbuf, p, grp, tq, nvalid);
+            const int item1 = u0 + (i + 1) / kTiles;
+            const int tile1 = (i + 1) - ((i + 1) / kTiles) * kTiles;
+            if (item1 >= cbase + 32) {
+                cur = nxt;
+                cbase += 32;
+                nxt = resolve(cbase + 32);
+            }
+            ucur = unit_at(item1 - cbase);
+            cur_tile = tile1;
+            load_k_tile<D>(nbuf, chunk_ptr(ucur) + tile1 * 16 * D, grp, tq, ucur.page >= 0);
+            if (tile1 == 0 && item1 + kScorePrefetch < u1) {
+                const UnitInfo pf = unit_at(item1 + kScorePrefetch - cbase);
+                if (lane == 0 && pf.page >= 0) prefetch_l2_bulk(chunk_ptr(pf), P * D * 2);
+            }
         }
-        if (cur.b != q_b || cur.kvh != q_kvh) {
-            q_b = cur.b;
-            q_kvh = cur.kvh;
-            const int h = cur.kvh * a.g + grp;
+        if (me.b != q_b || me.kvh != q_kvh) {
+            q_b = me.b;
+            q_kvh = me.kvh;
+            const int h = me.kvh * a.g + grp;
 #pragma unroll
-            for (int c = 0; c < KTile<D>::kChunks; ++c)
+            for (int c = 0; c < C; ++c)
                 qf[c] = grp < a.g ? __ldg(reinterpret_cast<const uint4*>(
-                                        a.q + ((long long)cur.b * a.Hq + h) * D + 32 * c + 8 * tq))
+                                        a.q + ((long long)me.b * a.Hq + h) * D + 32 * c + 8 * tq))
                                   : make_uint4(0, 0, 0, 0);
         }
         float acc[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-        for (int c = 0; c < KTile<D>::kChunks; ++c) {
+        for (int c = 0; c < C; ++c) {
             mma_bf16_16x8x16(acc, cbuf.lo[c].x, cbuf.hi[c].x, cbuf.lo[c].y, cbuf.hi[c].y, qf[c].x, qf[c].y);
             mma_bf16_16x8x16(acc, cbuf.lo[c].z, cbuf.hi[c].z, cbuf.lo[c].w, cbuf.hi[c].w, qf[c].z, qf[c].w);
         }
         // token slots grp, grp+8 of this tile; heads 2tq, 2tq+1
-        const int L = a.ctx_lens[cur.b];
-        const int valid_tok = min(P, L - cur.blk * P) - cur.tile * 16;
+        const int L = __ldg(a.ctx_lens + me.b);
+        const int valid_tok = min(P, L - me.blk * P) - tile * 16;
+        const bool ok = me.page >= 0;
         float x4[4];
-        x4[0] = (cvalid && grp < valid_tok) ? acc[0] * a.scale : -kInf;
-        x4[1] = (cvalid && grp < valid_tok) ? acc[1] * a.scale : -kInf;
-        x4[2] = (cvalid && grp + 8 < valid_tok) ? acc[2] * a.scale : -kInf;
-        x4[3] = (cvalid && grp + 8 < valid_tok) ? acc[3] * a.scale : -kInf;
+        x4[0] = (ok && grp < valid_tok) ? acc[0] * a.scale : -kInf;
+        x4[1] = (ok && grp < valid_tok) ? acc[1] * a.scale : -kInf;
+        x4[2] = (ok && grp + 8 < valid_tok) ? acc[2] * a.scale : -kInf;
+        x4[3] = (ok && grp + 8 < valid_tok) ? acc[3] * a.scale : -kInf;
 #pragma unroll
         for (int tt = 0; tt < kTiles; ++tt)      // static indices keep xs in registers
-            if (tt == cur.tile)
+            if (tt == tile)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) xs[tt][e] = x4[e];
-        const long long unit = ((long long)cur.b * a.Hkv + cur.kvh) * a.max_blocks + cur.blk;
+        const long long unit = ((long long)me.b * a.Hkv + me.kvh) * a.max_blocks + me.blk;
         if (a.token_scores) {
-            float* ts = a.token_scores + (unit * P + cur.tile * 16) * a.g;
+            float* ts = a.token_scores + (unit * P + tile * 16) * a.g;
             const int h0 = 2 * tq, h1 = 2 * tq + 1;
-            if (h0 < a.g) {
-                ts[grp * a.g + h0] = x4[0];
-                ts[(grp + 8) * a.g + h0] = x4[2];
-            }
-            if (h1 < a.g) {
-                ts[grp * a.g + h1] = x4[1];
-                ts[(grp + 8) * a.g + h1] = x4[3];
+            if (h1 < a.g && (a.g & 1) == 0) {
+                *reinterpret_cast<float2*>(ts + grp * a.g + h0) = make_float2(x4[0], x4[1]);
+                *reinterpret_cast<float2*>(ts + (grp + 8) * a.g + h0) = make_float2(x4[2], x4[3]);
+            } else {
+                if (h0 < a.g) {
+                    ts[grp * a.g + h0] = x4[0];
+                    ts[(grp + 8) * a.g + h0] = x4[2];
+                }
+                if (h1 < a.g) {
+                    ts[grp * a.g + h1] = x4[1];
+                    ts[(grp + 8) * a.g + h1] = x4[3];
+                }
             }
         }
-        if (cur.tile == kTiles - 1) {
+        if (tile == kTiles - 1) {
             // block stats for heads 2tq (j = 0) and 2tq + 1 (j = 1)
 #pragma unroll
             for (int j = 0; j < 2; ++j) {
@@ -251,12 +277,11 @@ score_blocks_kernel(const ScoreArgs a) {
                 if (grp == 0 && h < a.g) a.stats[unit * a.g + h] = make_float4(m, l1, u, 0.f);
             }
         }
-        cur = nxt;
     };
 
     for (int i = 0; i < ntiles; i += 2) {
-        step(buf0, v0, buf1, v1, i);
-        if (i + 1 < ntiles) step(buf1, v1, buf0, v0, i + 1);
+        step(buf0, buf1, i);
+        if (i + 1 < ntiles) step(buf1, buf0, i + 1);
     }
 }
 
@@ -347,11 +372,22 @@ __device__ __forceinline__ uint32_t order_key(float f) {
     return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
+// Shared memory of prune_finalize: block scores / flags, then (when cached)
+// the block stats of the segment, head-major.
 template <int G>
+__host__ __device__ constexpr size_t fin_smem_bytes(int max_blocks, bool cache) {
+    return (size_t)max_blocks * 4 * (cache ? 1 + 3 * G : 1);
+}
+
+template <int G, bool kCache>
 __global__ void __launch_bounds__(kFinThreads)
 prune_finalize_kernel(const FinArgs a) {
-    extern __shared__ float sh_score[];          // [max_blocks] scores, then flags
-    __shared__ float red[(kFinThreads / 32) * 16];
+    extern __shared__ __align__(16) float fin_smem[];
+    float* sh_score = fin_smem;                       // [max_blocks]: scores, then keep flags
+    float* sh_m = fin_smem + a.max_blocks;            // [G][max_blocks] (kCache)
+    float* sh_l = sh_m + G * a.max_blocks;
+    float* sh_u = sh_l + G * a.max_blocks;
+    __shared__ float red[(kFinThreads / 32) * 3 * 8];
     __shared__ int ired[kFinThreads / 32];
     __shared__ int hist[256];
     __shared__ int sel_digit, sel_rem;
@@ -362,50 +398,63 @@ prune_finalize_kernel(const FinArgs a) {
     const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
     const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
     const long long segbase = (long long)seg * a.max_blocks;
+    const int per = (nb + nt - 1) / nt;          // contiguous block range per thread
+    const int j0 = min(tid * per, nb), j1 = min(j0 + per, nb);
+    const float4* st = a.stats + segbase * G;
 
-    // page ids of the sequence
+    // pass 1 (the only pass over global memory when the stats fit in shared
+    // memory): page ids, stats cache, max per head
     int bad = 0;
-    for (int j = tid; j < nb; j += nt) {
+    float M[G];
+#pragma unroll
+    for (int h = 0; h < G; ++h) M[h] = -kInf;
+    for (int j = j0; j < j1; ++j) {
         const int pg = a.block_table[(long long)b * a.max_blocks + j];
         bad |= (pg < 0 || (long long)pg >= a.num_pages);
+#pragma unroll
+        for (int h = 0; h < G; ++h) {
+            const float4 s = st[j * G + h];
+            if (kCache) {
+                sh_m[h * a.max_blocks + j] = s.x;
+                sh_l[h * a.max_blocks + j] = s.y;
+                sh_u[h * a.max_blocks + j] = s.z;
+            }
+            M[h] = fmaxf(M[h], s.x);
+        }
     }
     const bool bad_page = __syncthreads_or(bad) != 0;
     if (a.err && kvh == 0 && tid == 0)
         a.err[b] = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page && !bad_ctx ? ETI_ERRF_BAD_PAGE : 0u);
     const int n = (bad_ctx || bad_page) ? 0 : nb;
-    const int per = (n + nt - 1) / nt;          // contiguous block range per thread
-    const int j0 = min(tid * per, n), j1 = min(j0 + per, n);
-    const float4* st = a.stats + segbase * G;
+    const int k0 = min(j0, n), k1 = min(j1, n);
 
-    float M[G], Z[G];
-    if (n > 0) {
-#pragma unroll
-        for (int h = 0; h < G; ++h) M[h] = -kInf;
-        for (int j = j0; j < j1; ++j)
-#pragma unroll
-            for (int h = 0; h < G; ++h) M[h] = fmaxf(M[h], st[j * G + h].x);
-        block_reduce_max<G>(M, red);
-    }
+    auto stat = [&](int j, int h) -> float4 {
+        if (kCache) return make_float4(sh_m[h * a.max_blocks + j], sh_l[h * a.max_blocks + j],
+                                       sh_u[h * a.max_blocks + j], 0.f);
+        return st[j * G + h];
+    };
 
     if (!a.given) {
         if (n > 0) {
-#pragma unroll
+            block_reduce_max<G>(M, red);
             // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
-            // c_b = e^{m_b - M}: exact around Z ~ 1, so log Z = log1p(Z - 1) keeps
-            // its relative precision when one token takes nearly all attention.
-            float Zs[2 * G];   // [h]: the part below 1; [G + h]: number of top blocks
+            // c_b = e^{m_b - M}: the "1"s of the blocks at the max are counted,
+            // not summed, so log Z = log1p(Z - 1) keeps its relative precision
+            // when one token takes nearly all of the attention.
+            float Zs[2 * G];
 #pragma unroll
             for (int h = 0; h < 2 * G; ++h) Zs[h] = 0.f;
-            for (int j = j0; j < j1; ++j)
+            for (int j = k0; j < k1; ++j)
 #pragma unroll
                 for (int h = 0; h < G; ++h) {
-                    const float4 s = st[j * G + h];
-                    const float cb = expf(s.x - M[h]);
-                    Zs[h] += cb * s.y + (s.x < M[h] ? cb : 0.f);
-                    Zs[G + h] += s.x < M[h] ? 0.f : 1.f;
+                    const float4 s = stat(j, h);
+                    const bool top = !(s.x < M[h]);
+                    const float cb = top ? 1.f : expf(s.x - M[h]);
+                    Zs[h] += cb * s.y + (top ? 0.f : cb);
+                    Zs[G + h] += top ? 1.f : 0.f;
                 }
             block_reduce_sum<2 * G>(Zs, red);
-            float lZ[G], Hs[G];
+            float lZ[G], Z[G], Hs[G];
 #pragma unroll
             for (int h = 0; h < G; ++h) {
                 const float zm1 = Zs[h] + (Zs[G + h] - 1.f);
@@ -413,22 +462,19 @@ prune_finalize_kernel(const FinArgs a) {
                 Z[h] = 1.f + zm1;
                 Hs[h] = 0.f;
             }
-            // I_b per head; sum = attention entropy of the head
-            for (int j = j0; j < j1; ++j)
+            // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
+            auto Ib = [&](float4 s, int h) {
+                return expf(s.x - M[h]) * ((1.f + s.y) * (lZ[h] + M[h] - s.x) - s.z) / Z[h];
+            };
+            for (int j = k0; j < k1; ++j)
 #pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    const float4 s = st[j * G + h];
-                    const float I = expf(s.x - M[h]) * ((1.f + s.y) * (lZ[h] + M[h] - s.x) - s.z) / Z[h];
-                    Hs[h] += I;
-                }
+                for (int h = 0; h < G; ++h) Hs[h] += Ib(stat(j, h), h);
             block_reduce_sum<G>(Hs, red);
-            for (int j = j0; j < j1; ++j) {
+            for (int j = k0; j < k1; ++j) {
                 float best = -kInf;
 #pragma unroll
                 for (int h = 0; h < G; ++h) {
-                    const float4 s = st[j * G + h];
-                    const float I = expf(s.x - M[h]) * ((1.f + s.y) * (lZ[h] + M[h] - s.x) - s.z) / Z[h];
-                    const float nrm = Hs[h] > 0.f ? (float)n * I / Hs[h] : 1.f;
+                    const float nrm = Hs[h] > 0.f ? (float)n * Ib(stat(j, h), h) / Hs[h] : 1.f;
                     best = fmaxf(best, nrm);
                 }
                 sh_score[j] = best;
@@ -444,14 +490,12 @@ prune_finalize_kernel(const FinArgs a) {
         uint32_t kth = 0xffffffffu;   // keys > kth are selected; `rem` of those == kth
         int rem = 0;
         int arg = -1;                 // B_min == 1: the first block of highest score
-        if (k == n && n > 0) {
-            kth = 0u; rem = 0;        // every block
-        } else if (k == 1) {
+        if (k == 1 && n > 1) {
             float bs = -kInf;
             int bj = 0x7fffffff;
-            for (int j = j0; j < j1; ++j) {
+            for (int j = k0; j < k1; ++j) {
                 const float v = sh_score[j];
-                if (v > bs || (bj == 0x7fffffff)) { bs = v; bj = j; }
+                if (v > bs || bj == 0x7fffffff) { bs = v; bj = j; }
             }
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) {
@@ -469,14 +513,14 @@ prune_finalize_kernel(const FinArgs a) {
             __syncthreads();
             arg = sel_digit;
             __syncthreads();
-        } else if (k > 0) {
+        } else if (k > 1 && k < n) {
             uint32_t prefix = 0, mask = 0;
             int need = k;
             for (int digit = 3; digit >= 0; --digit) {
                 const int sh = digit * 8;
                 for (int i = tid; i < 256; i += nt) hist[i] = 0;
                 __syncthreads();
-                for (int j = j0; j < j1; ++j) {
+                for (int j = k0; j < k1; ++j) {
                     const uint32_t key = order_key(sh_score[j]);
                     if ((key & mask) == prefix) atomicAdd(&hist[(key >> sh) & 255], 1);
                 }
@@ -514,16 +558,15 @@ prune_finalize_kernel(const FinArgs a) {
         // flags: threshold or budget (ties at the k-th key go to the lower index)
         const float th = a.theta[b];
         int eq = 0;
-        for (int j = j0; j < j1; ++j) eq += (k > 1 && k < n && order_key(sh_score[j]) == kth);
+        for (int j = k0; j < k1; ++j) eq += (k > 1 && k < n && order_key(sh_score[j]) == kth);
         int eq_tot;
         int eq_rank = block_excl_scan(eq, ired, &eq_tot);
-        for (int j = j0; j < j1; ++j) {
-            const float s = sh_score[j];
-            const uint32_t key = order_key(s);
-            bool keep = s >= th;
-            if (k == n) keep = true;
-            else if (k == 1) keep |= (j == arg);
-            else if (k > 1) {
+        for (int j = k0; j < k1; ++j) {
+            const float sc = sh_score[j];
+            bool keep = sc >= th || k >= n;
+            if (k == 1) keep |= (j == arg);
+            else if (k > 1 && k < n) {
+                const uint32_t key = order_key(sc);
                 if (key > kth) keep = true;
                 else if (key == kth) { keep |= eq_rank < rem; ++eq_rank; }
             }
@@ -532,7 +575,7 @@ prune_finalize_kernel(const FinArgs a) {
         __syncthreads();
     } else {
         // given keep set
-        for (int j = j0; j < j1; ++j) sh_score[j] = 0.f;
+        for (int j = k0; j < k1; ++j) sh_score[j] = 0.f;
         __syncthreads();
         if (a.given_idx) {
             const int c = min(max(a.given_cnt[seg], 0), a.max_blocks);
@@ -541,17 +584,17 @@ prune_finalize_kernel(const FinArgs a) {
                 if (j >= 0 && j < n) sh_score[j] = 1.f;
             }
         } else {
-            for (int j = j0; j < j1; ++j) sh_score[j] = a.given_mask ? (a.given_mask[segbase + j] ? 1.f : 0.f) : 1.f;
+            for (int j = k0; j < k1; ++j) sh_score[j] = a.given_mask ? (a.given_mask[segbase + j] ? 1.f : 0.f) : 1.f;
         }
         __syncthreads();
     }
 
     // compaction (ascending block index)
     int cnt = 0;
-    for (int j = j0; j < j1; ++j) cnt += sh_score[j] != 0.f;
+    for (int j = k0; j < k1; ++j) cnt += sh_score[j] != 0.f;
     int total;
     int pos = block_excl_scan(cnt, ired, &total);
-    for (int j = j0; j < j1; ++j)
+    for (int j = k0; j < k1; ++j)
         if (sh_score[j] != 0.f) a.kept_idx[segbase + pos++] = j;
     for (int i = total + tid; i < a.max_blocks; i += nt) a.kept_idx[segbase + i] = -1;
     if (a.keep_mask)
@@ -563,19 +606,17 @@ prune_finalize_kernel(const FinArgs a) {
     if (a.kept_norm) {
         float Mk[G], Lk[G];
 #pragma unroll
-        for (int h = 0; h < G; ++h) Mk[h] = -kInf;
-        for (int j = j0; j < j1; ++j)
+        for (int h = 0; h < G; ++h) { Mk[h] = -kInf; Lk[h] = 0.f; }
+        for (int j = k0; j < k1; ++j)
             if (sh_score[j] != 0.f)
 #pragma unroll
-                for (int h = 0; h < G; ++h) Mk[h] = fmaxf(Mk[h], st[j * G + h].x);
+                for (int h = 0; h < G; ++h) Mk[h] = fmaxf(Mk[h], stat(j, h).x);
         block_reduce_max<G>(Mk, red);
-#pragma unroll
-        for (int h = 0; h < G; ++h) Lk[h] = 0.f;
-        for (int j = j0; j < j1; ++j)
+        for (int j = k0; j < k1; ++j)
             if (sh_score[j] != 0.f)
 #pragma unroll
                 for (int h = 0; h < G; ++h) {
-                    const float4 s = st[j * G + h];
+                    const float4 s = stat(j, h);
                     Lk[h] += (1.f + s.y) * expf(s.x - Mk[h]);
                 }
         block_reduce_sum<G>(Lk, red);
@@ -608,11 +649,12 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = 2 * sms;
-    const size_t smem = (size_t)(B + 1) * sizeof(int);
+    const size_t cum_bytes = ((size_t)(B + 1) * 4 + 15) & ~size_t(15);
     cudaError_t e;
 #define ETI_SCORE_CASE(DD, PP)                                                              \
     if (D == DD && P == PP) {                                                               \
         auto k = score_blocks_kernel<DD, PP>;                                               \
+        const size_t smem = cum_bytes;                                                      \
         if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
         k<<<grid, kScoreThreads, smem, stream>>>(a);                                        \
         e = cudaGetLastError();                                                             \
@@ -640,12 +682,16 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     a.given_idx = given_idx; a.given_cnt = given_cnt; a.keep_mask = keep_mask;
     a.kept_idx = kept_idx; a.kept_cnt = kept_cnt; a.block_score = block_score;
     a.kept_norm = kept_norm; a.err = err;
-    const size_t smem = (size_t)max_blocks * sizeof(float);
     const int grid = B * Hkv;
     cudaError_t e = cudaSuccess;
+    int dev = 0, optin = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
 #define ETI_FIN_CASE(GG)                                                                    \
     case GG: {                                                                              \
-        auto k = prune_finalize_kernel<GG>;                                                 \
+        const bool cache = fin_smem_bytes<GG>(max_blocks, true) <= (size_t)optin / 2;      \
+        const size_t smem = fin_smem_bytes<GG>(max_blocks, cache);                          \
+        auto k = cache ? prune_finalize_kernel<GG, true> : prune_finalize_kernel<GG, false>; \
         if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
         k<<<grid, kFinThreads, smem, stream>>>(a);                                          \
         e = cudaGetLastError();                                                             \

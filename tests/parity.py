@@ -40,8 +40,10 @@ def run_ets(eti, lg: dict, params=None, seed=0, offset=0, V=None):
                theta_next=torch.empty(B, dtype=f32, device=dev),
                surprisal=torch.empty(B, dtype=f32, device=dev),
                err=torch.empty(B, dtype=i32, device=dev))
+    ws = torch.empty(eti.entropy_temp_sample_workspace_size(B, V or lg["logits"].shape[1]),
+                     dtype=torch.uint8, device=dev)
     eti.eti_entropy_temp_sample(lg["logits"], lg["T_in"], lg["H_prev"], tau, lg["H_target"],
-                                out["tok"], out["H"], out["T_out"], out["err"], params=params,
+                                out["tok"], out["H"], out["T_out"], out["err"], ws, params=params,
                                 seed=seed, offset=offset, dH=out["dH"],
                                 theta_next=out["theta_next"], tok_surprisal=out["surprisal"], V=V)
     torch.cuda.synchronize()

@@ -65,15 +65,20 @@ def test_entropy_call_validation(lib):
     fake = P(256)
     prm = eti.ctrl_params()
     f = lib.eti_entropy_temp_sample
+    ws = lib.eti_entropy_temp_sample_workspace_size(4, 10)
+    assert ws > 0
     # bad shapes
-    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, NULL) == -2
-    assert f(fake, 4, 0, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, NULL) == -2
-    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, NULL) == -2
+    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -2
+    assert f(fake, 4, 0, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -2
+    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -2
     # B == 0 is a no-op
-    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, *[NULL] * 7, NULL) == 0
+    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, *[NULL] * 7, NULL, 0, NULL) == 0
     # required pointers
-    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, NULL) == -1
-    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, *[fake] * 7, NULL) == -1
+    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -1
+    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, *[fake] * 7, fake, ws, NULL) == -1
+    # workspace
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, NULL, ws, NULL) == -4
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws - 1, NULL) == -4
 
 
 def test_attention_call_validation(lib):
@@ -118,4 +123,4 @@ def test_binding_refuses_cpu_tensors(lib):
     with pytest.raises(eti.EtiError):
         eti.eti_entropy_temp_sample(x, x[:, 0], x[:, 0], x[:, 0], x[:, 0],
                                     torch.zeros(2, dtype=torch.int32), x[:, 0], x[:, 0],
-                                    torch.zeros(2, dtype=torch.int32))
+                                    torch.zeros(2, dtype=torch.int32), torch.zeros(64, dtype=torch.uint8))
