@@ -71,6 +71,8 @@ typedef uint16_t eti_bf16;
 #define ETI_ERR_WORKSPACE   (-4)  /* ws is NULL or smaller than *_workspace_size() */
 #define ETI_ERR_CUDA        (-5)  /* a kernel launch failed (cudaGetLastError) */
 #define ETI_ERR_ALIGN       (-6)  /* a bf16 tensor is not 16-byte aligned */
+#define ETI_ERR_TOO_LARGE   (-7)  /* the problem needs more than the fixed scratch of
+                                     eti_entropy_temp_sample_noalloc */
 
 /* per-sequence data error bits written to err_flags */
 #define ETI_ERRF_BAD_PAGE     0x1u  /* a block_table entry is outside [0, num_pages) */
@@ -143,6 +145,41 @@ int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
                             int32_t* tok, float* H, float* T_out,
                             float* dH, float* theta_next, float* tok_surprisal,
                             uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * eti_entropy_temp_sample_noalloc -- the same computation, arguments and
+ * results as eti_entropy_temp_sample, for callers that cannot allocate
+ * device memory at all: code that is handed only its input and output
+ * buffers by a host framework that owns every device allocation (a plugin
+ * or callback with no workspace argument and no allocator to ask), or a
+ * latency-critical host thread that must never enter the CUDA allocator.
+ * The paper has no counterpart; this is a deployment convenience.
+ *
+ * Instead of a workspace, the call uses a fixed scratch array compiled into
+ * this library (eti_entropy_temp_sample_noalloc_max_bytes() bytes, one copy
+ * on every GPU that loads the library, kept until the process exits).  It
+ * never calls cudaMalloc, cudaFree or any allocating routine.
+ *  - The first call on a device looks up that array's device address
+ *    (cudaGetSymbolAddress) with the device current, once per device; make
+ *    that first call before any stream capture.
+ *  - Every call on a device shares the one array and it keeps the previous
+ *    call's contents; nothing in it needs to start at zero, because every
+ *    entry a call reads was written earlier by the same call.  Calls whose
+ *    execution overlaps on the GPU (other streams, or several host threads)
+ *    race on the array: serialise them.
+ *  - A problem whose scratch (eti_entropy_temp_sample_workspace_size(B, V))
+ *    exceeds the array returns ETI_ERR_TOO_LARGE and enqueues nothing; at
+ *    152 SMs the limit is about 10,300 sequences, whatever V is.
+ */
+size_t eti_entropy_temp_sample_noalloc_max_bytes(void);
+
+int eti_entropy_temp_sample_noalloc(const float* logits, int B, int V, int64_t ld,
+                                    const float* T_in, const float* H_prev, float* tau,
+                                    const float* H_target, const eti_ctrl_params* params,
+                                    uint64_t seed, uint64_t offset,
+                                    int32_t* tok, float* H, float* T_out,
+                                    float* dH, float* theta_next, float* tok_surprisal,
+                                    uint32_t* err_flags, void* stream);
 
 /*
  * eti_score_prune_blocks -- the entropic keep set of half (b).

@@ -22,7 +22,8 @@ _lib = None
 
 ETI_OK = 0
 STATUS = {0: "ok", -1: "null pointer", -2: "bad shape", -3: "unsupported shape",
-          -4: "workspace too small", -5: "CUDA launch failed", -6: "misaligned tensor"}
+          -4: "workspace too small", -5: "CUDA launch failed", -6: "misaligned tensor",
+          -7: "too large for the fixed scratch"}
 ERRF_BAD_PAGE, ERRF_BAD_CTX, ERRF_NONFINITE, ERRF_ALL_NEG_INF, ERRF_BAD_TEMP = 1, 2, 4, 8, 16
 
 # C-ABI symbols declared in include/eti.h
@@ -30,7 +31,8 @@ SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_entropy_temp_sam
            "eti_score_prune_workspace_size",
            "eti_score_prune_blocks", "eti_score_blocks", "eti_prune_blocks",
            "eti_paged_decode_workspace_size", "eti_paged_decode", "eti_version",
-           "eti_status_string")
+           "eti_status_string", "eti_entropy_temp_sample_noalloc",
+           "eti_entropy_temp_sample_noalloc_max_bytes")
 
 
 class EtiError(RuntimeError):
@@ -69,6 +71,10 @@ def load(path: str | None = None):
         lib.eti_entropy_temp_sample_workspace_size.restype = sz
         lib.eti_entropy_temp_sample.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64,
                                                 P, P, P, P, P, P, P, P, sz, P]
+        lib.eti_entropy_temp_sample_noalloc.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64,
+                                                        P, P, P, P, P, P, P, P]
+        lib.eti_entropy_temp_sample_noalloc.restype = i32
+        lib.eti_entropy_temp_sample_noalloc_max_bytes.restype = sz
         lib.eti_entropy_temp_sample.restype = i32
         lib.eti_score_prune_workspace_size.argtypes = [i32] * 6
         lib.eti_score_prune_workspace_size.restype = sz
@@ -151,6 +157,28 @@ def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, 
         _dev(tok_surprisal, "tok_surprisal", f32, B), _dev(err_flags, "err_flags", torch.int32, B),
         _dev(ws, "ws", torch.uint8), ws.numel() if ws is not None else 0, _stream(stream))
     _check(st, "eti_entropy_temp_sample")
+
+
+def eti_entropy_temp_sample_noalloc(logits, T_in, H_prev, tau, H_target, tok, H, T_out, err_flags,
+                                    params: CtrlParams | None = None, seed: int = 0,
+                                    offset: int = 0, dH=None, theta_next=None, tok_surprisal=None,
+                                    V: int | None = None, stream=None):
+    """eti_entropy_temp_sample without a workspace (fixed library scratch); see include/eti.h."""
+    B, ld = logits.shape
+    V = ld if V is None else int(V)
+    if logits.stride(1) != 1 or logits.stride(0) != ld:
+        raise EtiError("logits must be a row-major [B, ld] tensor")
+    f32, i32 = torch.float32, torch.int32
+    params = params or ctrl_params()
+    st = load().eti_entropy_temp_sample_noalloc(
+        _dev(logits, "logits", f32), B, V, ld, _dev(T_in, "T_in", f32, B),
+        _dev(H_prev, "H_prev", f32, B), _dev(tau, "tau", f32, B), _dev(H_target, "H_target", f32, B),
+        ctypes.byref(params), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+        _dev(tok, "tok", i32, B), _dev(H, "H", f32, B), _dev(T_out, "T_out", f32, B),
+        _dev(dH, "dH", f32, B), _dev(theta_next, "theta_next", f32, B),
+        _dev(tok_surprisal, "tok_surprisal", f32, B), _dev(err_flags, "err_flags", torch.int32, B),
+        _stream(stream))
+    _check(st, "eti_entropy_temp_sample_noalloc")
 
 
 def _attn_shapes(q, k_cache, block_table):

@@ -114,6 +114,7 @@ const char* eti_status_string(int s) {
         case ETI_ERR_WORKSPACE: return "workspace missing or too small";
         case ETI_ERR_CUDA: return "CUDA launch failed";
         case ETI_ERR_ALIGN: return "a bf16 tensor is not 16-byte aligned";
+        case ETI_ERR_TOO_LARGE: return "problem exceeds the fixed scratch of the no-allocation entry point";
         default: return "unknown status";
     }
 }

@@ -30,6 +30,8 @@
 //                the Taylor series of -log(1 - v), whose remainder is below
 //                v^6/7 < 2^-24 / 7 relative.
 // u = (2 (word & 0x7FFFFF) + 1) / 2^24 is formed exactly as 1.m - (1 - 2^-24).
+#include <mutex>
+
 #include "common.cuh"
 
 namespace eti {
@@ -372,4 +374,60 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
     if (cudaGetLastError() != cudaSuccess) return ETI_ERR_CUDA;
     entropy_sample_finalize_kernel<<<(B + 3) / 4, 128, 0, stream>>>(a);
     return cudaGetLastError() == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
+}
+
+// ---------------------------------------------------------------------------
+// eti_entropy_temp_sample_noalloc: the same computation with its scratch in a
+// fixed array of this library instead of a caller workspace (see eti.h).
+
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = 256 * 1024;
+constexpr int kNoAllocMaxDevices = 64;
+
+// One copy per device that loads the library; it lives until the process exits.
+static __device__ __align__(256) unsigned char g_ets_scratch[kNoAllocScratchBytes];
+
+std::mutex g_ets_scratch_mu;
+void* g_ets_scratch_ptr[kNoAllocMaxDevices] = {};
+
+// Device address of g_ets_scratch on the current device, looked up once per
+// device (the host-side name of the array is not a device address).
+int ets_scratch_address(void** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return ETI_ERR_CUDA;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return ETI_ERR_UNSUPPORTED;
+    std::lock_guard<std::mutex> lock(g_ets_scratch_mu);
+    if (!g_ets_scratch_ptr[dev]) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_ets_scratch) != cudaSuccess || !p) return ETI_ERR_CUDA;
+        g_ets_scratch_ptr[dev] = p;
+    }
+    *out = g_ets_scratch_ptr[dev];
+    return ETI_OK;
+}
+
+}  // namespace
+
+extern "C" size_t eti_entropy_temp_sample_noalloc_max_bytes(void) { return kNoAllocScratchBytes; }
+
+extern "C" int eti_entropy_temp_sample_noalloc(const float* logits, int B, int V, int64_t ld,
+                                               const float* T_in, const float* H_prev, float* tau,
+                                               const float* H_target, const eti_ctrl_params* params,
+                                               uint64_t seed, uint64_t offset,
+                                               int32_t* tok, float* H, float* T_out,
+                                               float* dH, float* theta_next, float* tok_surprisal,
+                                               uint32_t* err_flags, void* stream) {
+    if (B < 0 || B > 65535 || V < 1 || ld < V) return ETI_ERR_SHAPE;
+    if (B == 0) return ETI_OK;
+    if (!logits || !T_in || !H_prev || !tau || !H_target || !params || !tok || !H || !T_out ||
+        !err_flags)
+        return ETI_ERR_NULL;
+    if (eti_entropy_partial_bytes(B) > kNoAllocScratchBytes) return ETI_ERR_TOO_LARGE;
+    void* scratch = nullptr;
+    const int st = ets_scratch_address(&scratch);
+    if (st != ETI_OK) return st;
+    return eti_launch_entropy_temp_sample(logits, B, V, (long long)ld, T_in, H_prev, tau, H_target,
+                                          params, seed, offset, tok, H, T_out, dH, theta_next,
+                                          tok_surprisal, err_flags, scratch, (cudaStream_t)stream);
 }
