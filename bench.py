@@ -10,7 +10,8 @@ The workload is the Llama-3-8B-shaped layer step (64 sequences, 32 query /
 vocabulary 128,256) with seeded synthetic inputs.
 
 Prints ONE JSON line (rank 0).  Timing: W warm-up steps, then K timed steps;
-before every step a buffer of twice the L2 size is written (L2 flush); each
+before every step a buffer of twice the L2 size is written and another one
+read (L2 flush, write-backs settled outside the timed region); each
 kernel call is bracketed by CUDA events on the launching stream and the step
 time is the sum of its calls.  `value` = sequences decoded per second per
 layer step over all ranks (each rank decodes its own batch: weak scaling).
@@ -179,7 +180,15 @@ def run_gpu(args):
     B_min = 1
     stream = torch.cuda.current_stream()
     L2 = torch.cuda.get_device_properties(device).L2_cache_size
-    flush = torch.empty(max(2 * L2, 256 << 20), dtype=torch.uint8, device=device)
+    flush_w = torch.empty(max(2 * L2, 256 << 20), dtype=torch.uint8, device=device)
+    flush_r = torch.ones(max(2 * L2, 256 << 20) // 4, dtype=torch.int32, device=device)
+
+    def flush_l2():
+        """Write a buffer of 2x L2, then read another one: the step's data is
+        evicted and the flush's own dirty lines are written back before the
+        timed region instead of inside its first kernel."""
+        flush_w.zero_()
+        flush_r.sum()
 
     def one_step(ev=None, offset=0):
         if ev is not None:
@@ -206,7 +215,7 @@ def run_gpu(args):
             ev[4].record(stream)
 
     for i in range(args.warmup):
-        flush.zero_()
+        flush_l2()
         one_step(offset=i)
     torch.cuda.synchronize()
     kept = int(step.kept_cnt.sum().item())
@@ -222,7 +231,7 @@ def run_gpu(args):
     with ClockSampler(local, clock_log) as clk:
         t0 = time.perf_counter()
         for i in range(args.steps):
-            flush.zero_()
+            flush_l2()
             one_step(evs[i], offset=args.warmup + i)
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
@@ -264,7 +273,7 @@ def run_gpu(args):
         "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
         "config": {"workload": f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} D={w.D} P={w.P} "
                                f"ctx U[{w.ctx[1]},{w.ctx[2]}] V={w.V}",
-                   "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write)",
+                   "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write, then 2x L2 read)",
                    "parallelism": f"replicas x{world} (independent batches)", "B_min": B_min,
                    "theta": "theta_next of the step's own entropy (defaults)",
                    "kept_fraction": round(kept / total_blocks, 4)},
