@@ -35,7 +35,8 @@
  *  - Supported shapes: head_dim D in {64, 128}; page size P in {16, 32};
  *    Hq % Hkv == 0 with group size g = Hq / Hkv <= 8; 1 <= max_blocks <= 32768;
  *    B <= 65535 (entropy/sample) or 8192 (attention calls); 1 <= V.
- *    q, k_cache, v_cache and the decode output must be 16-byte aligned.
+ *    q, k_cache, v_cache, token_scores and the decode output must be 16-byte
+ *    aligned.
  *
  * Layouts
  *  - q          bf16  [B][Hq][D]
@@ -80,6 +81,8 @@ typedef uint16_t eti_bf16;
 #define ETI_ERRF_NONFINITE    0x4u  /* a logit is NaN or +inf */
 #define ETI_ERRF_ALL_NEG_INF  0x8u  /* every logit of the row is -inf */
 #define ETI_ERRF_BAD_TEMP     0x10u /* T_in is not a positive finite number */
+#define ETI_ERRF_TIMEOUT      0x20u /* a device-side wait for a tile copy gave up (the
+                                       sequence's results are not valid) */
 
 /*
  * Controller parameters (Section 3.3 temperature law, Section 3.2 safety

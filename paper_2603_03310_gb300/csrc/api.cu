@@ -31,6 +31,35 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
                       cudaStream_t stream);
 int eti_decode_nwarps();
 
+// cuTensorMapEncodeTiled, fetched from the driver at first use (no link
+// dependency on libcuda).
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+int eti_make_kv_tensor_map(CUtensorMap* map, const void* base, long long rows, int D) {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !p)
+            return ETI_ERR_CUDA;
+        fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    if (rows <= 0 || (rows >> 32) != 0) return ETI_ERR_SHAPE;
+    const cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+    const cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+    const cuuint32_t box[2] = {64, 16};
+    const cuuint32_t estr[2] = {1, 1};
+    const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims,
+                          strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? ETI_OK : ETI_ERR_CUDA;
+}
+
 namespace {
 
 constexpr int kMaxB = 8192;
@@ -80,7 +109,7 @@ DecodeWs carve_decode(void* ws, int B, int Hq, int Hkv, int D, int P, int max_bl
         w.knorm = c.take<float>((size_t)B * Hq * 2);
     }
     w.cum = c.take<int>(nseg + 1);
-    w.info = c.take<int>(4);
+    w.info = c.take<int>(4);   // total kept blocks, share per warp, timeout flag
     w.warp_seg = c.take<int>(nwarps);
     w.partial = c.take<float>(((size_t)nwarps + nseg) * g * D);
     *bytes = c.off;
@@ -234,7 +263,7 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
     const bool have_scores = token_scores && kept_norm && have_lists;
     if (!v_cache || !block_table || !ctx_lens || !out || !err_flags) return ETI_ERR_NULL;
     if (!have_scores && (!q || !k_cache)) return ETI_ERR_NULL;
-    if (!aligned16(v_cache) || !aligned16(out) ||
+    if (!aligned16(v_cache) || !aligned16(out) || (have_scores && !aligned16(token_scores)) ||
         (!have_scores && (!aligned16(q) || !aligned16(k_cache))))
         return ETI_ERR_ALIGN;
     const int nwarps = eti_decode_nwarps();

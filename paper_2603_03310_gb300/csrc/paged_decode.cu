@@ -11,16 +11,20 @@
 //
 // Work split (warp-level stream-K): the kept blocks of all (sequence, kv head)
 // segments form one list; warp w takes the contiguous range
-// [w*share, (w+1)*share).  Each warp loads its 16-token tiles straight into
-// registers with 128-bit loads, one tile ahead of use, and keeps a deeper
-// stream in flight with bulk L2 prefetches (one instruction per kept V chunk)
-// a few blocks further ahead.  Page ids are resolved 32 blocks at a time, one
-// lane per block, a batch ahead of use.  p.V runs on bf16 m16n8k16 tensor-core tiles
+// [w*share, (w+1)*share).  Each warp streams its 16-token tiles through a
+// private ring of shared-memory stages filled by the Tensor Memory
+// Accelerator: one elected lane issues two 2-D tiled copies (64-element boxes
+// with the 128-byte swizzle, so the fragment reads below are conflict-free)
+// and a 1-D bulk copy of the tile's scores per stage, completing on the
+// stage's mbarrier; every wait is bounded.  Page ids are resolved 32 blocks at
+// a time, one lane per block, into a small table a batch ahead of use.  p.V runs on bf16 m16n8k16 tensor-core tiles
 // (head_dim = M, query heads = N, tokens = K): V rows are transposed into A
 // fragments with byte permutes, the probabilities form the B fragment.
 // A segment that lies inside one warp's range is written straight to `out`;
 // otherwise the warp's part goes to partial slot (warp + segment) and the
 // combine kernel adds the slots in warp order (deterministic).
+#include <cstring>
+
 #include "common.cuh"
 
 namespace eti {
@@ -69,6 +73,7 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
         a.cum[a.nseg] = total;
         a.info[0] = total;
         a.info[1] = share;
+        a.info[2] = 0;      // set by the decode kernel if a tile copy never arrived
     }
     for (int c = tid; c < a.nwarps; c += kPlanThreads) a.warp_seg[c] = a.nseg;
     __syncthreads();
@@ -97,13 +102,20 @@ struct DecArgs {
     float* partial;                // [(nwarps + nseg)][g][D]
 };
 
-constexpr int kDecPrefetch = 6;    // kept blocks prefetched into L2 ahead of the loads
-
 template <int D>
 struct DecLayout {
     static constexpr int E = D / 16;              // bf16 per row half per thread
+    static constexpr int kTile = 16 * D * 2;      // bytes of one 16-token V tile
+    static constexpr int kScores = 16 * 8 * 4;    // room for one tile's scores (g <= 8)
+    static constexpr int kStages = D == 128 ? 3 : 5;
     using Vec = typename std::conditional<E == 8, uint4, uint2>::type;
 };
+
+template <int D>
+__host__ __device__ constexpr size_t dec_smem_bytes() {
+    return 1024 + (size_t)kDecWarps * DecLayout<D>::kStages * (DecLayout<D>::kTile + DecLayout<D>::kScores + 8)
+           + (size_t)kDecWarps * 64 * 16;
+}
 
 template <int D>
 __device__ __forceinline__ uint32_t vreg(const typename DecLayout<D>::Vec& v, int i) {
@@ -122,10 +134,18 @@ __device__ __forceinline__ uint32_t pair_elem(const typename DecLayout<D>::Vec& 
     return (j & 1) ? hi_halves(x, y) : lo_halves(x, y);
 }
 
+// A-fragment rows owned by a thread (tq = lane & 3): 2tq, 2tq+1, 2tq+8, 2tq+9
+__device__ __forceinline__ int frag_row(int tq, int k) { return 2 * tq + (k & 1) + (k >> 1) * 8; }
+
+// The thread's E elements of row `row`, half `half` (d = half * D/2 + E * grp),
+// from a 128-byte-swizzled tile (one 2 KB box per 64-element half for D = 128).
 template <int D>
-__device__ __forceinline__ typename DecLayout<D>::Vec ld_vec(const uint16_t* p) {
-    if constexpr (DecLayout<D>::E == 8) return ldg_stream_u4(p);
-    else return ldg_stream_u2(p);
+__device__ __forceinline__ typename DecLayout<D>::Vec lds_row(uint32_t tile, int row, int half, int grp) {
+    if constexpr (D == 128) {
+        return lds_u4(tile + half * 2048 + swz128(row, grp));
+    } else {
+        return lds_u2(tile + swz128(row, 4 * half + (grp >> 1)) + (grp & 1) * 8);
+    }
 }
 
 template <int D>
@@ -136,27 +156,18 @@ __device__ __forceinline__ typename DecLayout<D>::Vec zero_vec() {
     return z;
 }
 
-// A-fragment rows owned by a thread (tq = lane & 3): 2tq, 2tq+1, 2tq+8, 2tq+9
-__device__ __forceinline__ int frag_row(int tq, int k) { return 2 * tq + (k & 1) + (k >> 1) * 8; }
-
-// one block of the warp's range, resolved by one lane
-struct ItemInfo {
-    int seg, blk, page, vtok;
-};
-
-template <int D>
-struct VTile {
-    typename DecLayout<D>::Vec r[4][2];   // rows 2t, 2t+1, 2t+8, 2t+9; halves
-    float x[4];                           // their scores for head grp
-    int seg;
-};
-
 template <int D, int P>
-__global__ void __launch_bounds__(kDecThreads, 1)
-paged_decode_kernel(const DecArgs a) {
+__global__ void __launch_bounds__(kDecThreads, 2)
+paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
     using LY = DecLayout<D>;
     constexpr int kTiles = P / 16;
     constexpr int J = D / 16;                    // MMAs per 16-token tile
+    constexpr int S = LY::kStages;
+    constexpr int TB = LY::kTile;
+    constexpr int SB = LY::kScores;
+    constexpr int H = D / 64;                    // 64-element boxes per tile row
+    extern __shared__ __align__(1024) unsigned char dec_smem_raw[];
+    unsigned char* dec_smem = dec_smem_raw + ((1024 - (smem_u32(dec_smem_raw) & 1023)) & 1023);
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5, grp = lane >> 2, tq = lane & 3;
     const int warp = blockIdx.x * kDecWarps + wl;
     const int total = a.info[0], share = a.info[1];
@@ -165,14 +176,28 @@ paged_decode_kernel(const DecArgs a) {
     if (u0 >= u1) return;
     const int nseg = a.B * a.Hkv;
     const int ntiles = (u1 - u0) * kTiles;
+    const uint32_t tiles = smem_u32(dec_smem) + wl * S * TB;
+    const uint32_t scores = smem_u32(dec_smem) + kDecWarps * S * TB + wl * S * SB;
+    const uint32_t bars = smem_u32(dec_smem) + kDecWarps * S * (TB + SB) + wl * S * 8;
+    int4* table = reinterpret_cast<int4*>(dec_smem + kDecWarps * S * (TB + SB + 8)) + wl * 64;
+    const int sbytes = 16 * a.g * 4;             // one tile's scores (a multiple of 16)
 
-    auto resolve = [&](int base, int seg_hint) -> ItemInfo {
-        ItemInfo it{seg_hint, 0, -1, 0};
-        const int u = base + lane;
+    if (lane == 0) {
+        for (int st = 0; st < S; ++st) mbar_init(bars + 8 * st, 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+
+    // items [u0 + 32k, u0 + 32k + 32) -> table slot k & 1: (segment, block,
+    // page or -1, valid tokens of the block)
+    int seg_hint = a.warp_seg[warp];
+    auto resolve = [&](int k) {
+        const int u = u0 + 32 * k + lane;
+        int4 e = make_int4(seg_hint, 0, -1, 0);
         if (u < u1) {
             int s = seg_hint;
             while (s < nseg - 1 && __ldg(a.cum + s + 1) <= u) ++s;
-            it.seg = s;
+            e.x = s;
             const int b = s / a.Hkv;
             const int L = __ldg(a.ctx_lens + b);
             const int nb = seq_blocks(L, P, a.max_blocks);
@@ -180,61 +205,40 @@ paged_decode_kernel(const DecArgs a) {
             if (blk >= 0 && blk < nb) {
                 const int pg = __ldg(a.block_table + (long long)b * a.max_blocks + blk);
                 if (pg >= 0 && (long long)pg < a.num_pages) {
-                    it.blk = blk;
-                    it.page = pg;
-                    it.vtok = min(P, L - blk * P);
+                    e.y = blk;
+                    e.z = pg;
+                    e.w = min(P, L - blk * P);
                 }
             }
         }
-        return it;
+        table[(k & 1) * 32 + lane] = e;
+        seg_hint = __shfl_sync(0xffffffffu, e.x, 31);
+        __syncwarp();
     };
-
-    ItemInfo cur = resolve(u0, a.warp_seg[warp]);
-    int cbase = u0;
-    ItemInfo nxt = resolve(u0 + 32, __shfl_sync(0xffffffffu, cur.seg, 31));
-    auto item_at = [&](int off) -> ItemInfo {
-        const int l = off & 31;
-        ItemInfo a0, a1;
-        a0.seg = __shfl_sync(0xffffffffu, cur.seg, l);   a1.seg = __shfl_sync(0xffffffffu, nxt.seg, l);
-        a0.blk = __shfl_sync(0xffffffffu, cur.blk, l);   a1.blk = __shfl_sync(0xffffffffu, nxt.blk, l);
-        a0.page = __shfl_sync(0xffffffffu, cur.page, l); a1.page = __shfl_sync(0xffffffffu, nxt.page, l);
-        a0.vtok = __shfl_sync(0xffffffffu, cur.vtok, l); a1.vtok = __shfl_sync(0xffffffffu, nxt.vtok, l);
-        return off < 32 ? a0 : a1;
+    auto entry = [&](int item) -> int4 {
+        const int r = item - u0;
+        return table[((r >> 5) & 1) * 32 + (r & 31)];
     };
-    auto v_chunk = [&](const ItemInfo& it) {
-        const int kvh = it.seg - (it.seg / a.Hkv) * a.Hkv;
-        return a.v_cache + ((long long)(it.page >= 0 ? it.page : 0) * a.Hkv + kvh) * P * D;
-    };
-    auto s_chunk = [&](const ItemInfo& it) {
-        return a.token_scores + ((long long)it.seg * a.max_blocks + it.blk) * P * a.g;
-    };
-    auto prefetch = [&](const ItemInfo& it) {
-        if (lane == 0 && it.page >= 0) {
-            prefetch_l2_bulk(v_chunk(it), P * D * 2);
-            if (((P * a.g * 4) & 15) == 0) prefetch_l2_bulk(s_chunk(it), P * a.g * 4);
-        }
-    };
-    auto load_tile = [&](VTile<D>& t, const ItemInfo& it, int tile) {
-        const uint16_t* vt = v_chunk(it) + tile * 16 * D;
-        const float* sc = s_chunk(it) + tile * 16 * a.g;
-        const bool ok = it.page >= 0;
+    auto issue = [&](int i, int st) {
+        if (lane == 0) {
+            const int item = u0 + i / kTiles;
+            const int tile = i - (i / kTiles) * kTiles;
+            const int4 e = entry(item);
+            const uint32_t bar = bars + 8 * st;
+            if (e.z >= 0) {
+                const int kvh = e.x - (e.x / a.Hkv) * a.Hkv;
+                mbar_arrive_expect_tx(bar, TB + sbytes);
+                const int y = (e.z * a.Hkv + kvh) * P + tile * 16;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            const int row = frag_row(tq, k);
-            if (ok && tile * 16 + row < it.vtok) {
-                t.r[k][0] = ld_vec<D>(vt + row * D + LY::E * grp);
-                t.r[k][1] = ld_vec<D>(vt + row * D + D / 2 + LY::E * grp);
-                t.x[k] = grp < a.g ? __ldg(sc + row * a.g + grp) : 0.f;
+                for (int h = 0; h < H; ++h) tma_load_2d(tiles + st * TB + h * 2048, &vmap, 64 * h, y, bar);
+                bulk_load_1d(scores + st * SB,
+                             a.token_scores + (((long long)e.x * a.max_blocks + e.y) * P + tile * 16) * a.g,
+                             sbytes, bar);
             } else {
-                t.r[k][0] = zero_vec<D>();
-                t.r[k][1] = zero_vec<D>();
-                t.x[k] = 0.f;
+                mbar_arrive(bar);
             }
         }
-        t.seg = it.seg;
     };
-
-    for (int k = 0; k < kDecPrefetch && u0 + k < u1; ++k) prefetch(item_at(k));
 
     float acc[J][4];
 #pragma unroll
@@ -278,56 +282,69 @@ paged_decode_kernel(const DecArgs a) {
         for (int j = 0; j < J; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
     };
 
+    resolve(0);
+    if (u1 - u0 > 32) resolve(1);
+#pragma unroll 1
+    for (int st = 0; st < S && st < ntiles; ++st) issue(st, st);
+
     int cur_seg = -1;
     float Mh = 0.f;
-    // consume one tile: probabilities (B fragment) and p.V on the tensor cores
-    auto consume = [&](const VTile<D>& t) {
-        if (t.seg != cur_seg) {
+    int i = 0;
+    bool timed_out = false;
+#pragma unroll 1
+    for (; i < ntiles; ++i) {
+        const int st = i % S;
+        const int item = u0 + i / kTiles;
+        const int tile = i - (i / kTiles) * kTiles;
+        if (tile == 0 && ((item - u0) & 31) == 0 && item > u0 && item - u0 + 32 < u1 - u0)
+            resolve(((item - u0) >> 5) + 1);
+        if (!mbar_wait(bars + 8 * st, (uint32_t)((i / S) & 1), kMaxWaitIters)) {
+            timed_out = true;
+            break;
+        }
+        const int4 e = entry(item);
+        if (e.x != cur_seg) {
             if (cur_seg >= 0) flush(cur_seg);
-            cur_seg = t.seg;
+            cur_seg = e.x;
             const int b = cur_seg / a.Hkv, kvh = cur_seg - b * a.Hkv;
             Mh = grp < a.g ? __ldg(a.kept_norm + ((long long)b * a.Hq + kvh * a.g + grp) * 2) : 0.f;
         }
+        const uint32_t tb = tiles + st * TB, sc = scores + st * SB;
+        const int vrow = e.z >= 0 ? e.w - tile * 16 : 0;   // valid rows of this tile
+        typename LY::Vec r[4][2];
         float p[4];
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-            // kept tokens have x <= M_h; zeroed rows (past the end, or a padded
-            // head) get weight 1 against a zero V row
-            p[k] = fast_ex2(fminf((t.x[k] - Mh) * kLog2e, 0.f));
+        for (int k = 0; k < 4; ++k) {
+            const int row = frag_row(tq, k);
+            const bool ok = row < vrow;
+            // rows past the sequence end hold whatever the page holds: zero them
+            r[k][0] = ok ? lds_row<D>(tb, row, 0, grp) : zero_vec<D>();
+            r[k][1] = ok ? lds_row<D>(tb, row, 1, grp) : zero_vec<D>();
+            const float x = (ok && grp < a.g) ? lds_f32(sc + (row * a.g + grp) * 4) : 0.f;
+            // kept tokens have x <= M_h; zeroed rows get a finite weight against a zero row
+            p[k] = fast_ex2(fminf((x - Mh) * kLog2e, 0.f));
+        }
+        // the stage may be refilled now
+        __syncwarp();
+        fence_proxy_async();
+        if (i + S < ntiles) issue(i + S, st);
         const uint32_t b0 = pack_bf16x2(p[0], p[1]);
         const uint32_t b1 = pack_bf16x2(p[2], p[3]);
 #pragma unroll
         for (int j = 0; j < J; ++j) {
-            const uint32_t a0 = pair_elem<D>(t.r[0][0], t.r[1][0], j);
-            const uint32_t a1 = pair_elem<D>(t.r[0][1], t.r[1][1], j);
-            const uint32_t a2 = pair_elem<D>(t.r[2][0], t.r[3][0], j);
-            const uint32_t a3 = pair_elem<D>(t.r[2][1], t.r[3][1], j);
+            const uint32_t a0 = pair_elem<D>(r[0][0], r[1][0], j);
+            const uint32_t a1 = pair_elem<D>(r[0][1], r[1][1], j);
+            const uint32_t a2 = pair_elem<D>(r[2][0], r[3][0], j);
+            const uint32_t a3 = pair_elem<D>(r[2][1], r[3][1], j);
             mma_bf16_16x8x16(acc[j], a0, a1, a2, a3, b0, b1);
         }
-    };
-
-    // next tile i + 1: load it (and prefetch further ahead into L2)
-    auto advance = [&](VTile<D>& t, int i) {
-        const int item = u0 + i / kTiles;
-        const int tile = i - (i / kTiles) * kTiles;
-        if (item >= cbase + 32) {
-            cur = nxt;
-            cbase += 32;
-            nxt = resolve(cbase + 32, __shfl_sync(0xffffffffu, cur.seg, 31));
-        }
-        load_tile(t, item_at(item - cbase), tile);
-        if (tile == 0 && item + kDecPrefetch < u1) prefetch(item_at(item + kDecPrefetch - cbase));
-    };
-
-    VTile<D> t0, t1;
-    load_tile(t0, item_at(0), 0);
-    for (int i = 0; i < ntiles; i += 2) {
-        if (i + 1 < ntiles) advance(t1, i + 1);
-        consume(t0);
-        if (i + 1 < ntiles) {
-            if (i + 2 < ntiles) advance(t0, i + 2);
-            consume(t1);
-        }
+    }
+    if (timed_out) {
+        // a copy never arrived: let the ones in flight land (bounded) and
+        // report it; the combine pass flags every sequence of the call
+        for (int k = i; k < ntiles && k < i + S; ++k) mbar_wait(bars + 8 * (k % S), (uint32_t)((k / S) & 1), 1024);
+        if (lane == 0) atomicOr(const_cast<int*>(a.info) + 2, 1);
+        return;
     }
     if (cur_seg >= 0) flush(cur_seg);
 }
@@ -362,7 +379,8 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const CombArgs a) {
     }
     const bool bad_page = __syncthreads_or(bad) != 0;
     if (a.err && kvh == 0 && tid == 0)
-        a.err[b] = bad_ctx ? ETI_ERRF_BAD_CTX : (bad_page ? ETI_ERRF_BAD_PAGE : 0u);
+        a.err[b] = (bad_ctx ? ETI_ERRF_BAD_CTX : (bad_page ? ETI_ERRF_BAD_PAGE : 0u)) |
+                   (a.info[2] ? ETI_ERRF_TIMEOUT : 0u);
     const int lo = a.cum[s], hi = a.cum[s + 1];
     const int share = a.info[1];
     uint16_t* o = a.out + ((long long)b * a.Hq + kvh * a.g) * a.D;
@@ -390,7 +408,7 @@ int eti_decode_nwarps() {
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    return sms * kDecWarps;
+    return 2 * sms * kDecWarps;
 }
 
 int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const int32_t* ctx_lens,
@@ -414,10 +432,23 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
     da.B = B; da.Hq = Hq; da.Hkv = Hkv; da.g = Hq / Hkv; da.max_blocks = max_blocks;
     da.num_pages = num_pages; da.out = out; da.partial = partial;
     const int grid = nwarps / kDecWarps;
+    if (num_pages <= 0 || num_pages * Hkv * P >= (1LL << 31)) {
+        if (num_pages > 0) return ETI_ERR_UNSUPPORTED;   // tile rows are int32 on the device
+    }
+    CUtensorMap vmap;
+    if (num_pages > 0) {
+        const int st = eti_make_kv_tensor_map(&vmap, v_cache, num_pages * Hkv * P, D);
+        if (st != ETI_OK) return st;
+    } else {
+        memset(&vmap, 0, sizeof(vmap));   // no page is valid: the kernel issues no copy
+    }
     bool launched = false;
 #define ETI_DEC_CASE(DD, PP)                                                              \
     if (!launched && D == DD && P == PP) {                                                \
-        paged_decode_kernel<DD, PP><<<grid, kDecThreads, 0, stream>>>(da);                \
+        auto k = paged_decode_kernel<DD, PP>;                                             \
+        const size_t sm = dec_smem_bytes<DD>();                                           \
+        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);    \
+        k<<<grid, kDecThreads, sm, stream>>>(vmap, da);                                   \
         launched = true;                                                                  \
     }
     ETI_DEC_CASE(128, 16)

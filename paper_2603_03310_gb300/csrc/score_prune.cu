@@ -73,45 +73,40 @@ __device__ int units_prefix(const int32_t* ctx_lens, int B, int P, int max_block
     return carry;
 }
 
-constexpr int kScorePrefetch = 6;   // blocks prefetched into L2 ahead of the loads
-
+// Per-warp ring of TMA tiles (16 tokens x D bf16, 128-byte swizzle).
 template <int D>
-struct KTile {
-    static constexpr int kChunks = D / 32;   // 16-byte loads per token row per thread
-    uint4 lo[kChunks];                        // token grp
-    uint4 hi[kChunks];                        // token grp + 8
-};
-
-template <int D>
-__device__ __forceinline__ void load_k_tile(KTile<D>& t, const uint16_t* tile, int grp, int tq,
-                                            bool valid) {
-#pragma unroll
-    for (int c = 0; c < KTile<D>::kChunks; ++c) {
-        if (valid) {
-            t.lo[c] = ldg_stream_u4(tile + grp * D + 32 * c + 8 * tq);
-            t.hi[c] = ldg_stream_u4(tile + (grp + 8) * D + 32 * c + 8 * tq);
-        } else {
-            t.lo[c] = make_uint4(0, 0, 0, 0);
-            t.hi[c] = make_uint4(0, 0, 0, 0);
-        }
-    }
-}
-
-// one unit of a warp's range, resolved by one lane
-struct UnitInfo {
-    int b, kvh, blk, page;
+struct ScoreRing {
+    static constexpr int kTile = 16 * D * 2;             // bytes of one 16-token tile
+    static constexpr int kStages = D == 128 ? 3 : 5;     // tiles in flight per warp
 };
 
 template <int D, int P>
+__host__ __device__ constexpr size_t score_smem_bytes(int B) {
+    return 1024                                                                 // alignment slack
+           + (size_t)kScoreWarps * ScoreRing<D>::kStages * ScoreRing<D>::kTile   // tiles
+           + (size_t)kScoreWarps * ScoreRing<D>::kStages * 8                    // barriers
+           + (size_t)kScoreWarps * 64 * 16                                      // unit tables
+           + (((size_t)(B + 1) * 4 + 15) & ~size_t(15));                        // prefix
+}
+
+template <int D, int P>
 __global__ void __launch_bounds__(kScoreThreads, 2)
-score_blocks_kernel(const ScoreArgs a) {
+score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a) {
     constexpr int kTiles = P / 16;
-    constexpr int C = KTile<D>::kChunks;
-    extern __shared__ int smem_cum[];
+    constexpr int S = ScoreRing<D>::kStages;
+    constexpr int TB = ScoreRing<D>::kTile;
+    constexpr int H = D / 64;                    // 64-element boxes per tile row
+    extern __shared__ __align__(1024) unsigned char score_smem_raw[];
+    // swizzled TMA tiles must start on a 1024-byte boundary
+    unsigned char* score_smem = score_smem_raw + ((1024 - (smem_u32(score_smem_raw) & 1023)) & 1023);
+    const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5, grp = lane >> 2, tq = lane & 3;
+    const uint32_t tiles = smem_u32(score_smem) + wl * S * TB;
+    const uint32_t bars = smem_u32(score_smem) + kScoreWarps * S * TB + wl * S * 8;
+    int4* table = reinterpret_cast<int4*>(score_smem + kScoreWarps * S * (TB + 8)) + wl * 64;
+    int* smem_cum = reinterpret_cast<int*>(score_smem + kScoreWarps * S * (TB + 8) + kScoreWarps * 64 * 16);
     __shared__ int warp_tot[kScoreWarps];
     const int total = units_prefix(a.ctx_lens, a.B, P, a.max_blocks, a.Hkv, smem_cum, warp_tot);
-    const int lane = threadIdx.x & 31, grp = lane >> 2, tq = lane & 3;
-    const int gwarp = blockIdx.x * kScoreWarps + (threadIdx.x >> 5);
+    const int gwarp = blockIdx.x * kScoreWarps + wl;
     const int nwarps = gridDim.x * kScoreWarps;
     const int share = (total + nwarps - 1) / nwarps;
     const int u0 = gwarp * share;
@@ -119,10 +114,17 @@ score_blocks_kernel(const ScoreArgs a) {
     if (u0 >= u1) return;
     const int ntiles = (u1 - u0) * kTiles;
 
-    // unit u -> (sequence, kv head, block, page); one lane per unit, 32 at a time
-    auto resolve = [&](int base) -> UnitInfo {
-        UnitInfo it{0, 0, 0, -1};
-        const int u = base + lane;
+    if (lane == 0) {
+        for (int st = 0; st < S; ++st) mbar_init(bars + 8 * st, 1);
+        fence_mbar_init();
+    }
+    __syncwarp();
+
+    // units [u0 + 32k, u0 + 32k + 32) -> table slot k & 1, one lane per unit:
+    // (sequence, kv head, block, page or -1)
+    auto resolve = [&](int k) {
+        const int u = u0 + 32 * k + lane;
+        int4 e = make_int4(0, 0, 0, -1);
         if (u < u1) {
             int lo = 0, hi = a.B - 1;   // largest b with cum[b] <= u
             while (lo < hi) {
@@ -131,86 +133,98 @@ score_blocks_kernel(const ScoreArgs a) {
             }
             const int nb = seq_blocks(__ldg(a.ctx_lens + lo), P, a.max_blocks);
             const int r = u - smem_cum[lo];
-            it.b = lo;
-            it.kvh = r / nb;
-            it.blk = r - it.kvh * nb;
-            const int pg = __ldg(a.block_table + (long long)lo * a.max_blocks + it.blk);
-            it.page = (pg >= 0 && (long long)pg < a.num_pages) ? pg : -1;
+            e.x = lo;
+            e.y = r / nb;
+            e.z = r - e.y * nb;
+            const int pg = __ldg(a.block_table + (long long)lo * a.max_blocks + e.z);
+            e.w = (pg >= 0 && (long long)pg < a.num_pages) ? pg : -1;
         }
-        return it;
+        table[(k & 1) * 32 + lane] = e;
+        __syncwarp();
     };
-    UnitInfo cur = resolve(u0);
-    int cbase = u0;
-    UnitInfo nxt = resolve(u0 + 32);
-    // unit at offset off (0..63) from cbase
-    auto unit_at = [&](int off) -> UnitInfo {
-        const int l = off & 31;
-        UnitInfo a0, a1;
-        a0.b = __shfl_sync(0xffffffffu, cur.b, l);     a1.b = __shfl_sync(0xffffffffu, nxt.b, l);
-        a0.kvh = __shfl_sync(0xffffffffu, cur.kvh, l); a1.kvh = __shfl_sync(0xffffffffu, nxt.kvh, l);
-        a0.blk = __shfl_sync(0xffffffffu, cur.blk, l); a1.blk = __shfl_sync(0xffffffffu, nxt.blk, l);
-        a0.page = __shfl_sync(0xffffffffu, cur.page, l); a1.page = __shfl_sync(0xffffffffu, nxt.page, l);
-        return off < 32 ? a0 : a1;
+    auto entry = [&](int item) -> int4 {
+        const int r = item - u0;
+        return table[((r >> 5) & 1) * 32 + (r & 31)];
     };
-    auto chunk_ptr = [&](const UnitInfo& it) {
-        return a.k_cache + ((long long)(it.page >= 0 ? it.page : 0) * a.Hkv + it.kvh) * P * D;
+    // issue the TMA copies of tile i into stage st (one elected lane)
+    auto issue = [&](int i, int st) {
+        if (lane == 0) {
+            const int item = u0 + i / kTiles;
+            const int tile = i - (i / kTiles) * kTiles;
+            const int4 e = entry(item);
+            const uint32_t bar = bars + 8 * st;
+            if (e.w >= 0) {
+                mbar_arrive_expect_tx(bar, TB);
+                const int y = (e.w * a.Hkv + e.y) * P + tile * 16;
+#pragma unroll
+                for (int h = 0; h < H; ++h) tma_load_2d(tiles + st * TB + h * 2048, &kmap, 64 * h, y, bar);
+            } else {
+                mbar_arrive(bar);   // nothing to copy: the block's page id is invalid
+            }
+        }
     };
-    // warm the L2 with the first blocks of the range (shuffles on every lane,
-    // one prefetch instruction from lane 0)
-    for (int k = 0; k < kScorePrefetch && u0 + k < u1; ++k) {
-        const UnitInfo it = unit_at(k);
-        if (lane == 0 && it.page >= 0) prefetch_l2_bulk(chunk_ptr(it), P * D * 2);
-    }
 
-    KTile<D> buf0, buf1;
-    UnitInfo ucur = unit_at(0);
-    load_k_tile<D>(buf0, chunk_ptr(ucur), grp, tq, ucur.page >= 0);
-    int cur_tile = 0;
-    uint4 qf[C];
+    resolve(0);
+    if (ntiles > 32 * kTiles) resolve(1);
+#pragma unroll 1
+    for (int st = 0; st < S && st < ntiles; ++st) issue(st, st);
+
+    uint4 qf[H][2];
     int q_b = -1, q_kvh = -1;
     float xs[kTiles][4];
+    int i = 0;
+    bool timed_out = false;
+#pragma unroll 1
+    for (; i < ntiles; ++i) {
+        const int st = i % S;
+        const int item = u0 + i / kTiles;
+        const int tile = i - (i / kTiles) * kTiles;
+        if (tile == 0 && ((item - u0) & 31) == 0 && item > u0 && item - u0 + 32 < u1 - u0)
+            resolve(((item - u0) >> 5) + 1);
+        if (!mbar_wait(bars + 8 * st, (uint32_t)((i / S) & 1), kMaxWaitIters)) {
+            timed_out = true;
+            break;
+        }
+        const int4 e = entry(item);
+        const int b = e.x, kvh = e.y, blk = e.z;
+        if (b != q_b || kvh != q_kvh) {
+            q_b = b;
+            q_kvh = kvh;
+            const int h = kvh * a.g + grp;
+#pragma unroll
+            for (int hh = 0; hh < H; ++hh)
+#pragma unroll
+                for (int c = 0; c < 2; ++c)
+                    qf[hh][c] = grp < a.g ? __ldg(reinterpret_cast<const uint4*>(
+                                                a.q + ((long long)b * a.Hq + h) * D + 64 * hh + 16 * tq + 8 * c))
+                                          : make_uint4(0, 0, 0, 0);
+        }
+        // q.k on the tensor cores: tokens = M, heads = N, head_dim = K; the
+        // thread's 16-byte chunks (2tq + c of each 64-element half) are read
+        // conflict-free from the swizzled tile, the same d permutation is used
+        // in the query fragment
+        const uint32_t tb = tiles + st * TB;
+        float acc[4] = {0.f, 0.f, 0.f, 0.f}, acc2[4] = {0.f, 0.f, 0.f, 0.f};   // two MMA chains
+#pragma unroll
+        for (int hh = 0; hh < H; ++hh)
+#pragma unroll
+            for (int c = 0; c < 2; ++c) {
+                const uint4 lo = lds_u4(tb + hh * 2048 + swz128(grp, 2 * tq + c));
+                const uint4 hi = lds_u4(tb + hh * 2048 + swz128(grp + 8, 2 * tq + c));
+                mma_bf16_16x8x16(acc, lo.x, hi.x, lo.y, hi.y, qf[hh][c].x, qf[hh][c].y);
+                mma_bf16_16x8x16(acc2, lo.z, hi.z, lo.w, hi.w, qf[hh][c].z, qf[hh][c].w);
+            }
+#pragma unroll
+        for (int e2 = 0; e2 < 4; ++e2) acc[e2] += acc2[e2];
+        // the tile's shared memory may be refilled now
+        __syncwarp();
+        fence_proxy_async();
+        if (i + S < ntiles) issue(i + S, st);
 
-    // one tile: load the next tile into `nbuf` (and prefetch further ahead),
-    // then consume `cbuf`
-    auto step = [&](const KTile<D>& cbuf, KTile<D>& nbuf, int i) {
-        const UnitInfo me = ucur;
-        const int tile = cur_tile;
-        if (i + 1 < ntiles) {
-            const int item1 = u0 + (i + 1) / kTiles;
-            const int tile1 = (i + 1) - ((i + 1) / kTiles) * kTiles;
-            if (item1 >= cbase + 32) {
-                cur = nxt;
-                cbase += 32;
-                nxt = resolve(cbase + 32);
-            }
-            ucur = unit_at(item1 - cbase);
-            cur_tile = tile1;
-            load_k_tile<D>(nbuf, chunk_ptr(ucur) + tile1 * 16 * D, grp, tq, ucur.page >= 0);
-            if (tile1 == 0 && item1 + kScorePrefetch < u1) {
-                const UnitInfo pf = unit_at(item1 + kScorePrefetch - cbase);
-                if (lane == 0 && pf.page >= 0) prefetch_l2_bulk(chunk_ptr(pf), P * D * 2);
-            }
-        }
-        if (me.b != q_b || me.kvh != q_kvh) {
-            q_b = me.b;
-            q_kvh = me.kvh;
-            const int h = me.kvh * a.g + grp;
-#pragma unroll
-            for (int c = 0; c < C; ++c)
-                qf[c] = grp < a.g ? __ldg(reinterpret_cast<const uint4*>(
-                                        a.q + ((long long)me.b * a.Hq + h) * D + 32 * c + 8 * tq))
-                                  : make_uint4(0, 0, 0, 0);
-        }
-        float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-        for (int c = 0; c < C; ++c) {
-            mma_bf16_16x8x16(acc, cbuf.lo[c].x, cbuf.hi[c].x, cbuf.lo[c].y, cbuf.hi[c].y, qf[c].x, qf[c].y);
-            mma_bf16_16x8x16(acc, cbuf.lo[c].z, cbuf.hi[c].z, cbuf.lo[c].w, cbuf.hi[c].w, qf[c].z, qf[c].w);
-        }
         // token slots grp, grp+8 of this tile; heads 2tq, 2tq+1
-        const int L = __ldg(a.ctx_lens + me.b);
-        const int valid_tok = min(P, L - me.blk * P) - tile * 16;
-        const bool ok = me.page >= 0;
+        const int L = __ldg(a.ctx_lens + b);
+        const int valid_tok = min(P, L - blk * P) - tile * 16;
+        const bool ok = e.w >= 0;
         float x4[4];
         x4[0] = (ok && grp < valid_tok) ? acc[0] * a.scale : -kInf;
         x4[1] = (ok && grp < valid_tok) ? acc[1] * a.scale : -kInf;
@@ -220,8 +234,8 @@ score_blocks_kernel(const ScoreArgs a) {
         for (int tt = 0; tt < kTiles; ++tt)      // static indices keep xs in registers
             if (tt == tile)
 #pragma unroll
-                for (int e = 0; e < 4; ++e) xs[tt][e] = x4[e];
-        const long long unit = ((long long)me.b * a.Hkv + me.kvh) * a.max_blocks + me.blk;
+                for (int ee = 0; ee < 4; ++ee) xs[tt][ee] = x4[ee];
+        const long long unit = ((long long)b * a.Hkv + kvh) * a.max_blocks + blk;
         if (a.token_scores) {
             float* ts = a.token_scores + (unit * P + tile * 16) * a.g;
             const int h0 = 2 * tq, h1 = 2 * tq + 1;
@@ -257,8 +271,8 @@ score_blocks_kernel(const ScoreArgs a) {
 #pragma unroll
                     for (int tt = 0; tt < kTiles; ++tt) {
 #pragma unroll
-                        for (int e = 0; e < 2; ++e) {
-                            const float d = xs[tt][j + 2 * e] - m;
+                        for (int ee = 0; ee < 2; ++ee) {
+                            const float d = xs[tt][j + 2 * ee] - m;
                             const float w = fast_ex2(d * kLog2e);
                             l1 += d < 0.f ? w : 0.f;
                             neq += d == 0.f ? 1.f : 0.f;
@@ -277,11 +291,19 @@ score_blocks_kernel(const ScoreArgs a) {
                 if (grp == 0 && h < a.g) a.stats[unit * a.g + h] = make_float4(m, l1, u, 0.f);
             }
         }
-    };
-
-    for (int i = 0; i < ntiles; i += 2) {
-        step(buf0, buf1, i);
-        if (i + 1 < ntiles) step(buf1, buf0, i + 1);
+    }
+    if (timed_out) {
+        // a copy never arrived: let the copies still in flight land (bounded),
+        // then mark every block this warp did not finish with NaN stats, which
+        // the keep-set pass reports as ETI_ERRF_TIMEOUT for its sequence
+        for (int k = i; k < ntiles && k < i + S; ++k) mbar_wait(bars + 8 * (k % S), (uint32_t)((k / S) & 1), 1024);
+        const float nan = __int_as_float(0x7fc00000);
+        for (int item = u0 + i / kTiles; item < u1; ++item) {
+            if (((item - u0) & 31) == 0 && item > u0) resolve((item - u0) >> 5);
+            const int4 e = entry(item);
+            const long long unit = ((long long)e.x * a.Hkv + e.y) * a.max_blocks + e.z;
+            if (lane < a.g) a.stats[unit * a.g + lane] = make_float4(nan, nan, nan, 0.f);
+        }
     }
 }
 
@@ -404,7 +426,7 @@ prune_finalize_kernel(const FinArgs a) {
 
     // pass 1 (the only pass over global memory when the stats fit in shared
     // memory): page ids, stats cache, max per head
-    int bad = 0;
+    int bad = 0, stale = 0;
     float M[G];
 #pragma unroll
     for (int h = 0; h < G; ++h) M[h] = -kInf;
@@ -414,6 +436,7 @@ prune_finalize_kernel(const FinArgs a) {
 #pragma unroll
         for (int h = 0; h < G; ++h) {
             const float4 s = st[j * G + h];
+            stale |= (s.x != s.x);          // NaN max: the scoring pass gave up on this block
             if (kCache) {
                 sh_m[h * a.max_blocks + j] = s.x;
                 sh_l[h * a.max_blocks + j] = s.y;
@@ -423,9 +446,14 @@ prune_finalize_kernel(const FinArgs a) {
         }
     }
     const bool bad_page = __syncthreads_or(bad) != 0;
-    if (a.err && kvh == 0 && tid == 0)
-        a.err[b] = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page && !bad_ctx ? ETI_ERRF_BAD_PAGE : 0u);
-    const int n = (bad_ctx || bad_page) ? 0 : nb;
+    const bool timed_out = __syncthreads_or(stale && !bad) != 0;
+    if (a.err && tid == 0) {
+        // err was cleared before this kernel; every kv head ORs in its bits
+        const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page && !bad_ctx ? ETI_ERRF_BAD_PAGE : 0u) |
+                           (timed_out ? ETI_ERRF_TIMEOUT : 0u);
+        if (e) atomicOr(a.err + b, e);
+    }
+    const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
     const int k0 = min(j0, n), k1 = min(j1, n);
 
     auto stat = [&](int j, int h) -> float4 {
@@ -641,22 +669,31 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
                             int max_blocks, long long num_pages, float scale, float* token_scores,
                             float4* stats, cudaStream_t stream) {
     if (B == 0) return ETI_OK;
+    if (num_pages <= 0) {
+        // no page can be valid: every sequence with blocks is reported by the
+        // keep-set pass; nothing to score
+        return ETI_OK;
+    }
     ScoreArgs a;
     a.q = q; a.k_cache = k_cache; a.block_table = block_table; a.ctx_lens = ctx_lens;
     a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.g = Hq / Hkv; a.max_blocks = max_blocks;
     a.num_pages = num_pages; a.scale = scale; a.token_scores = token_scores; a.stats = stats;
+    // tile row coordinates are int32 on the device
+    if (num_pages * Hkv * P >= (1LL << 31)) return ETI_ERR_UNSUPPORTED;
+    CUtensorMap kmap;
+    int st = eti_make_kv_tensor_map(&kmap, k_cache, num_pages * Hkv * P, D);
+    if (st != ETI_OK) return st;
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = 2 * sms;
-    const size_t cum_bytes = ((size_t)(B + 1) * 4 + 15) & ~size_t(15);
     cudaError_t e;
 #define ETI_SCORE_CASE(DD, PP)                                                              \
     if (D == DD && P == PP) {                                                               \
         auto k = score_blocks_kernel<DD, PP>;                                               \
-        const size_t smem = cum_bytes;                                                      \
-        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-        k<<<grid, kScoreThreads, smem, stream>>>(a);                                        \
+        const size_t smem = score_smem_bytes<DD, PP>(B);                                    \
+        cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);    \
+        k<<<grid, kScoreThreads, smem, stream>>>(kmap, a);                                  \
         e = cudaGetLastError();                                                             \
         return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;                                    \
     }
@@ -684,6 +721,7 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     a.kept_norm = kept_norm; a.err = err;
     const int grid = B * Hkv;
     cudaError_t e = cudaSuccess;
+    if (err && cudaMemsetAsync(err, 0, (size_t)B * sizeof(uint32_t), stream) != cudaSuccess) return ETI_ERR_CUDA;
     int dev = 0, optin = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
