@@ -269,7 +269,7 @@ def run_gpu(args):
     traffic = args.traffic if args.traffic is not None else ncu_traffic(
         {"score": "score_blocks", "prune": "prune_finalize", "decode": "paged_decode"}.get(dom))
     roof = {"kernel": {"score": "score_blocks", "prune": "prune_finalize",
-                       "decode": "paged_decode (plan + decode + combine)",
+                       "decode": "paged_decode (plan + decode; split segments merged in-kernel)",
                        "sample": "entropy_temp_sample"}[dom],
             "bound": "hbm", "achieved": round(achieved[dom], 1), "peak": peak, "unit": "GB/s",
             "frac": round(achieved[dom] / peak, 4), "peak_source": peak_src,
@@ -301,7 +301,9 @@ def run_gpu(args):
                                ((mean_ms["score"] + mean_ms["prune"] + mean_ms["decode"]) / 1e3) / 1e12, 3),
         "gpu_launches": 6 * args.steps,
         "launches_per_step": {"score_blocks": 1, "prune_finalize": 1, "decode_plan": 1,
-                              "paged_decode": 1, "decode_combine": 1, "entropy_temp_sample": 1},
+                              "paged_decode": 1,
+                              "entropy_sample_partial": 1, "entropy_sample_finalize": 1,
+                              "memset (error flags, not a kernel of the library)": 1},
         "e2e": e2e,
         "wall_s_timed_region": round(wall, 4),
         "clocks": clk.summary(),

@@ -27,9 +27,9 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
                       const int32_t* kept_idx, const int32_t* kept_cnt, const float* token_scores,
                       const float* kept_norm, int B, int Hq, int Hkv, int D, int P, int max_blocks,
                       long long num_pages, uint16_t* out, uint32_t* err, int* plan_cum,
-                      int* plan_info, int* plan_warp_seg, float* partial, int nwarps,
-                      cudaStream_t stream);
-int eti_decode_nwarps();
+                      int* plan_info, int* plan_warp_seg, int* plan_ticket, float* partial,
+                      int nwarps, cudaStream_t stream);
+int eti_decode_nwarps(int D, int g);
 
 // cuTensorMapEncodeTiled, fetched from the driver at first use (no link
 // dependency on libcuda).
@@ -93,7 +93,7 @@ struct Carver {
 
 struct DecodeWs {
     float* scores; float4* stats; int32_t* kidx; int32_t* kcnt; float* knorm;
-    int* cum; int* info; int* warp_seg; float* partial;
+    int* cum; int* info; int* warp_seg; int* ticket; float* partial;
 };
 
 DecodeWs carve_decode(void* ws, int B, int Hq, int Hkv, int D, int P, int max_blocks,
@@ -109,8 +109,9 @@ DecodeWs carve_decode(void* ws, int B, int Hq, int Hkv, int D, int P, int max_bl
         w.knorm = c.take<float>((size_t)B * Hq * 2);
     }
     w.cum = c.take<int>(nseg + 1);
-    w.info = c.take<int>(4);   // total kept blocks, share per warp, timeout flag
+    w.info = c.take<int>(4);   // total kept blocks, share per warp
     w.warp_seg = c.take<int>(nwarps);
+    w.ticket = c.take<int>(nseg);
     w.partial = c.take<float>(((size_t)nwarps + nseg) * g * D);
     *bytes = c.off;
     return w;
@@ -244,7 +245,7 @@ size_t eti_paged_decode_workspace_size(int B, int Hq, int Hkv, int D, int P, int
                                        int have_scores) {
     if (check_attn_shape(B, Hq, Hkv, D, P, max_blocks, 0) != ETI_OK) return 0;
     size_t bytes = 0;
-    carve_decode(nullptr, B, Hq, Hkv, D, P, max_blocks, have_scores, eti_decode_nwarps(), &bytes);
+    carve_decode(nullptr, B, Hq, Hkv, D, P, max_blocks, have_scores, eti_decode_nwarps(D, Hq / Hkv), &bytes);
     return bytes;
 }
 
@@ -266,7 +267,7 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
     if (!aligned16(v_cache) || !aligned16(out) || (have_scores && !aligned16(token_scores)) ||
         (!have_scores && (!aligned16(q) || !aligned16(k_cache))))
         return ETI_ERR_ALIGN;
-    const int nwarps = eti_decode_nwarps();
+    const int nwarps = eti_decode_nwarps(D, Hq / Hkv);
     size_t need = 0;
     carve_decode(nullptr, B, Hq, Hkv, D, P, max_blocks, have_scores, nwarps, &need);
     if (!ws || ws_bytes < need) return ETI_ERR_WORKSPACE;
@@ -289,7 +290,7 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
     }
     return eti_launch_decode(v_cache, block_table, ctx_lens, kept_idx, kept_cnt, token_scores,
                              kept_norm, B, Hq, Hkv, D, P, max_blocks, (long long)num_pages, out,
-                             err_flags, w.cum, w.info, w.warp_seg, w.partial, nwarps, s);
+                             err_flags, w.cum, w.info, w.warp_seg, w.ticket, w.partial, nwarps, s);
 }
 
 }  // extern "C"

@@ -222,7 +222,32 @@ __device__ __forceinline__ int seq_blocks(int L, int P, int max_blocks) {
 
 constexpr int kMaxWaitIters = 1 << 20;
 
+// Programmatic dependent launch: let the next kernel in the stream be
+// scheduled now (it still waits for this grid to finish before reading our
+// results), and wait for the previous grid's results before reading them.
+// Both are no-ops when the kernel was launched without the attribute.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 }  // namespace eti
+
+// Launch with programmatic stream serialization (overlaps this kernel's
+// launch with the previous kernel's tail).
+template <typename... KArgs, typename... Args>
+inline cudaError_t eti_launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                  cudaStream_t stream, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
 
 // Host: a 2-D bf16 tensor map over a [rows][D] array with boxes of
 // 16 rows x 64 elements (128 bytes) and the 128-byte swizzle.

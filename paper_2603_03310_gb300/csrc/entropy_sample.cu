@@ -79,8 +79,9 @@ __device__ __forceinline__ void state_init(RowState& s) {
     s.m = -kInf; s.mc = -kInf; s.S = 0.f; s.U = 0.f; s.r = 0.f; s.bi = 0x7fffffff;
 }
 
-// Move the state to a new, larger reference max `nm`.
-__device__ __forceinline__ void state_rebase(RowState& s, float nm, float c) {
+// Move the state to a new, larger reference max `nm`; returns the factor
+// 2^{mc_old - mc_new} by which every term of the state was scaled.
+__device__ __forceinline__ float state_rebase(RowState& s, float nm, float c) {
     const float nmc = nm * c;
     float a = 0.f, d = 0.f;
     if (s.m != -kInf) {
@@ -92,6 +93,7 @@ __device__ __forceinline__ void state_rebase(RowState& s, float nm, float c) {
     s.r *= a;
     s.m = nm;
     s.mc = nmc;
+    return a;
 }
 
 // Merge partial `o` into `s` (both may be empty).
@@ -125,16 +127,29 @@ __device__ __forceinline__ RowState state_shfl_xor(const RowState& s, int o) {
     return r;
 }
 
+// Race prefilter.  -log u >= 1 - u, so E2 >= log2(e) v with v = 1 - u, and
+// both evaluations of E2 above stay within 2^-18 (relative) of the true
+// value; a token with w <= rk v, rk = r_lb log2(e) (1 - 2^-16), therefore has
+// w / E2 below r_lb by at least 2^-17 relative and cannot win, where r_lb is
+// any ratio already reached in this row (own best, or a bound shared by the
+// warp).  Only the tokens that pass evaluate E2, so the draw is unchanged.
+constexpr float kRaceKappa = 1.4426950408889634f * (1.0f - 1.0f / 65536.0f);
+
 // One token: entropy sums and the race.
-__device__ __forceinline__ void consume(RowState& s, float z, uint32_t word, int x, float c) {
+__device__ __forceinline__ void consume(RowState& s, float& rk, float z, uint32_t word, int x, float c) {
     const float t = fmaf(z, c, -s.mc);
     const float w = fast_ex2(t);
     s.S += w;
     s.U = fmaf(w, fmaxf(t, -250.f), s.U);   // -inf logits add 0 (w = 0); NaN still reaches S
-    const float E = exp_variate_log2(word);
-    if (w > s.r * E) {                        // rare after the first few tokens
-        s.r = __fdividef(w, E);
-        s.bi = x;
+    // 1 - u = (2 (0x7FFFFF - j) + 1) 2^-24, formed exactly like u
+    const float v = __uint_as_float((~word & 0x7FFFFFu) | 0x3F800000u) - __uint_as_float(0x3F7FFFFFu);
+    if (w > rk * v) {                         // rare once rk has grown
+        const float E = exp_variate_log2(word);
+        if (w > s.r * E) {
+            s.r = __fdividef(w, E);
+            s.bi = x;
+            rk = fmaxf(rk, s.r * kRaceKappa);
+        }
     }
 }
 
@@ -184,6 +199,8 @@ __device__ __forceinline__ void load_group(float (&z)[4], const float* row, int 
 template <bool kVec>
 __global__ void __launch_bounds__(kEtsThreads, kEtsCtasPerSm)
 entropy_sample_partial_kernel(const EtsArgs a) {
+    pdl_trigger();
+    pdl_wait();
     __shared__ RowState warp_part[kEtsThreads / 32];
     const int tid = threadIdx.x;
     const long long total = (long long)a.B * a.ngroups;
@@ -206,6 +223,11 @@ entropy_sample_partial_kernel(const EtsArgs a) {
         const float* row = a.logits + (long long)b * a.ld;
         RowState s;
         state_init(s);
+        float rk = 0.f;              // race prefilter bound, in the state's frame
+        bool shared = false;         // the warp's bound has been folded into rk
+        // every lane of the warp walks this row piece (the same steps), so the
+        // warp may exchange its bound with full-mask shuffles
+        const bool warp_full = g0 + (tid | 31) < g1;
         if (!bad_T && g0 + tid < g1) {
             constexpr int step = kEtsPair * kEtsThreads;
             float cur[kEtsPair][4], nxt[kEtsPair][4];
@@ -233,20 +255,33 @@ entropy_sample_partial_kernel(const EtsArgs a) {
                         for (int e = 0; e < 4; ++e) nan |= (cur[k][e] != cur[k][e]);
                     if (nan) s.S = __int_as_float(0x7fc00000);
                 } else {
-                    if (bm > s.m) state_rebase(s, bm, c);
+                    if (bm > s.m) rk *= state_rebase(s, bm, c);
 #pragma unroll
                     for (int k = 0; k < kEtsPair; ++k) {
                         const int g = base + k * kEtsThreads + tid;
                         if (g < g1) {
                             const uint4 r = philox4x32_10(make_uint4((uint32_t)g, (uint32_t)b, a.off_lo, a.off_hi), k0, k1);
-                            consume(s, cur[k][0], r.x, 4 * g + 0, c);
-                            consume(s, cur[k][1], r.y, 4 * g + 1, c);
-                            consume(s, cur[k][2], r.z, 4 * g + 2, c);
-                            consume(s, cur[k][3], r.w, 4 * g + 3, c);
+                            consume(s, rk, cur[k][0], r.x, 4 * g + 0, c);
+                            consume(s, rk, cur[k][1], r.y, 4 * g + 1, c);
+                            consume(s, rk, cur[k][2], r.z, 4 * g + 2, c);
+                            consume(s, rk, cur[k][3], r.w, 4 * g + 3, c);
                         }
                     }
                 }
                 if (!more) break;
+                if (!shared && warp_full) {
+                    // After the first step, share the best ratio of the warp as
+                    // a bound: lr = log2 r + mc is the ratio in the row's common
+                    // frame, and the 2^-10 shaved off covers the rounding of
+                    // lr and of its conversion back to this state's frame.  The
+                    // cap keeps rk finite, so a later rebase by 0 gives 0.
+                    shared = true;
+                    float lr = s.r > 0.f ? fast_lg2(s.r) + s.mc : -kInf;
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) lr = fmaxf(lr, __shfl_xor_sync(0xffffffffu, lr, o));
+                    if (lr > -kInf && s.m != -kInf)
+                        rk = fmaxf(rk, fminf(fast_ex2(lr - s.mc - 0.0009765625f) * kRaceKappa, 1e38f));
+                }
 #pragma unroll
                 for (int k = 0; k < kEtsPair; ++k)
 #pragma unroll
@@ -271,6 +306,8 @@ entropy_sample_partial_kernel(const EtsArgs a) {
 // Per row: merge the partial slots in CTA order, then the scalar epilogue.
 __global__ void __launch_bounds__(128)
 entropy_sample_finalize_kernel(const EtsArgs a) {
+    pdl_trigger();
+    pdl_wait();
     const int lane = threadIdx.x & 31;
     const int b = blockIdx.x * 4 + (threadIdx.x >> 5);
     if (b >= a.B) return;
@@ -369,11 +406,11 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
     a.share = (total + ncta - 1) / ncta;
     a.part = static_cast<RowState*>(part);
     const bool vec = (ld % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
-    if (vec) entropy_sample_partial_kernel<true><<<ncta, kEtsThreads, 0, stream>>>(a);
-    else entropy_sample_partial_kernel<false><<<ncta, kEtsThreads, 0, stream>>>(a);
-    if (cudaGetLastError() != cudaSuccess) return ETI_ERR_CUDA;
-    entropy_sample_finalize_kernel<<<(B + 3) / 4, 128, 0, stream>>>(a);
-    return cudaGetLastError() == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
+    const cudaError_t e1 = vec ? eti_launch_pdl(entropy_sample_partial_kernel<true>, dim3(ncta), dim3(kEtsThreads), 0, stream, a)
+                               : eti_launch_pdl(entropy_sample_partial_kernel<false>, dim3(ncta), dim3(kEtsThreads), 0, stream, a);
+    if (e1 != cudaSuccess) return ETI_ERR_CUDA;
+    return eti_launch_pdl(entropy_sample_finalize_kernel, dim3((B + 3) / 4), dim3(128), 0, stream, a) == cudaSuccess
+               ? ETI_OK : ETI_ERR_CUDA;
 }
 
 // ---------------------------------------------------------------------------

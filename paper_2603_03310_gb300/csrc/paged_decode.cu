@@ -21,8 +21,13 @@
 // (head_dim = M, query heads = N, tokens = K): V rows are transposed into A
 // fragments with byte permutes, the probabilities form the B fragment.
 // A segment that lies inside one warp's range is written straight to `out`;
-// otherwise the warp's part goes to partial slot (warp + segment) and the
-// combine kernel adds the slots in warp order (deterministic).
+// otherwise the warp's part goes to partial slot (warp + segment), and the
+// warp that closes the segment's ticket last adds its slots in warp order
+// (deterministic) and writes the output: no second kernel, no waiting.
+//
+// The plan kernel that runs first forms the prefix of kept counts, each
+// warp's first segment, zeroes the tickets, and writes every sequence's error
+// word (context length and page ids checked once, one warp per sequence).
 #include <cstring>
 
 #include "common.cuh"
@@ -34,18 +39,43 @@ constexpr int kDecThreads = kDecWarps * 32;
 constexpr int kPlanThreads = 1024;
 
 // --------------------------------------------------------------------------
-// plan: prefix of kept counts, the per-warp share and each warp's first segment
+// plan: prefix of kept counts, the per-warp share, each warp's first
+// segment, zeroed tickets (CTA 0); the error word of every sequence (the
+// other CTAs, one warp per sequence)
 struct PlanArgs {
     const int32_t* kept_cnt;
+    const int32_t* ctx_lens;
+    const int32_t* block_table;
+    long long num_pages;
+    int B, Hkv, P;
     int nseg, nwarps, max_blocks;
     int* cum;       // [nseg + 1]
     int* info;      // [0] = total kept blocks, [1] = share per warp
     int* warp_seg;  // [nwarps]
+    int* ticket;    // [nseg]
+    uint32_t* err;  // [B]
 };
 
 __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArgs a) {
-    __shared__ int wsum[kPlanThreads / 32];
+    pdl_trigger();
+    pdl_wait();
     const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+    if (blockIdx.x > 0) {
+        const int b = (blockIdx.x - 1) * (kPlanThreads / 32) + w;
+        if (b >= a.B) return;
+        const int L = a.ctx_lens[b];
+        const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
+        const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
+        int bad = 0;
+        for (int j = lane; j < nb; j += 32) {
+            const int pg = a.block_table[(long long)b * a.max_blocks + j];
+            bad |= (pg < 0 || (long long)pg >= a.num_pages);
+        }
+        bad = __any_sync(0xffffffffu, bad);
+        if (lane == 0) a.err[b] = bad_ctx ? ETI_ERRF_BAD_CTX : (bad ? ETI_ERRF_BAD_PAGE : 0u);
+        return;
+    }
+    __shared__ int wsum[kPlanThreads / 32];
     int carry = 0;
     for (int base = 0; base < a.nseg; base += kPlanThreads) {
         const int s = base + tid;
@@ -63,7 +93,10 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
             if (i < w) ofs += wsum[i];
             tot += wsum[i];
         }
-        if (s < a.nseg) a.cum[s] = carry + ofs + x - v;
+        if (s < a.nseg) {
+            a.cum[s] = carry + ofs + x - v;
+            a.ticket[s] = 0;
+        }
         carry += tot;
         __syncthreads();
     }
@@ -73,7 +106,6 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
         a.cum[a.nseg] = total;
         a.info[0] = total;
         a.info[1] = share;
-        a.info[2] = 0;      // set by the decode kernel if a tile copy never arrived
     }
     for (int c = tid; c < a.nwarps; c += kPlanThreads) a.warp_seg[c] = a.nseg;
     __syncthreads();
@@ -100,20 +132,24 @@ struct DecArgs {
     long long num_pages;
     uint16_t* out;                 // bf16 [B][Hq][D]
     float* partial;                // [(nwarps + nseg)][g][D]
+    int* ticket;                   // [nseg], zeroed by the plan kernel
+    uint32_t* err;                 // [B], written by the plan kernel
 };
 
 template <int D>
 struct DecLayout {
     static constexpr int E = D / 16;              // bf16 per row half per thread
     static constexpr int kTile = 16 * D * 2;      // bytes of one 16-token V tile
-    static constexpr int kScores = 16 * 8 * 4;    // room for one tile's scores (g <= 8)
     static constexpr int kStages = D == 128 ? 3 : 5;
     using Vec = typename std::conditional<E == 8, uint4, uint2>::type;
 };
 
+// bytes of one tile's scores (16 tokens x g heads, fp32)
+__host__ __device__ inline int dec_score_bytes(int g) { return 16 * g * 4; }
+
 template <int D>
-__host__ __device__ constexpr size_t dec_smem_bytes() {
-    return 1024 + (size_t)kDecWarps * DecLayout<D>::kStages * (DecLayout<D>::kTile + DecLayout<D>::kScores + 8)
+__host__ __device__ inline size_t dec_smem_bytes(int g) {
+    return 1024 + (size_t)kDecWarps * DecLayout<D>::kStages * (DecLayout<D>::kTile + dec_score_bytes(g) + 8)
            + (size_t)kDecWarps * 64 * 16;
 }
 
@@ -164,8 +200,10 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
     constexpr int J = D / 16;                    // MMAs per 16-token tile
     constexpr int S = LY::kStages;
     constexpr int TB = LY::kTile;
-    constexpr int SB = LY::kScores;
     constexpr int H = D / 64;                    // 64-element boxes per tile row
+    pdl_trigger();
+    pdl_wait();
+    const int SB = dec_score_bytes(a.g);
     extern __shared__ __align__(1024) unsigned char dec_smem_raw[];
     unsigned char* dec_smem = dec_smem_raw + ((1024 - (smem_u32(dec_smem_raw) & 1023)) & 1023);
     const int lane = threadIdx.x & 31, wl = threadIdx.x >> 5, grp = lane >> 2, tq = lane & 3;
@@ -173,14 +211,26 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
     const int total = a.info[0], share = a.info[1];
     const int u0 = warp * share;
     const int u1 = min(u0 + share, total);
-    if (u0 >= u1) return;
     const int nseg = a.B * a.Hkv;
+    // segments with nothing kept have no writer: their output is zeroed here
+    auto zero_empty = [&]() {
+        for (int s = warp; s < nseg; s += gridDim.x * kDecWarps) {
+            if (__ldg(a.cum + s + 1) > __ldg(a.cum + s)) continue;
+            const int b = s / a.Hkv, kvh = s - b * a.Hkv;
+            uint16_t* o = a.out + ((long long)b * a.Hq + kvh * a.g) * D;
+            for (int e = lane * 8; e < a.g * D; e += 256) *reinterpret_cast<uint4*>(o + e) = make_uint4(0, 0, 0, 0);
+        }
+    };
+    if (u0 >= u1) {
+        zero_empty();
+        return;
+    }
     const int ntiles = (u1 - u0) * kTiles;
     const uint32_t tiles = smem_u32(dec_smem) + wl * S * TB;
     const uint32_t scores = smem_u32(dec_smem) + kDecWarps * S * TB + wl * S * SB;
     const uint32_t bars = smem_u32(dec_smem) + kDecWarps * S * (TB + SB) + wl * S * 8;
     int4* table = reinterpret_cast<int4*>(dec_smem + kDecWarps * S * (TB + SB + 8)) + wl * 64;
-    const int sbytes = 16 * a.g * 4;             // one tile's scores (a multiple of 16)
+    const int sbytes = SB;                       // one tile's scores (a multiple of 16)
 
     if (lane == 0) {
         for (int st = 0; st < S; ++st) mbar_init(bars + 8 * st, 1);
@@ -244,12 +294,50 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
 #pragma unroll
     for (int j = 0; j < J; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
 
+    // the last warp of a split segment: add the slots (warp + seg) of warps
+    // w0..w1 in warp order, normalise, write bf16 (zeros for a bad sequence)
+    auto merge = [&](int seg, int lo, int hi, bool bad) {
+        const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
+        const int w0 = lo / share, nw = (hi - 1) / share - w0 + 1;
+        const long long stride = (long long)a.g * D;      // floats between consecutive slots
+        const float4* base = reinterpret_cast<const float4*>(a.partial + (long long)(w0 + seg) * stride);
+        const int n4 = a.g * D / 4;                         // float4 per slot
+        constexpr int kM = D / 16;                          // float4 per lane for g = 8
+        float4 v[kM];
+#pragma unroll
+        for (int k = 0; k < kM; ++k) v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int w = 0; w < nw; ++w) {
+#pragma unroll
+            for (int k = 0; k < kM; ++k) {
+                const int e4 = lane + 32 * k;
+                if (e4 < n4) {
+                    // L2 reads: the other warps' slots were published by their tickets
+                    const float4 x = __ldcg(base + (long long)w * (stride / 4) + e4);
+                    v[k].x += x.x; v[k].y += x.y; v[k].z += x.z; v[k].w += x.w;
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kM; ++k) {
+            const int e4 = lane + 32 * k;
+            if (e4 < n4) {
+                const int h = (4 * e4) / D, d = 4 * e4 - h * D;
+                const float l = __ldg(a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2 + 1);
+                const float inv = (!bad && l > 0.f) ? 1.f / l : 0.f;
+                *reinterpret_cast<uint2*>(a.out + ((long long)b * a.Hq + kvh * a.g + h) * D + d) =
+                    make_uint2(pack_bf16x2(v[k].x * inv, v[k].y * inv), pack_bf16x2(v[k].z * inv, v[k].w * inv));
+            }
+        }
+    };
+
     // write the accumulated segment: straight to `out` when the whole segment
-    // is in this warp's range, else into partial slot (warp + seg)
+    // is in this warp's range, else into partial slot (warp + seg) and take a
+    // ticket; the warp that takes the segment's last ticket merges the slots
     auto flush = [&](int seg) {
         const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
         const int lo = __ldg(a.cum + seg), hi = __ldg(a.cum + seg + 1);
         const bool whole = lo >= u0 && hi <= u1;
+        const bool bad = (a.err[b] & (ETI_ERRF_BAD_CTX | ETI_ERRF_BAD_PAGE)) != 0u;
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
             const int h = 2 * tq + e;
@@ -262,7 +350,7 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
                     for (int j = 0; j < J; ++j) v[j] = acc[j][2 * half + e];
                     if (whole) {
                         const float l = __ldg(a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2 + 1);
-                        const float inv = l > 0.f ? 1.f / l : 0.f;
+                        const float inv = (!bad && l > 0.f) ? 1.f / l : 0.f;
                         uint32_t pk[J / 2];
 #pragma unroll
                         for (int j = 0; j < J / 2; ++j) pk[j] = pack_bf16x2(v[2 * j] * inv, v[2 * j + 1] * inv);
@@ -280,6 +368,16 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
         }
 #pragma unroll
         for (int j = 0; j < J; ++j) acc[j][0] = acc[j][1] = acc[j][2] = acc[j][3] = 0.f;
+        if (!whole) {
+            __threadfence();          // this lane's part of the slot, before the ticket
+            __syncwarp();
+            int last = 0;
+            if (lane == 0) last = atomicAdd(a.ticket + seg, 1) == (hi - 1) / share - lo / share;
+            if (__shfl_sync(0xffffffffu, last, 0)) {
+                __threadfence();
+                merge(seg, lo, hi, bad);
+            }
+        }
     };
 
     resolve(0);
@@ -340,63 +438,26 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
         }
     }
     if (timed_out) {
-        // a copy never arrived: let the ones in flight land (bounded) and
-        // report it; the combine pass flags every sequence of the call
+        // a copy never arrived: let the ones in flight land (bounded), flag
+        // every sequence of the rest of this range, and still close their
+        // segments (tickets included) so no output is left unwritten
         for (int k = i; k < ntiles && k < i + S; ++k) mbar_wait(bars + 8 * (k % S), (uint32_t)((k / S) & 1), 1024);
-        if (lane == 0) atomicOr(const_cast<int*>(a.info) + 2, 1);
+        for (int sg = cur_seg >= 0 ? cur_seg : a.warp_seg[warp]; sg < nseg && __ldg(a.cum + sg) < u1; ++sg) {
+            if (__ldg(a.cum + sg + 1) <= __ldg(a.cum + sg)) continue;
+            if (lane == 0) atomicOr(a.err + sg / a.Hkv, ETI_ERRF_TIMEOUT);
+            flush(sg);
+        }
+        zero_empty();
         return;
     }
     if (cur_seg >= 0) flush(cur_seg);
+    zero_empty();
 }
 
-// --------------------------------------------------------------------------
-// combine: add the partial slots of segments split across warps; zero the
-// output of segments with nothing kept or of invalid sequences.
-struct CombArgs {
-    const int* cum;
-    const int* info;
-    const float* partial;
-    const float* kept_norm;
-    const int32_t* ctx_lens;
-    const int32_t* block_table;
-    long long num_pages;
-    int B, Hq, Hkv, g, D, P, max_blocks;
-    uint16_t* out;
-    uint32_t* err;
-};
-
-__global__ void __launch_bounds__(128) decode_combine_kernel(const CombArgs a) {
-    const int s = blockIdx.x;
-    const int b = s / a.Hkv, kvh = s - b * a.Hkv;
-    const int tid = threadIdx.x;
-    const int L = a.ctx_lens[b];
-    const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
-    const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
-    int bad = 0;
-    for (int j = tid; j < nb; j += blockDim.x) {
-        const int pg = a.block_table[(long long)b * a.max_blocks + j];
-        bad |= (pg < 0 || (long long)pg >= a.num_pages);
-    }
-    const bool bad_page = __syncthreads_or(bad) != 0;
-    if (a.err && kvh == 0 && tid == 0)
-        a.err[b] = (bad_ctx ? ETI_ERRF_BAD_CTX : (bad_page ? ETI_ERRF_BAD_PAGE : 0u)) |
-                   (a.info[2] ? ETI_ERRF_TIMEOUT : 0u);
-    const int lo = a.cum[s], hi = a.cum[s + 1];
-    const int share = a.info[1];
-    uint16_t* o = a.out + ((long long)b * a.Hq + kvh * a.g) * a.D;
-    if (bad_ctx || bad_page || hi <= lo) {
-        for (int e = tid; e < a.g * a.D; e += blockDim.x) o[e] = 0;
-        return;
-    }
-    const int w0 = lo / share, w1 = (hi - 1) / share;
-    if (w0 == w1) return;   // one warp covered the segment and wrote it
-    for (int e = tid; e < a.g * a.D; e += blockDim.x) {
-        const int h = e / a.D, d = e - h * a.D;
-        float v = 0.f;
-        for (int w = w0; w <= w1; ++w) v += a.partial[((long long)(w + s) * a.g + h) * a.D + d];
-        const float l = a.kept_norm[((long long)b * a.Hq + kvh * a.g + h) * 2 + 1];
-        o[e] = __bfloat16_as_ushort(__float2bfloat16_rn(l > 0.f ? v / l : 0.f));
-    }
+// CTAs of the decode kernel per SM for this shape (as many as fit, up to 2)
+inline int dec_ctas_per_sm(int D, int g) {
+    const size_t sm = D == 128 ? dec_smem_bytes<128>(g) : dec_smem_bytes<64>(g);
+    return sm + 1024 <= 233472 / 2 ? 2 : 1;
 }
 
 }  // namespace eti
@@ -404,26 +465,30 @@ __global__ void __launch_bounds__(128) decode_combine_kernel(const CombArgs a) {
 using namespace eti;
 
 // warps of the persistent decode grid on the current device
-int eti_decode_nwarps() {
+int eti_decode_nwarps(int D, int g) {
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    return 2 * sms * kDecWarps;
+    return dec_ctas_per_sm(D, g) * sms * kDecWarps;
 }
 
 int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const int32_t* ctx_lens,
                       const int32_t* kept_idx, const int32_t* kept_cnt, const float* token_scores,
                       const float* kept_norm, int B, int Hq, int Hkv, int D, int P, int max_blocks,
                       long long num_pages, uint16_t* out, uint32_t* err, int* plan_cum,
-                      int* plan_info, int* plan_warp_seg, float* partial, int nwarps,
-                      cudaStream_t stream) {
+                      int* plan_info, int* plan_warp_seg, int* plan_ticket, float* partial,
+                      int nwarps, cudaStream_t stream) {
     if (B == 0) return ETI_OK;
     const int nseg = B * Hkv;
     PlanArgs pa;
-    pa.kept_cnt = kept_cnt; pa.nseg = nseg; pa.nwarps = nwarps; pa.max_blocks = max_blocks;
+    pa.kept_cnt = kept_cnt; pa.ctx_lens = ctx_lens; pa.block_table = block_table;
+    pa.num_pages = num_pages; pa.B = B; pa.Hkv = Hkv; pa.P = P;
+    pa.nseg = nseg; pa.nwarps = nwarps; pa.max_blocks = max_blocks;
     pa.cum = plan_cum; pa.info = plan_info; pa.warp_seg = plan_warp_seg;
-    decode_plan_kernel<<<1, kPlanThreads, 0, stream>>>(pa);
-    if (cudaGetLastError() != cudaSuccess) return ETI_ERR_CUDA;
+    pa.ticket = plan_ticket; pa.err = err;
+    const int plan_grid = 1 + (B + kPlanThreads / 32 - 1) / (kPlanThreads / 32);
+    if (eti_launch_pdl(decode_plan_kernel, dim3(plan_grid), dim3(kPlanThreads), 0, stream, pa) != cudaSuccess)
+        return ETI_ERR_CUDA;
 
     DecArgs da;
     da.v_cache = v_cache; da.block_table = block_table; da.ctx_lens = ctx_lens;
@@ -431,6 +496,7 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
     da.cum = plan_cum; da.info = plan_info; da.warp_seg = plan_warp_seg;
     da.B = B; da.Hq = Hq; da.Hkv = Hkv; da.g = Hq / Hkv; da.max_blocks = max_blocks;
     da.num_pages = num_pages; da.out = out; da.partial = partial;
+    da.ticket = plan_ticket; da.err = err;
     const int grid = nwarps / kDecWarps;
     if (num_pages <= 0 || num_pages * Hkv * P >= (1LL << 31)) {
         if (num_pages > 0) return ETI_ERR_UNSUPPORTED;   // tile rows are int32 on the device
@@ -446,9 +512,10 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
 #define ETI_DEC_CASE(DD, PP)                                                              \
     if (!launched && D == DD && P == PP) {                                                \
         auto k = paged_decode_kernel<DD, PP>;                                             \
-        const size_t sm = dec_smem_bytes<DD>();                                           \
+        const size_t sm = dec_smem_bytes<DD>(Hq / Hkv);                                   \
         cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);    \
-        k<<<grid, kDecThreads, sm, stream>>>(vmap, da);                                   \
+        if (eti_launch_pdl(k, dim3(grid), dim3(kDecThreads), sm, stream, vmap, da) != cudaSuccess) \
+            return ETI_ERR_CUDA;                                                          \
         launched = true;                                                                  \
     }
     ETI_DEC_CASE(128, 16)
@@ -457,13 +524,5 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
     ETI_DEC_CASE(64, 32)
 #undef ETI_DEC_CASE
     if (!launched) return ETI_ERR_UNSUPPORTED;
-    if (cudaGetLastError() != cudaSuccess) return ETI_ERR_CUDA;
-
-    CombArgs ca;
-    ca.cum = plan_cum; ca.info = plan_info; ca.partial = partial; ca.kept_norm = kept_norm;
-    ca.ctx_lens = ctx_lens; ca.block_table = block_table; ca.num_pages = num_pages;
-    ca.B = B; ca.Hq = Hq; ca.Hkv = Hkv; ca.g = Hq / Hkv; ca.D = D; ca.P = P;
-    ca.max_blocks = max_blocks; ca.out = out; ca.err = err;
-    decode_combine_kernel<<<nseg, 128, 0, stream>>>(ca);
     return cudaGetLastError() == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
 }

@@ -96,6 +96,8 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
     constexpr int S = ScoreRing<D>::kStages;
     constexpr int TB = ScoreRing<D>::kTile;
     constexpr int H = D / 64;                    // 64-element boxes per tile row
+    pdl_trigger();
+    pdl_wait();
     extern __shared__ __align__(1024) unsigned char score_smem_raw[];
     // swizzled TMA tiles must start on a 1024-byte boundary
     unsigned char* score_smem = score_smem_raw + ((1024 - (smem_u32(score_smem_raw) & 1023)) & 1023);
@@ -404,6 +406,8 @@ __host__ __device__ constexpr size_t fin_smem_bytes(int max_blocks, bool cache) 
 template <int G, bool kCache>
 __global__ void __launch_bounds__(kFinThreads)
 prune_finalize_kernel(const FinArgs a) {
+    pdl_trigger();
+    pdl_wait();
     extern __shared__ __align__(16) float fin_smem[];
     float* sh_score = fin_smem;                       // [max_blocks]: scores, then keep flags
     float* sh_m = fin_smem + a.max_blocks;            // [G][max_blocks] (kCache)
@@ -660,6 +664,325 @@ prune_finalize_kernel(const FinArgs a) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// prune_finalize for segments of up to 16 * NT block-heads, one CTA of NT
+// threads per (sequence, kv head).  Flat layout: with GP the power of two
+// >= G, thread t owns query head h = t % GP of the blocks j = t / GP +
+// k * (NT / GP), k < kFlatPer, so the stats loads are coalesced, every
+// (block, head) term stays in registers from the load to the kept-token
+// normaliser, e^{m_b - M} is evaluated once, and the per-head reductions run
+// over lanes of equal h.  The GP lanes of a block end up with the same group
+// score, so they take the same keep decision; ranks in ascending block order
+// (budget ties, compaction) come from ballots over the head-0 lanes.
+constexpr int kFlatPer = 16;
+
+template <int G>
+struct FlatGP { static constexpr int v = G <= 1 ? 1 : G <= 2 ? 2 : G <= 4 ? 4 : 8; };
+
+// per-head reduction of N values over the lanes (and warps) of equal h;
+// red holds N * 32 * GP floats and must not be reused before the next barrier
+template <int GP, int N, bool kMax>
+__device__ __forceinline__ void head_reduce(float (&v)[N], float* red) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int o = 16; o >= GP; o >>= 1)
+#pragma unroll
+        for (int i = 0; i < N; ++i) {
+            const float y = __shfl_xor_sync(0xffffffffu, v[i], o);
+            v[i] = kMax ? fmaxf(v[i], y) : v[i] + y;
+        }
+    if (lane < GP)
+#pragma unroll
+        for (int i = 0; i < N; ++i) red[(i * 32 + w) * GP + lane] = v[i];
+    __syncthreads();
+    const int h = lane & (GP - 1);
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        float r = kMax ? -kInf : 0.f;
+        for (int u = 0; u < nw; ++u) {
+            const float y = red[(i * 32 + u) * GP + h];
+            r = kMax ? fmaxf(r, y) : r + y;
+        }
+        v[i] = r;
+    }
+}
+
+// Exclusive ranks in ascending block order of the flagged blocks (flags
+// agree across the GP lanes of a block); returns the number flagged.
+// scan holds kFlatPer * 32 + 1 ints.
+template <int GP>
+__device__ __forceinline__ int flat_ranks(const bool (&f)[kFlatPer], int (&pos)[kFlatPer], int* scan) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    const bool lead = (lane & (GP - 1)) == 0;
+    const uint32_t below = (1u << (lane & ~(GP - 1))) - 1u;   // lanes of earlier blocks
+    uint32_t bal[kFlatPer];
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) {
+        bal[k] = __ballot_sync(0xffffffffu, f[k] && lead);
+        if (lane == 0) scan[k * nw + w] = __popc(bal[k]);
+    }
+    __syncthreads();
+    if (w == 0) {
+        // exclusive scan of the (chunk, warp) counts, chunk-major
+        const int E = kFlatPer * nw, per = (E + 31) >> 5;
+        const int e0 = min(lane * per, E), e1 = min(e0 + per, E);
+        int s = 0;
+        for (int e = e0; e < e1; ++e) s += scan[e];
+        int x = s;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        int run = x - s;
+        for (int e = e0; e < e1; ++e) { const int c = scan[e]; scan[e] = run; run += c; }
+        if (lane == 31) scan[E] = x;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) pos[k] = scan[k * nw + w] + __popc(bal[k] & below);
+    return scan[kFlatPer * nw];
+}
+
+template <int G, int NT>
+__global__ void __launch_bounds__(NT)
+prune_finalize_flat_kernel(const FinArgs a) {
+    constexpr int GP = FlatGP<G>::v;
+    constexpr int JS = NT / GP;                  // block stride between a thread's chunks
+    pdl_trigger();
+    pdl_wait();
+    extern __shared__ __align__(16) float ff_smem[];
+    float* sh_score = ff_smem;                   // [max_blocks] (budget select only)
+    __shared__ float red[4][2 * 32 * GP];
+    __shared__ int scan[2][kFlatPer * 32 + 1];
+    __shared__ int hist[256];
+    __shared__ int sel_digit, sel_rem;
+    __shared__ float arg_v[32];
+    __shared__ int arg_j[32];
+    const int seg = blockIdx.x;
+    const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int h = lane & (GP - 1);
+    const int jt = tid / GP;
+    const int L = a.ctx_lens[b];
+    const float th = a.theta[b];
+    const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
+    const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
+    const long long segbase = (long long)seg * a.max_blocks;
+    const float4* st = a.stats + segbase * G;
+
+    int bad = 0;
+    for (int j = tid; j < nb; j += NT) {
+        const int pg = a.block_table[(long long)b * a.max_blocks + j];
+        bad |= (pg < 0 || (long long)pg >= a.num_pages);
+    }
+    float m[kFlatPer], l1[kFlatPer], w[kFlatPer];   // w: u_b, then the block term I_b
+    int stale = 0;
+    float Mh[1] = {-kInf};
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) {
+        const int j = jt + k * JS;
+        m[k] = -kInf; l1[k] = 0.f; w[k] = 0.f;
+        if (h < G && j < nb) {
+            const float4 s = st[(long long)j * G + h];
+            m[k] = s.x; l1[k] = s.y; w[k] = s.z;
+            stale |= (s.x != s.x);              // NaN max: the scoring pass gave up on this block
+            Mh[0] = fmaxf(Mh[0], s.x);
+        }
+    }
+    const bool bad_page = __syncthreads_or(bad) != 0;
+    const bool timed_out = __syncthreads_or(stale) != 0 && !bad_page;
+    if (a.err && tid == 0) {
+        // err was cleared before this kernel; every kv head ORs in its bits
+        const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page ? ETI_ERRF_BAD_PAGE : 0u) |
+                           (timed_out ? ETI_ERRF_TIMEOUT : 0u);
+        if (e) atomicOr(a.err + b, e);
+    }
+    const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
+    bool valid[kFlatPer];
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) valid[k] = h < G && jt + k * JS < n;
+
+    float M = -kInf, score[kFlatPer];
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) score[k] = -kInf;
+    if (n > 0) {
+        head_reduce<GP, 1, true>(Mh, red[0]);
+        M = Mh[0];
+        // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
+        // c_b = e^{m_b - M}: the "1"s of the blocks at the max are counted, not
+        // summed, so log Z = log1p(Z - 1) keeps its relative precision when one
+        // token takes nearly all of the attention.
+        float zs[2] = {0.f, 0.f}, c[kFlatPer];
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k)
+            c[k] = 0.f;
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k)
+            if (valid[k]) {
+                const bool top = !(m[k] < M);
+                c[k] = top ? 1.f : expf(m[k] - M);
+                zs[0] += c[k] * l1[k] + (top ? 0.f : c[k]);
+                zs[1] += top ? 1.f : 0.f;
+            }
+        head_reduce<GP, 2, false>(zs, red[1]);
+        const float zm1 = zs[0] + (zs[1] - 1.f);
+        const float lZ = log1pf(zm1), Z = 1.f + zm1;
+        // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
+        // (l1 becomes (1 + l1_b) e^{m_b - M}, the block's share of Z)
+        float Hs[1] = {0.f};
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k)
+            if (valid[k]) {
+                w[k] = c[k] * ((1.f + l1[k]) * (lZ + M - m[k]) - w[k]) / Z;
+                Hs[0] += w[k];
+                l1[k] = (1.f + l1[k]) * c[k];
+            }
+        head_reduce<GP, 1, false>(Hs, red[2]);
+        // group score: the largest normalised term over the heads of the block
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            float s = valid[k] ? (Hs[0] > 0.f ? (float)n * w[k] / Hs[0] : 1.f) : -kInf;
+#pragma unroll
+            for (int o = 1; o < GP; o <<= 1) s = fmaxf(s, __shfl_xor_sync(0xffffffffu, s, o));
+            score[k] = s;
+        }
+    }
+    if (a.block_score) {
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const int j = jt + k * JS;
+            if (h == 0 && j < n) a.block_score[segbase + j] = score[k];
+        }
+        for (int j = n + tid; j < a.max_blocks; j += NT) a.block_score[segbase + j] = 0.f;
+    }
+
+    // B_min budget: the first k blocks by (score desc, index asc)
+    const int kb = min(max(a.B_min, 0), n);
+    bool keep[kFlatPer];
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) keep[k] = jt + k * JS < n && (score[k] >= th || kb >= n);
+    if (kb == 1 && n > 1) {
+        float bs = -kInf;
+        int bj = 0x7fffffff;
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const int j = jt + k * JS;
+            if (j < n && (score[k] > bs || bj == 0x7fffffff)) { bs = score[k]; bj = j; }
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bs, o);
+            const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+            if (ov > bs || (ov == bs && oj < bj)) { bs = ov; bj = oj; }
+        }
+        if (lane == 0) { arg_v[tid >> 5] = bs; arg_j[tid >> 5] = bj; }
+        __syncthreads();
+        for (int u = 0; u < NT / 32; ++u)
+            if (arg_v[u] > bs || (arg_v[u] == bs && arg_j[u] < bj)) { bs = arg_v[u]; bj = arg_j[u]; }
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) keep[k] |= (jt + k * JS == bj);
+    } else if (kb > 1 && kb < n) {
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const int j = jt + k * JS;
+            if (h == 0 && j < n) sh_score[j] = score[k];
+        }
+        __syncthreads();
+        uint32_t prefix = 0, mask = 0;
+        int need = kb;
+        for (int digit = 3; digit >= 0; --digit) {
+            const int sh = digit * 8;
+            for (int i = tid; i < 256; i += NT) hist[i] = 0;
+            __syncthreads();
+            for (int j = tid; j < n; j += NT) {
+                const uint32_t key = order_key(sh_score[j]);
+                if ((key & mask) == prefix) atomicAdd(&hist[(key >> sh) & 255], 1);
+            }
+            __syncthreads();
+            // bucket where the count from the top reaches `need`
+            if (tid < 32) {
+                int cnt8[8], s8 = 0;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) { cnt8[e] = hist[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
+                int incl = s8;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (tid >= o) incl += y;
+                }
+                int above = incl - s8;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    if (above < need && need <= above + cnt8[e]) {
+                        sel_digit = 255 - (tid * 8 + e);
+                        sel_rem = need - above;
+                    }
+                    above += cnt8[e];
+                }
+            }
+            __syncthreads();
+            prefix |= (uint32_t)sel_digit << sh;
+            mask |= 255u << sh;
+            need = sel_rem;
+            __syncthreads();
+        }
+        // keys above the k-th are in; of those equal to it, the lowest indices
+        bool eq[kFlatPer];
+        int eq_pos[kFlatPer];
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const uint32_t key = order_key(score[k]);
+            eq[k] = jt + k * JS < n && key == prefix;
+            keep[k] |= jt + k * JS < n && key > prefix;
+        }
+        flat_ranks<GP>(eq, eq_pos, scan[0]);
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) keep[k] |= eq[k] && eq_pos[k] < need;
+    }
+
+    // compaction (ascending block index)
+    int pos[kFlatPer];
+    const int total = flat_ranks<GP>(keep, pos, scan[1]);
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) {
+        const int j = jt + k * JS;
+        if (h == 0 && keep[k]) a.kept_idx[segbase + pos[k]] = j;
+        if (a.keep_mask && h == 0 && j < n) a.keep_mask[segbase + j] = keep[k] ? 1 : 0;
+    }
+    for (int i = total + tid; i < a.max_blocks; i += NT) a.kept_idx[segbase + i] = -1;
+    if (a.keep_mask)
+        for (int j = n + tid; j < a.max_blocks; j += NT) a.keep_mask[segbase + j] = 0;
+    if (tid == 0) a.kept_cnt[seg] = total;
+
+    // softmax normaliser over the kept tokens of each query head
+    if (a.kept_norm) {
+        float Mk[1] = {-kInf};
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k)
+            if (valid[k] && keep[k]) Mk[0] = fmaxf(Mk[0], m[k]);
+        head_reduce<GP, 1, true>(Mk, red[3]);
+        float Lk[1] = {0.f};
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k)
+            if (valid[k] && keep[k]) {
+                if (Mk[0] == M) {
+                    Lk[0] += l1[k];
+                } else {
+                    // the largest logit's block was pruned: rescale from the stats
+                    const float4 s = st[(long long)(jt + k * JS) * G + h];
+                    Lk[0] += (1.f + s.y) * expf(s.x - Mk[0]);
+                }
+            }
+        head_reduce<GP, 1, false>(Lk, red[0]);
+        if (tid < GP && h < G) {
+            float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2;
+            kn[0] = Mk[0];
+            kn[1] = Lk[0];
+        }
+    }
+}
+
 }  // namespace eti
 
 using namespace eti;
@@ -686,15 +1009,14 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int grid = 2 * sms;
     cudaError_t e;
 #define ETI_SCORE_CASE(DD, PP)                                                              \
     if (D == DD && P == PP) {                                                               \
         auto k = score_blocks_kernel<DD, PP>;                                               \
         const size_t smem = score_smem_bytes<DD, PP>(B);                                    \
+        const int grid = (smem + 2048 <= 233472 / 2 ? 2 : 1) * sms;   /* CTAs that fit */   \
         cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);    \
-        k<<<grid, kScoreThreads, smem, stream>>>(kmap, a);                                  \
-        e = cudaGetLastError();                                                             \
+        e = eti_launch_pdl(k, dim3(grid), dim3(kScoreThreads), smem, stream, kmap, a);      \
         return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;                                    \
     }
     ETI_SCORE_CASE(128, 16)
@@ -725,14 +1047,29 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     int dev = 0, optin = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    // the flat kernel holds a segment in registers: 16 block-heads a thread
+    const int gp = a.g <= 1 ? 1 : a.g <= 2 ? 2 : a.g <= 4 ? 4 : 8;
+    const long long flat_need = ((long long)max_blocks * gp + kFlatPer - 1) / kFlatPer;
+    const int flat_nt = !given && theta && flat_need <= 512
+                            ? (flat_need <= 128 ? 128 : flat_need <= 256 ? 256 : 512) : 0;
+#define ETI_FIN_FLAT(GG, NT)                                                                \
+    if (flat_nt == NT) {                                                                    \
+        auto k = prune_finalize_flat_kernel<GG, NT>;                                        \
+        const size_t smem = (size_t)max_blocks * 4;                                         \
+        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
+        e = eti_launch_pdl(k, dim3(grid), dim3(NT), smem, stream, a);                       \
+        break;                                                                              \
+    }
 #define ETI_FIN_CASE(GG)                                                                    \
     case GG: {                                                                              \
+        ETI_FIN_FLAT(GG, 128)                                                               \
+        ETI_FIN_FLAT(GG, 256)                                                               \
+        ETI_FIN_FLAT(GG, 512)                                                               \
         const bool cache = fin_smem_bytes<GG>(max_blocks, true) <= (size_t)optin / 2;      \
         const size_t smem = fin_smem_bytes<GG>(max_blocks, cache);                          \
         auto k = cache ? prune_finalize_kernel<GG, true> : prune_finalize_kernel<GG, false>; \
         if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-        k<<<grid, kFinThreads, smem, stream>>>(a);                                          \
-        e = cudaGetLastError();                                                             \
+        e = eti_launch_pdl(k, dim3(grid), dim3(kFinThreads), smem, stream, a);              \
         break;                                                                              \
     }
     switch (a.g) {
@@ -747,5 +1084,6 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
         default: return ETI_ERR_UNSUPPORTED;
     }
 #undef ETI_FIN_CASE
+#undef ETI_FIN_FLAT
     return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
 }
