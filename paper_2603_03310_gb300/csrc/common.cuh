@@ -147,6 +147,17 @@ __device__ __forceinline__ void bulk_load_1d(uint32_t dst, const void* src, uint
         :: "r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
 }
 
+// Four 8x8 b16 matrices from shared memory, each transposed (ldmatrix .trans):
+// lane l gives the address of row l % 8 of matrix l / 8 (16 contiguous bytes);
+// register i of lane (4 g + t) then holds rows 2t, 2t+1 of column g of matrix i.
+__device__ __forceinline__ void ldsm_x4_trans(uint32_t (&r)[4], uint32_t addr) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]) : "r"(addr) : "memory");
+}
+__device__ __forceinline__ void sts_zero_u4(uint32_t addr) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %1, %1, %1};" :: "r"(addr), "r"(0u) : "memory");
+}
+
 // Offset of the 16-byte chunk `chunk` of row `row` inside a TMA box with
 // 128-byte rows and the 128-byte swizzle (chunk index xor row mod 8).
 __device__ __forceinline__ uint32_t swz128(int row, int chunk) {

@@ -138,10 +138,8 @@ struct DecArgs {
 
 template <int D>
 struct DecLayout {
-    static constexpr int E = D / 16;              // bf16 per row half per thread
     static constexpr int kTile = 16 * D * 2;      // bytes of one 16-token V tile
     static constexpr int kStages = D == 128 ? 3 : 5;
-    using Vec = typename std::conditional<E == 8, uint4, uint2>::type;
 };
 
 // bytes of one tile's scores (16 tokens x g heads, fp32)
@@ -153,53 +151,16 @@ __host__ __device__ inline size_t dec_smem_bytes(int g) {
            + (size_t)kDecWarps * 64 * 16;
 }
 
-template <int D>
-__device__ __forceinline__ uint32_t vreg(const typename DecLayout<D>::Vec& v, int i) {
-    if constexpr (DecLayout<D>::E == 8) {
-        return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
-    } else {
-        return i == 0 ? v.x : v.y;
-    }
-}
-
-// bf16 element j of rows (ra, rb) packed as (ra.j, rb.j)
-template <int D>
-__device__ __forceinline__ uint32_t pair_elem(const typename DecLayout<D>::Vec& ra,
-                                              const typename DecLayout<D>::Vec& rb, int j) {
-    const uint32_t x = vreg<D>(ra, j >> 1), y = vreg<D>(rb, j >> 1);
-    return (j & 1) ? hi_halves(x, y) : lo_halves(x, y);
-}
-
 // A-fragment rows owned by a thread (tq = lane & 3): 2tq, 2tq+1, 2tq+8, 2tq+9
 __device__ __forceinline__ int frag_row(int tq, int k) { return 2 * tq + (k & 1) + (k >> 1) * 8; }
-
-// The thread's E elements of row `row`, half `half` (d = half * D/2 + E * grp),
-// from a 128-byte-swizzled tile (one 2 KB box per 64-element half for D = 128).
-template <int D>
-__device__ __forceinline__ typename DecLayout<D>::Vec lds_row(uint32_t tile, int row, int half, int grp) {
-    if constexpr (D == 128) {
-        return lds_u4(tile + half * 2048 + swz128(row, grp));
-    } else {
-        return lds_u2(tile + swz128(row, 4 * half + (grp >> 1)) + (grp & 1) * 8);
-    }
-}
-
-template <int D>
-__device__ __forceinline__ typename DecLayout<D>::Vec zero_vec() {
-    typename DecLayout<D>::Vec z;
-    if constexpr (DecLayout<D>::E == 8) z = make_uint4(0, 0, 0, 0);
-    else z = make_uint2(0, 0);
-    return z;
-}
 
 template <int D, int P>
 __global__ void __launch_bounds__(kDecThreads, 2)
 paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
-    using LY = DecLayout<D>;
     constexpr int kTiles = P / 16;
     constexpr int J = D / 16;                    // MMAs per 16-token tile
-    constexpr int S = LY::kStages;
-    constexpr int TB = LY::kTile;
+    constexpr int S = DecLayout<D>::kStages;
+    constexpr int TB = DecLayout<D>::kTile;
     constexpr int H = D / 64;                    // 64-element boxes per tile row
     pdl_trigger();
     pdl_wait();
@@ -338,30 +299,26 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
         const int lo = __ldg(a.cum + seg), hi = __ldg(a.cum + seg + 1);
         const bool whole = lo >= u0 && hi <= u1;
         const bool bad = (a.err[b] & (ETI_ERRF_BAD_CTX | ETI_ERRF_BAD_PAGE)) != 0u;
+        // acc[j][e], acc[j][2 + e]: head 2 tq + e at d = 16 j + grp and 16 j + 8 + grp
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
             const int h = 2 * tq + e;
             if (h < a.g) {
+                if (whole) {
+                    const float l = __ldg(a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2 + 1);
+                    const float inv = (!bad && l > 0.f) ? 1.f / l : 0.f;
+                    uint16_t* o = a.out + ((long long)b * a.Hq + kvh * a.g + h) * D + grp;
 #pragma unroll
-                for (int half = 0; half < 2; ++half) {
-                    const int d0 = half * (D / 2) + J * grp;
-                    float v[J];
+                    for (int j = 0; j < J; ++j) {
+                        o[16 * j] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[j][e] * inv));
+                        o[16 * j + 8] = __bfloat16_as_ushort(__float2bfloat16_rn(acc[j][2 + e] * inv));
+                    }
+                } else {
+                    float* o = a.partial + ((long long)(warp + seg) * a.g + h) * D + grp;
 #pragma unroll
-                    for (int j = 0; j < J; ++j) v[j] = acc[j][2 * half + e];
-                    if (whole) {
-                        const float l = __ldg(a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2 + 1);
-                        const float inv = (!bad && l > 0.f) ? 1.f / l : 0.f;
-                        uint32_t pk[J / 2];
-#pragma unroll
-                        for (int j = 0; j < J / 2; ++j) pk[j] = pack_bf16x2(v[2 * j] * inv, v[2 * j + 1] * inv);
-                        uint16_t* o = a.out + ((long long)b * a.Hq + kvh * a.g + h) * D + d0;
-                        if constexpr (J == 8) *reinterpret_cast<uint4*>(o) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                        else *reinterpret_cast<uint2*>(o) = make_uint2(pk[0], pk[1]);
-                    } else {
-                        float* o = a.partial + ((long long)(warp + seg) * a.g + h) * D + d0;
-#pragma unroll
-                        for (int j = 0; j < J; j += 4)
-                            *reinterpret_cast<float4*>(o + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+                    for (int j = 0; j < J; ++j) {
+                        o[16 * j] = acc[j][e];
+                        o[16 * j + 8] = acc[j][2 + e];
                     }
                 }
             }
@@ -408,19 +365,36 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
             Mh = grp < a.g ? __ldg(a.kept_norm + ((long long)b * a.Hq + kvh * a.g + grp) * 2) : 0.f;
         }
         const uint32_t tb = tiles + st * TB, sc = scores + st * SB;
-        const int vrow = e.z >= 0 ? e.w - tile * 16 : 0;   // valid rows of this tile
-        typename LY::Vec r[4][2];
+        // valid rows of this tile, in [0, 16] (the second tile of a 32-token page
+        // can lie wholly past the sequence end)
+        const int vrow = e.z >= 0 ? max(0, min(16, e.w - tile * 16)) : 0;
+        if (vrow < 16) {
+            // rows past the sequence end (or of a skipped page) hold whatever the
+            // stage holds: zero them, so that a finite weight meets a zero row
+            for (int c = lane; c < (16 - vrow) * (D / 8); c += 32) {
+                const int row = vrow + c / (D / 8), ch = c % (D / 8);
+                sts_zero_u4(tb + (ch >> 3) * 2048 + row * 128 + (ch & 7) * 16);
+            }
+            __syncwarp();
+        }
         float p[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
             const int row = frag_row(tq, k);
-            const bool ok = row < vrow;
-            // rows past the sequence end hold whatever the page holds: zero them
-            r[k][0] = ok ? lds_row<D>(tb, row, 0, grp) : zero_vec<D>();
-            r[k][1] = ok ? lds_row<D>(tb, row, 1, grp) : zero_vec<D>();
-            const float x = (ok && grp < a.g) ? lds_f32(sc + (row * a.g + grp) * 4) : 0.f;
+            const float x = (row < vrow && grp < a.g) ? lds_f32(sc + (row * a.g + grp) * 4) : 0.f;
             // kept tokens have x <= M_h; zeroed rows get a finite weight against a zero row
             p[k] = fast_ex2(fminf((x - Mh) * kLog2e, 0.f));
+        }
+        // A fragments of V^T (head_dim = M, tokens = K), MMA j on d = 16 j .. 16 j + 15:
+        // matrix q of lane l is (tokens 8 (q >> 1) .. +7, d = 16 j + 8 (q & 1) .. +7)
+        uint32_t af[J][4];
+        {
+            const int q = lane >> 3, rr = (lane & 7) + (q >> 1) * 8;
+#pragma unroll
+            for (int j = 0; j < J; ++j) {
+                const int d = 16 * j + 8 * (q & 1);
+                ldsm_x4_trans(af[j], tb + (d >> 6) * 2048 + swz128(rr, (d & 63) >> 3));
+            }
         }
         // the stage may be refilled now
         __syncwarp();
@@ -429,13 +403,7 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
         const uint32_t b0 = pack_bf16x2(p[0], p[1]);
         const uint32_t b1 = pack_bf16x2(p[2], p[3]);
 #pragma unroll
-        for (int j = 0; j < J; ++j) {
-            const uint32_t a0 = pair_elem<D>(r[0][0], r[1][0], j);
-            const uint32_t a1 = pair_elem<D>(r[0][1], r[1][1], j);
-            const uint32_t a2 = pair_elem<D>(r[2][0], r[3][0], j);
-            const uint32_t a3 = pair_elem<D>(r[2][1], r[3][1], j);
-            mma_bf16_16x8x16(acc[j], a0, a1, a2, a3, b0, b1);
-        }
+        for (int j = 0; j < J; ++j) mma_bf16_16x8x16(acc[j], af[j][0], af[j][1], af[j][2], af[j][3], b0, b1);
     }
     if (timed_out) {
         // a copy never arrived: let the ones in flight land (bounded), flag
