@@ -160,10 +160,12 @@ def ncu_traffic(kernel):
     import hashlib
     try:
         rec = json.load(open(os.path.join(ROOT, "profiles", "ncu_traffic.json")))[kernel]
-        src = open(os.path.join(ROOT, rec["source"]), "rb").read()
+        h = hashlib.sha256()
+        for path in rec["sources"]:
+            h.update(open(os.path.join(ROOT, path), "rb").read())
     except (OSError, KeyError, TypeError, ValueError):
         return None
-    return rec["bytes"] if hashlib.sha256(src).hexdigest() == rec["sha256"] else None
+    return rec["bytes"] if h.hexdigest() == rec["sha256"] else None
 
 
 def run_gpu(args):
@@ -277,7 +279,8 @@ def run_gpu(args):
         peak, peak_src = 6800.0, "fallback"
     achieved = {n: abytes[n] / (mean_ms[n] / 1e3) / 1e9 for n in names}
     traffic = args.traffic if args.traffic is not None else ncu_traffic(
-        {"score": "score_blocks", "prune": "prune_finalize", "decode": "paged_decode"}.get(dom))
+        {"score": "score_blocks", "prune": "prune_finalize", "decode": "paged_decode",
+         "sample": "entropy_sample_partial"}.get(dom))
     roof = {"kernel": {"score": "score_blocks", "prune": "prune_finalize",
                        "decode": "paged_decode (plan + decode; split segments merged in-kernel)",
                        "sample": "entropy_temp_sample"}[dom],
