@@ -135,22 +135,9 @@ __device__ __forceinline__ RowState state_shfl_xor(const RowState& s, int o) {
 // warp).  Only the tokens that pass evaluate E2, so the draw is unchanged.
 constexpr float kRaceKappa = 1.4426950408889634f * (1.0f - 1.0f / 65536.0f);
 
-// One token: entropy sums and the race.
-__device__ __forceinline__ void consume(RowState& s, float& rk, float z, uint32_t word, int x, float c) {
-    const float t = fmaf(z, c, -s.mc);
-    const float w = fast_ex2(t);
-    s.S += w;
-    s.U = fmaf(w, fmaxf(t, -250.f), s.U);   // -inf logits add 0 (w = 0); NaN still reaches S
-    // 1 - u = (2 (0x7FFFFF - j) + 1) 2^-24, formed exactly like u
-    const float v = __uint_as_float((~word & 0x7FFFFFu) | 0x3F800000u) - __uint_as_float(0x3F7FFFFFu);
-    if (w > rk * v) {                         // rare once rk has grown
-        const float E = exp_variate_log2(word);
-        if (w > s.r * E) {
-            s.r = __fdividef(w, E);
-            s.bi = x;
-            rk = fmaxf(rk, s.r * kRaceKappa);
-        }
-    }
+// v = 1 - u = (2 (0x7FFFFF - j) + 1) 2^-24 for the word's uniform u, formed exactly
+__device__ __forceinline__ float one_minus_u(uint32_t word) {
+    return __uint_as_float((~word & 0x7FFFFFu) | 0x3F800000u) - __uint_as_float(0x3F7FFFFFu);
 }
 
 constexpr int kEtsThreads = 256;
@@ -167,6 +154,8 @@ struct EtsArgs {
     const float* H_target;
     eti_ctrl_params p;
     uint32_t seed_lo, seed_hi, off_lo, off_hi;
+    uint32_t rk0[10], rk1[10];   // Philox round keys (the key bumped r times); the kernels
+                                 // read them from the parameter bank, not from registers
     int32_t* tok;
     float* H;
     float* T_out;
@@ -198,7 +187,7 @@ __device__ __forceinline__ void load_group(float (&z)[4], const float* row, int 
 // row-major list of all rows' 4-token groups, one row piece at a time.
 template <bool kVec>
 __global__ void __launch_bounds__(kEtsThreads, kEtsCtasPerSm)
-entropy_sample_partial_kernel(const EtsArgs a) {
+entropy_sample_partial_kernel(const __grid_constant__ EtsArgs a) {
     pdl_trigger();
     pdl_wait();
     __shared__ RowState warp_part[kEtsThreads / 32];
@@ -207,12 +196,6 @@ entropy_sample_partial_kernel(const EtsArgs a) {
     long long q0 = (long long)blockIdx.x * a.share;
     const long long q1 = min(q0 + a.share, total);
     const int full_groups = a.V >> 2;
-    uint32_t k0[10], k1[10];
-#pragma unroll
-    for (int r = 0; r < 10; ++r) {
-        k0[r] = a.seed_lo + (uint32_t)r * 0x9E3779B9u;
-        k1[r] = a.seed_hi + (uint32_t)r * 0xBB67AE85u;
-    }
     while (q0 < q1) {
         const int b = (int)(q0 / a.ngroups);
         const int g0 = (int)(q0 - (long long)b * a.ngroups);
@@ -256,16 +239,39 @@ entropy_sample_partial_kernel(const EtsArgs a) {
                     if (nan) s.S = __int_as_float(0x7fc00000);
                 } else {
                     if (bm > s.m) rk *= state_rebase(s, bm, c);
+                    // entropy sums for every token, the race prefilter folded into
+                    // one flag; groups past the piece hold -inf (w = 0, never drawn)
+                    float w[kEtsPair][4];
+                    uint32_t word[kEtsPair][4];
+                    bool any = false;
 #pragma unroll
                     for (int k = 0; k < kEtsPair; ++k) {
                         const int g = base + k * kEtsThreads + tid;
-                        if (g < g1) {
-                            const uint4 r = philox4x32_10(make_uint4((uint32_t)g, (uint32_t)b, a.off_lo, a.off_hi), k0, k1);
-                            consume(s, rk, cur[k][0], r.x, 4 * g + 0, c);
-                            consume(s, rk, cur[k][1], r.y, 4 * g + 1, c);
-                            consume(s, rk, cur[k][2], r.z, 4 * g + 2, c);
-                            consume(s, rk, cur[k][3], r.w, 4 * g + 3, c);
+                        const uint4 r = philox4x32_10(make_uint4((uint32_t)g, (uint32_t)b, a.off_lo, a.off_hi), a.rk0, a.rk1);
+                        word[k][0] = r.x; word[k][1] = r.y; word[k][2] = r.z; word[k][3] = r.w;
+#pragma unroll
+                        for (int e = 0; e < 4; ++e) {
+                            const float t = fmaf(cur[k][e], c, -s.mc);
+                            w[k][e] = fast_ex2(t);
+                            s.S += w[k][e];
+                            s.U = fmaf(w[k][e], fmaxf(t, -250.f), s.U);   // -inf adds 0; NaN reaches S
+                            any |= w[k][e] > rk * one_minus_u(word[k][e]);
                         }
+                    }
+                    if (any) {
+                        // rare once rk has grown: the exact race, in token order
+#pragma unroll
+                        for (int k = 0; k < kEtsPair; ++k)
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                if (w[k][e] > rk * one_minus_u(word[k][e])) {
+                                    const float E = exp_variate_log2(word[k][e]);
+                                    if (w[k][e] > s.r * E) {
+                                        s.r = __fdividef(w[k][e], E);
+                                        s.bi = 4 * (base + k * kEtsThreads + tid) + e;
+                                        rk = fmaxf(rk, s.r * kRaceKappa);
+                                    }
+                                }
                     }
                 }
                 if (!more) break;
@@ -398,6 +404,10 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
     a.logits = logits; a.B = B; a.V = V; a.ld = ld; a.T_in = T_in; a.H_prev = H_prev;
     a.tau = tau; a.H_target = H_target; a.p = *p;
     a.seed_lo = (uint32_t)seed; a.seed_hi = (uint32_t)(seed >> 32);
+    for (int r = 0; r < 10; ++r) {
+        a.rk0[r] = a.seed_lo + (uint32_t)r * 0x9E3779B9u;
+        a.rk1[r] = a.seed_hi + (uint32_t)r * 0xBB67AE85u;
+    }
     a.off_lo = (uint32_t)offset; a.off_hi = (uint32_t)(offset >> 32);
     a.tok = tok; a.H = H; a.T_out = T_out; a.dH = dH; a.theta_next = theta_next;
     a.surprisal = surprisal; a.err = err;
