@@ -75,7 +75,7 @@ def _load():
             lib.oracle_entropy_temp_sample.argtypes = (
                 [P, i32, i64, i64, P, P, P, P, P, u64, u64] + [P] * 9)
             lib.oracle_score_prune.argtypes = (
-                [P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, i32] + [P] * 8)
+                [P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, i32, i32, P] + [P] * 8)
             lib.oracle_paged_attention.argtypes = (
                 [P, P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, P, P])
             _lib = lib
@@ -161,12 +161,18 @@ def entropy_temp_sample(logits, T_in, H_prev, tau_in, H_target, ctrl_params=None
     return out
 
 
+SCORE_A, SCORE_E, SCORE_M = 0, 1, 2
+
+
 def score_prune(q, k_cache, block_table, ctx_lens, scale: float, theta, B_min: int,
-                num_pages: int | None = None, want_heads: bool = False):
+                num_pages: int | None = None, want_heads: bool = False,
+                score_mode: int = SCORE_A, surp=None):
     """Entropic block scores, keep mask and compacted kept lists.
 
     q: bf16 bit patterns uint16 [B, Hq, D]; k_cache uint16 [pages, Hkv, P, D];
-    block_table int32 [B, max_blocks]; ctx_lens int32 [B]; theta float32 [B].
+    block_table int32 [B, max_blocks]; ctx_lens int32 [B]; theta float32 [B];
+    score_mode 0 (A: -log a_i), 1 (E: stored token surprisal surp float32
+    [pages, P]) or 2 (M: attention mass).
     """
     lib = _load()
     q = _c(q, np.uint16)
@@ -187,8 +193,14 @@ def score_prune(q, k_cache, block_table, ctx_lens, scale: float, theta, B_min: i
     head_A = np.empty((B, Hq, mb), np.float64) if want_heads else None
     head_H = np.empty((B, Hq), np.float64) if want_heads else None
     err = np.empty(B, np.uint32)
+    if score_mode == SCORE_E:
+        surp = _c(surp, np.float32)
+        assert surp.shape == (pages, P)
+    else:
+        surp = None
     lib.oracle_score_prune(_ptr(q), _ptr(k_cache), _ptr(bt), _ptr(cl), B, Hq, Hkv, D, P, mb,
-                           num_pages, float(scale), _ptr(th), int(B_min), _ptr(keep), _ptr(kidx),
+                           num_pages, float(scale), _ptr(th), int(B_min), int(score_mode),
+                           _ptr(surp), _ptr(keep), _ptr(kidx),
                            _ptr(kcnt), _ptr(score), _ptr(head_I), _ptr(head_A), _ptr(head_H),
                            _ptr(err))
     res = dict(keep_mask=keep, kept_idx=kidx, kept_cnt=kcnt, block_score=score, err=err)

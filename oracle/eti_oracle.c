@@ -21,7 +21,11 @@
  *       sigma = -1 restores (H grows with T), sigma = +1 is the printed form.
  *   R2  entropy, sample and surprisal all use the incoming T_t; T' is for t+1.
  *   R4  block surprisal I(v_i) := -log a_i (attention as a distribution over
- *       the values), so sum_b I_b is the attention entropy.
+ *       the values), so sum_b I_b is the attention entropy (score mode A, the
+ *       default).  The other readings of "the surprisal associated with the
+ *       value vector": mode E, I(v_i) := the stored surprisal -log p(x_i |
+ *       x_<i) of the token at position i (recorded when it was generated);
+ *       mode M, I(v_i) := 1, so I_b is the block's attention mass.
  *   R5  one keep decision per (sequence, kv head, block); group score is the
  *       max over the query heads that share the kv head.
  *   R6  threshold applies to the normalised score n_b * I_b / sum_b' I_b'.
@@ -285,7 +289,9 @@ static int rank_cmp(const void *pa, const void *pb) {
  * Entropic block scores and keep set (Section 3.2 with readings R4-R7).
  *
  * For each query head h and token i < L_b:  a_i = softmax_i(x_i) over all
- * L_b tokens;  I_b^(h) = sum_{i in block} a_i * (-log a_i);
+ * L_b tokens;  I_b^(h) = sum_{i in block} a_i * I_i with I_i = -log a_i
+ * (score_mode 0, A), surp[page(i) * P + i mod P] (1, E: the stored token
+ * surprisal, paged like the keys: [num_pages][P]) or 1 (2, M);
  * normalised  Ibar_b^(h) = n_b I_b^(h) / sum_b' I_b'^(h)  (1 when the sum is 0);
  * group score Ibar_b = max over the heads of the kv group.
  * keep_b  iff  Ibar_b >= theta[b]  or  b is among the first min(B_min, n_b)
@@ -301,7 +307,7 @@ static int rank_cmp(const void *pa, const void *pb) {
 void oracle_score_prune(const uint16_t *q, const uint16_t *k_cache, const int32_t *block_table,
                         const int32_t *ctx_lens, int B, int Hq, int Hkv, int D, int P,
                         int max_blocks, int64_t num_pages, double scale,
-                        const float *theta, int B_min,
+                        const float *theta, int B_min, int score_mode, const float *surp,
                         uint8_t *keep_mask, int32_t *kept_idx, int32_t *kept_cnt,
                         double *block_score, double *head_I, double *head_A, double *head_H,
                         uint32_t *err) {
@@ -345,7 +351,14 @@ void oracle_score_prune(const uint16_t *q, const uint16_t *k_cache, const int32_
                     for (int i = j * P; i < i1; ++i) {
                         double a = exp(x[i] - M) / Z;
                         mass += a;
-                        if (a > 0.0) s += a * (-log(a));
+                        if (score_mode == 1) {
+                            int64_t page = block_table[(int64_t)b * max_blocks + j];
+                            s += a * (double)surp[page * P + (i - j * P)];
+                        } else if (score_mode == 2) {
+                            s += a;
+                        } else if (a > 0.0) {
+                            s += a * (-log(a));
+                        }
                     }
                     Ih[j] = s;
                     Ah[j] = mass;

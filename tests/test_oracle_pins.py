@@ -397,6 +397,92 @@ def test_uniform_attention_closed_form():
             assert np.allclose(r["block_score"][b, kvh, :nb], want, rtol=0, atol=1e-12)
 
 
+def _page_store(n, per_token, seed=0):
+    """A token-surprisal store [pages, P] holding per_token(b, i) at the slot of
+    token i of sequence b (other slots: a large poison value)."""
+    pages, _, P, _ = n["k"].shape
+    store = np.full((pages, P), 1e30, np.float32)
+    for b in range(len(n["L"])):
+        for i in range(int(n["L"][b])):
+            store[n["bt"][b, i // P], i % P] = per_token(b, i)
+    return store
+
+
+def _torch_attention(n, b, h, g):
+    K = torch.from_numpy(_dense(n, b, "k"))
+    x = (K[h // g] @ torch.from_numpy(_q(n)[b, h])) * n["scale"]
+    return torch.softmax(x, 0).numpy()
+
+
+def test_score_mode_M_is_the_block_attention_mass():
+    """Mode M (I(v_i) := 1): I_b is the block's attention mass, the masses add to
+    1 per head, and the group score is max_h n_b * mass_b (torch softmax)."""
+    w, kv, n = _small_kv()
+    r = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1,
+                           want_heads=True, score_mode=oracle.SCORE_M)
+    g = w.Hq // w.Hkv
+    for b in range(w.B):
+        nb = -(-int(n["L"][b]) // w.P)
+        best = np.full((w.Hkv, nb), -np.inf)
+        for h in range(w.Hq):
+            a = _torch_attention(n, b, h, g)
+            mass = np.array([a[j * w.P:(j + 1) * w.P].sum() for j in range(nb)])
+            assert np.allclose(r["head_I"][b, h, :nb], mass, atol=1e-12)
+            assert abs(r["head_H"][b, h] - 1.0) < 1e-12
+            best[h // g] = np.maximum(best[h // g], nb * mass)
+        assert np.allclose(r["block_score"][b, :, :nb], best, atol=1e-10)
+
+
+def test_score_mode_E_brute_force_with_page_lookup():
+    """Mode E: I_b = sum a_i s_i with s_i read through the block table from a
+    paged store; checked against torch attention weights and the unpaged s."""
+    w, kv, n = _small_kv(seed=5)
+    rng = np.random.default_rng(3)
+    s_tok = [rng.exponential(2.0, int(L)).astype(np.float32) for L in n["L"]]
+    store = _page_store(n, lambda b, i: s_tok[b][i])
+    r = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1,
+                           want_heads=True, score_mode=oracle.SCORE_E, surp=store)
+    g = w.Hq // w.Hkv
+    for b in range(w.B):
+        nb = -(-int(n["L"][b]) // w.P)
+        best = np.full((w.Hkv, nb), -np.inf)
+        for h in range(w.Hq):
+            a = _torch_attention(n, b, h, g)
+            t = a * s_tok[b].astype(np.float64)
+            I = np.array([t[j * w.P:(j + 1) * w.P].sum() for j in range(nb)])
+            assert np.allclose(r["head_I"][b, h, :nb], I, rtol=1e-12, atol=1e-14)
+            best[h // g] = np.maximum(best[h // g], nb * I / I.sum())
+        assert np.allclose(r["block_score"][b, :, :nb], best, rtol=1e-10)
+
+
+def test_score_mode_E_with_attention_surprisal_is_mode_A():
+    """One head per sequence: storing s_i = -log a_i (fp64 torch) turns mode E
+    into mode A, so the two readings agree where they must."""
+    w, kv, n = _small_kv(Hq=1, Hkv=1, seed=9)
+    a = {b: _torch_attention(n, b, 0, 1) for b in range(w.B)}
+    store = _page_store(n, lambda b, i: -np.log(a[b][i]))
+    rA = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1)
+    rE = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1,
+                            score_mode=oracle.SCORE_E, surp=store)
+    # the store holds s_i rounded to fp32: relative 2^-24 per term
+    assert np.allclose(rE["block_score"], rA["block_score"], rtol=1e-6, atol=1e-9)
+    assert np.array_equal(rE["keep_mask"], rA["keep_mask"])
+
+
+def test_score_mode_E_constant_and_zero_surprisal():
+    """s_i = c > 0 for every token gives mode M (c cancels in the
+    normalisation); s_i = 0 makes every sum 0, so every block scores 1."""
+    w, kv, n = _small_kv(seed=13)
+    args = (n["q"], n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1)
+    rM = oracle.score_prune(*args, score_mode=oracle.SCORE_M)
+    rC = oracle.score_prune(*args, score_mode=oracle.SCORE_E, surp=_page_store(n, lambda b, i: 3.25))
+    assert np.allclose(rC["block_score"], rM["block_score"], rtol=1e-12, atol=1e-14)
+    r0 = oracle.score_prune(*args, score_mode=oracle.SCORE_E, surp=_page_store(n, lambda b, i: 0.0))
+    for b in range(w.B):
+        nb = -(-int(n["L"][b]) // w.P)
+        assert np.array_equal(r0["block_score"][b, :, :nb], np.ones((w.Hkv, nb)))
+
+
 def test_keep_set_rules():
     w, kv, n = _small_kv(B=3, lens=(200, 129, 48), seed=22)
     args = (n["q"], n["k"], n["bt"], n["L"], n["scale"])
