@@ -130,7 +130,7 @@ void eti_ctrl_defaults(eti_ctrl_params* p);
  *                (x / 4, b, lo32(offset), hi32(offset)), key (lo32(seed),
  *                hi32(seed)), word x mod 4, u = (2 (word & 0x7FFFFF) + 1) / 2^24;
  *                ties go to the lowest token id; -inf logits are never drawn
- *   tok_surprisal[b] = -log p(tok)
+ *   tok_surprisal[b] = -log p(tok)  (also written to surp_store, see above)
  * H, dH, T_out, theta_next, tok_surprisal: fp32 [B]; tok: int32 [B];
  * dH, theta_next, tok_surprisal may be NULL.  T_in, H_prev, H_target: fp32
  * [B].  T_out may alias T_in.
@@ -141,12 +141,28 @@ void eti_ctrl_defaults(eti_ctrl_params* p);
  */
 size_t eti_entropy_temp_sample_workspace_size(int B, int V);
 
+/*
+ * Where eti_entropy_temp_sample records each drawn token's surprisal for
+ * score mode E (the whole struct is nullable; it is a HOST pointer read
+ * before the call returns, the arrays are device memory):
+ *   store[slot_mapping[b]] = -log p(tok[b])
+ * for every sequence with no error bit and 0 <= slot_mapping[b] < num_slots
+ * (the slot of the position the new token takes in the caller's paged
+ * layout: page * P + offset; a negative slot skips the sequence).
+ */
+typedef struct {
+    float* store;                 /* fp32 [num_slots] */
+    const int64_t* slot_mapping;  /* int64 [B] */
+    int64_t num_slots;
+} eti_surp_store;
+
 int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
                             const float* T_in, const float* H_prev, float* tau,
                             const float* H_target, const eti_ctrl_params* params,
                             uint64_t seed, uint64_t offset,
                             int32_t* tok, float* H, float* T_out,
                             float* dH, float* theta_next, float* tok_surprisal,
+                            const eti_surp_store* surp_store,
                             uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream);
 
 /*
@@ -182,16 +198,33 @@ int eti_entropy_temp_sample_noalloc(const float* logits, int B, int V, int64_t l
                                     uint64_t seed, uint64_t offset,
                                     int32_t* tok, float* H, float* T_out,
                                     float* dH, float* theta_next, float* tok_surprisal,
+                                    const eti_surp_store* surp_store,
                                     uint32_t* err_flags, void* stream);
+
+/*
+ * Score modes: the reading of "the surprisal associated with the value
+ * vector" I(v_i) in the block score of Section 3.2.
+ *   ETI_SCORE_A  I(v_i) = -log a_i (attention as a distribution over the
+ *                values; the block scores add up to the attention entropy)
+ *   ETI_SCORE_E  I(v_i) = the stored surprisal -log p(x_i | x_<i) of the
+ *                token at position i, recorded when it was generated; the
+ *                store is fp32 [num_pages][P], paged like the keys (token i
+ *                of sequence b at tok_surp[block_table[b][i / P] * P + i % P])
+ *                and written by eti_entropy_temp_sample's surp_store output
+ *   ETI_SCORE_M  I(v_i) = 1 (the block's attention mass)
+ */
+#define ETI_SCORE_A 0
+#define ETI_SCORE_E 1
+#define ETI_SCORE_M 2
 
 /*
  * eti_score_prune_blocks -- the entropic keep set of half (b).
  *
  * For each sequence b, query head h and token i < ctx_lens[b]:
  *   x_i = scale * q[b,h,:] . k_i,   a_i = softmax_i(x_i) over all tokens,
- *   I_b^(h) = sum_{i in block} a_i (-log a_i)
- * (Section 3.2 with the surprisal of value i read as -log a_i, so that the
- * block scores add up to the attention entropy), normalised to
+ *   I_b^(h) = sum_{i in block} a_i I(v_i)
+ * (Section 3.2; I(v_i) by score_mode, see above; tok_surp is read only in
+ * mode E and must then be non-null), normalised to
  *   Ibar_b^(h) = n_b I_b^(h) / sum_b' I_b'^(h)   (1 when the sum is 0),
  * grouped per kv head as Ibar_b = max over the g query heads of the group.
  * Block b of (sequence, kv head) is kept iff Ibar_b >= theta[b_seq] (Section
@@ -214,7 +247,7 @@ int eti_score_prune_blocks(const eti_bf16* q, const eti_bf16* k_cache,
                            const int32_t* block_table, const int32_t* ctx_lens,
                            int B, int Hq, int Hkv, int D, int P, int max_blocks,
                            int64_t num_pages, float scale,
-                           const float* theta, int B_min,
+                           const float* theta, int B_min, int score_mode, const float* tok_surp,
                            uint8_t* keep_mask, int32_t* kept_idx, int32_t* kept_cnt,
                            float* block_score, float* token_scores, float* kept_norm,
                            uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream);
@@ -225,23 +258,28 @@ int eti_score_prune_blocks(const eti_bf16* q, const eti_bf16* k_cache,
  * workspace):
  *   eti_score_blocks  -- the scoring pass over every key page: token_scores
  *                        (nullable) and block_stats fp32 [B][Hkv][max_blocks][g][4]
- *                        = (m = max x, sum e^{x - m} - 1, sum e^{x - m}(x - m), 0)
- *                        per block and query head (the second entry excludes one
- *                        token at the max, which contributes exactly 1, so it
- *                        keeps full relative precision; garbage past n_b).
+ *                        = (m = max x, sum e^{x - m} - 1, sum e^{x - m}(x - m),
+ *                        sum e^{x - m} s_i) per block and query head (the second
+ *                        entry excludes one token at the max, which contributes
+ *                        exactly 1, so it keeps full relative precision; the
+ *                        fourth uses the stored surprisal s_i when tok_surp is
+ *                        non-null and is 0 otherwise; garbage past n_b).
  *   eti_prune_blocks  -- the keep set, budget, compaction and kept-token
- *                        normaliser from block_stats; writes err_flags.
+ *                        normaliser from block_stats in the given score_mode
+ *                        (mode E needs stats made with tok_surp); writes
+ *                        err_flags.
+ * An unknown score_mode returns ETI_ERR_UNSUPPORTED.
  */
 int eti_score_blocks(const eti_bf16* q, const eti_bf16* k_cache,
                      const int32_t* block_table, const int32_t* ctx_lens,
                      int B, int Hq, int Hkv, int D, int P, int max_blocks,
-                     int64_t num_pages, float scale,
+                     int64_t num_pages, float scale, const float* tok_surp,
                      float* token_scores, float* block_stats, void* stream);
 
 int eti_prune_blocks(const float* block_stats, const int32_t* block_table,
                      const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
                      int max_blocks, int64_t num_pages, const float* theta, int B_min,
-                     uint8_t* keep_mask, int32_t* kept_idx, int32_t* kept_cnt,
+                     int score_mode, uint8_t* keep_mask, int32_t* kept_idx, int32_t* kept_cnt,
                      float* block_score, float* kept_norm, uint32_t* err_flags, void* stream);
 
 /*

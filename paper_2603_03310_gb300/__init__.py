@@ -70,20 +70,20 @@ def load(path: str | None = None):
         lib.eti_entropy_temp_sample_workspace_size.argtypes = [i32, i32]
         lib.eti_entropy_temp_sample_workspace_size.restype = sz
         lib.eti_entropy_temp_sample.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64,
-                                                P, P, P, P, P, P, P, P, sz, P]
+                                                P, P, P, P, P, P, P, P, P, sz, P]
         lib.eti_entropy_temp_sample_noalloc.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64,
-                                                        P, P, P, P, P, P, P, P]
+                                                        P, P, P, P, P, P, P, P, P]
         lib.eti_entropy_temp_sample_noalloc.restype = i32
         lib.eti_entropy_temp_sample_noalloc_max_bytes.restype = sz
         lib.eti_entropy_temp_sample.restype = i32
         lib.eti_score_prune_workspace_size.argtypes = [i32] * 6
         lib.eti_score_prune_workspace_size.restype = sz
-        lib.eti_score_prune_blocks.argtypes = ([P, P, P, P] + [i32] * 6 + [i64, f32, P, i32]
+        lib.eti_score_prune_blocks.argtypes = ([P, P, P, P] + [i32] * 6 + [i64, f32, P, i32, i32, P]
                                                + [P] * 7 + [P, sz, P])
         lib.eti_score_prune_blocks.restype = i32
-        lib.eti_score_blocks.argtypes = [P, P, P, P] + [i32] * 6 + [i64, f32, P, P, P]
+        lib.eti_score_blocks.argtypes = [P, P, P, P] + [i32] * 6 + [i64, f32, P, P, P, P]
         lib.eti_score_blocks.restype = i32
-        lib.eti_prune_blocks.argtypes = [P, P, P] + [i32] * 6 + [i64, P, i32] + [P] * 7
+        lib.eti_prune_blocks.argtypes = [P, P, P] + [i32] * 6 + [i64, P, i32, i32] + [P] * 7
         lib.eti_prune_blocks.restype = i32
         lib.eti_paged_decode_workspace_size.argtypes = [i32] * 7
         lib.eti_paged_decode_workspace_size.restype = sz
@@ -137,10 +137,27 @@ def entropy_temp_sample_workspace_size(B: int, V: int) -> int:
     return int(load().eti_entropy_temp_sample_workspace_size(B, V))
 
 
+class SurpStore(ctypes.Structure):
+    """eti_surp_store (include/eti.h)."""
+    _fields_ = [("store", ctypes.c_void_p), ("slot_mapping", ctypes.c_void_p),
+                ("num_slots", ctypes.c_int64)]
+
+
+def _surp_store(surp_store, slot_mapping, B):
+    """(surp_store fp32 tensor, slot_mapping int64 [B]) -> SurpStore by reference, or None."""
+    if surp_store is None and slot_mapping is None:
+        return None
+    if surp_store is None or slot_mapping is None:
+        raise EtiError("surp_store and slot_mapping go together")
+    st = SurpStore(_dev(surp_store, "surp_store", torch.float32),
+                   _dev(slot_mapping, "slot_mapping", torch.int64, B), surp_store.numel())
+    return ctypes.byref(st)
+
+
 def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, err_flags, ws,
                             params: CtrlParams | None = None, seed: int = 0, offset: int = 0,
                             dH=None, theta_next=None, tok_surprisal=None, V: int | None = None,
-                            stream=None):
+                            surp_store=None, slot_mapping=None, stream=None):
     """Half (a) of the step; see include/eti.h.  logits fp32 [B, ld]."""
     B, ld = logits.shape
     V = ld if V is None else int(V)
@@ -154,7 +171,8 @@ def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, 
         ctypes.byref(params), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
         _dev(tok, "tok", i32, B), _dev(H, "H", f32, B), _dev(T_out, "T_out", f32, B),
         _dev(dH, "dH", f32, B), _dev(theta_next, "theta_next", f32, B),
-        _dev(tok_surprisal, "tok_surprisal", f32, B), _dev(err_flags, "err_flags", torch.int32, B),
+        _dev(tok_surprisal, "tok_surprisal", f32, B), _surp_store(surp_store, slot_mapping, B),
+        _dev(err_flags, "err_flags", torch.int32, B),
         _dev(ws, "ws", torch.uint8), ws.numel() if ws is not None else 0, _stream(stream))
     _check(st, "eti_entropy_temp_sample")
 
@@ -162,7 +180,8 @@ def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, 
 def eti_entropy_temp_sample_noalloc(logits, T_in, H_prev, tau, H_target, tok, H, T_out, err_flags,
                                     params: CtrlParams | None = None, seed: int = 0,
                                     offset: int = 0, dH=None, theta_next=None, tok_surprisal=None,
-                                    V: int | None = None, stream=None):
+                                    V: int | None = None, surp_store=None, slot_mapping=None,
+                                    stream=None):
     """eti_entropy_temp_sample without a workspace (fixed library scratch); see include/eti.h."""
     B, ld = logits.shape
     V = ld if V is None else int(V)
@@ -176,8 +195,8 @@ def eti_entropy_temp_sample_noalloc(logits, T_in, H_prev, tau, H_target, tok, H,
         ctypes.byref(params), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
         _dev(tok, "tok", i32, B), _dev(H, "H", f32, B), _dev(T_out, "T_out", f32, B),
         _dev(dH, "dH", f32, B), _dev(theta_next, "theta_next", f32, B),
-        _dev(tok_surprisal, "tok_surprisal", f32, B), _dev(err_flags, "err_flags", torch.int32, B),
-        _stream(stream))
+        _dev(tok_surprisal, "tok_surprisal", f32, B), _surp_store(surp_store, slot_mapping, B),
+        _dev(err_flags, "err_flags", torch.int32, B), _stream(stream))
     _check(st, "eti_entropy_temp_sample_noalloc")
 
 
@@ -202,8 +221,10 @@ def paged_decode_workspace_size(B, Hq, Hkv, D, P, max_blocks, have_scores: bool)
 def eti_score_prune_blocks(q, k_cache, block_table, ctx_lens, scale: float, theta, B_min: int,
                            keep_mask, kept_idx, kept_cnt, err_flags, ws,
                            block_score=None, token_scores=None, kept_norm=None,
-                           num_pages: int | None = None, stream=None):
-    """Entropic keep set of half (b); see include/eti.h."""
+                           num_pages: int | None = None, score_mode: int = 0, tok_surp=None,
+                           stream=None):
+    """Entropic keep set of half (b); see include/eti.h.  score_mode 0 (A), 1 (E,
+    with the token-surprisal store tok_surp fp32 [num_pages, P]) or 2 (M)."""
     B, Hq, Hkv, D, P, mb, npg = _attn_shapes(q, k_cache, block_table)
     num_pages = npg if num_pages is None else num_pages
     bf, i32, f32, u8 = torch.bfloat16, torch.int32, torch.float32, torch.uint8
@@ -211,7 +232,8 @@ def eti_score_prune_blocks(q, k_cache, block_table, ctx_lens, scale: float, thet
     st = load().eti_score_prune_blocks(
         _dev(q, "q", bf), _dev(k_cache, "k_cache", bf), _dev(block_table, "block_table", i32),
         _dev(ctx_lens, "ctx_lens", i32, B), B, Hq, Hkv, D, P, mb, int(num_pages), float(scale),
-        _dev(theta, "theta", f32, B), int(B_min),
+        _dev(theta, "theta", f32, B), int(B_min), int(score_mode),
+        _dev(tok_surp, "tok_surp", f32, npg * P),
         _dev(keep_mask, "keep_mask", u8, B * Hkv * mb), _dev(kept_idx, "kept_idx", i32, B * Hkv * mb),
         _dev(kept_cnt, "kept_cnt", i32, B * Hkv), _dev(block_score, "block_score", f32, B * Hkv * mb),
         _dev(token_scores, "token_scores", f32, B * Hkv * mb * P * g),
@@ -221,7 +243,7 @@ def eti_score_prune_blocks(q, k_cache, block_table, ctx_lens, scale: float, thet
 
 
 def eti_score_blocks(q, k_cache, block_table, ctx_lens, scale: float, block_stats,
-                     token_scores=None, num_pages: int | None = None, stream=None):
+                     token_scores=None, num_pages: int | None = None, tok_surp=None, stream=None):
     """The scoring pass alone (block stats and, optionally, token scores)."""
     B, Hq, Hkv, D, P, mb, npg = _attn_shapes(q, k_cache, block_table)
     num_pages = npg if num_pages is None else num_pages
@@ -230,6 +252,7 @@ def eti_score_blocks(q, k_cache, block_table, ctx_lens, scale: float, block_stat
         _dev(q, "q", torch.bfloat16), _dev(k_cache, "k_cache", torch.bfloat16),
         _dev(block_table, "block_table", torch.int32), _dev(ctx_lens, "ctx_lens", torch.int32, B),
         B, Hq, Hkv, D, P, mb, int(num_pages), float(scale),
+        _dev(tok_surp, "tok_surp", torch.float32, npg * P),
         _dev(token_scores, "token_scores", torch.float32, B * Hkv * mb * P * g),
         _dev(block_stats, "block_stats", torch.float32, B * Hq * mb * 4), _stream(stream))
     _check(st, "eti_score_blocks")
@@ -237,14 +260,15 @@ def eti_score_blocks(q, k_cache, block_table, ctx_lens, scale: float, block_stat
 
 def eti_prune_blocks(block_stats, block_table, ctx_lens, shape, theta, B_min: int, keep_mask,
                      kept_idx, kept_cnt, err_flags, block_score=None, kept_norm=None,
-                     num_pages: int = 0, stream=None):
+                     num_pages: int = 0, score_mode: int = 0, stream=None):
     """The keep set from block stats; shape = (B, Hq, Hkv, D, P, max_blocks)."""
     B, Hq, Hkv, D, P, mb = shape
     i32, f32, u8 = torch.int32, torch.float32, torch.uint8
     st = load().eti_prune_blocks(
         _dev(block_stats, "block_stats", f32, B * Hq * mb * 4), _dev(block_table, "block_table", i32),
         _dev(ctx_lens, "ctx_lens", i32, B), B, Hq, Hkv, D, P, mb, int(num_pages),
-        _dev(theta, "theta", f32, B), int(B_min), _dev(keep_mask, "keep_mask", u8, B * Hkv * mb),
+        _dev(theta, "theta", f32, B), int(B_min), int(score_mode),
+        _dev(keep_mask, "keep_mask", u8, B * Hkv * mb),
         _dev(kept_idx, "kept_idx", i32, B * Hkv * mb), _dev(kept_cnt, "kept_cnt", i32, B * Hkv),
         _dev(block_score, "block_score", f32, B * Hkv * mb), _dev(kept_norm, "kept_norm", f32, B * Hq * 2),
         _dev(err_flags, "err_flags", i32, B), _stream(stream))

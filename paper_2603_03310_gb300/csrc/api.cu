@@ -11,15 +11,17 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
                                    const float* H_target, const eti_ctrl_params* p,
                                    uint64_t seed, uint64_t offset, int32_t* tok, float* H,
                                    float* T_out, float* dH, float* theta_next, float* surprisal,
-                                   uint32_t* err, void* part, cudaStream_t stream);
+                                   const eti_surp_store* store, uint32_t* err, void* part,
+                                   cudaStream_t stream);
 size_t eti_entropy_partial_bytes(int B);
 int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const int32_t* block_table,
                             const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
-                            int max_blocks, long long num_pages, float scale, float* token_scores,
-                            float4* stats, cudaStream_t stream);
+                            int max_blocks, long long num_pages, float scale, const float* tok_surp,
+                            float* token_scores, float4* stats, cudaStream_t stream);
 int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, const int32_t* block_table,
                               long long num_pages, int B, int Hq, int Hkv, int P, int max_blocks,
-                              const float* theta, int B_min, int given, const uint8_t* given_mask,
+                              const float* theta, int B_min, int score_mode, int given,
+                              const uint8_t* given_mask,
                               const int32_t* given_idx, const int32_t* given_cnt, uint8_t* keep_mask,
                               int32_t* kept_idx, int32_t* kept_cnt, float* block_score,
                               float* kept_norm, uint32_t* err, cudaStream_t stream);
@@ -160,16 +162,18 @@ int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
                             uint64_t seed, uint64_t offset,
                             int32_t* tok, float* H, float* T_out,
                             float* dH, float* theta_next, float* tok_surprisal,
+                            const eti_surp_store* surp_store,
                             uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream) {
     if (B < 0 || B > 65535 || V < 1 || ld < V) return ETI_ERR_SHAPE;
     if (B == 0) return ETI_OK;
     if (!logits || !T_in || !H_prev || !tau || !H_target || !params || !tok || !H || !T_out ||
         !err_flags)
         return ETI_ERR_NULL;
+    if (surp_store && (!surp_store->store || !surp_store->slot_mapping)) return ETI_ERR_NULL;
     if (!ws || ws_bytes < eti_entropy_temp_sample_workspace_size(B, V)) return ETI_ERR_WORKSPACE;
     return eti_launch_entropy_temp_sample(logits, B, V, (long long)ld, T_in, H_prev, tau, H_target,
                                           params, seed, offset, tok, H, T_out, dH, theta_next,
-                                          tok_surprisal, err_flags, ws, (cudaStream_t)stream);
+                                          tok_surprisal, surp_store, err_flags, ws, (cudaStream_t)stream);
 }
 
 size_t eti_score_prune_workspace_size(int B, int Hq, int Hkv, int D, int P, int max_blocks) {
@@ -183,13 +187,15 @@ int eti_score_prune_blocks(const eti_bf16* q, const eti_bf16* k_cache,
                            const int32_t* block_table, const int32_t* ctx_lens,
                            int B, int Hq, int Hkv, int D, int P, int max_blocks,
                            int64_t num_pages, float scale,
-                           const float* theta, int B_min,
+                           const float* theta, int B_min, int score_mode, const float* tok_surp,
                            uint8_t* keep_mask, int32_t* kept_idx, int32_t* kept_cnt,
                            float* block_score, float* token_scores, float* kept_norm,
                            uint32_t* err_flags, void* ws, size_t ws_bytes, void* stream) {
     int st = check_attn_shape(B, Hq, Hkv, D, P, max_blocks, num_pages);
     if (st != ETI_OK) return st;
+    if (score_mode < ETI_SCORE_A || score_mode > ETI_SCORE_M) return ETI_ERR_UNSUPPORTED;
     if (B == 0) return ETI_OK;
+    if (score_mode == ETI_SCORE_E && !tok_surp) return ETI_ERR_NULL;
     if (!q || !k_cache || !block_table || !ctx_lens || !theta || !keep_mask || !kept_idx ||
         !kept_cnt || !err_flags)
         return ETI_ERR_NULL;
@@ -200,35 +206,37 @@ int eti_score_prune_blocks(const eti_bf16* q, const eti_bf16* k_cache,
     cudaStream_t s = (cudaStream_t)stream;
     float4* stats = static_cast<float4*>(ws);
     st = eti_launch_score_blocks(q, k_cache, block_table, ctx_lens, B, Hq, Hkv, D, P, max_blocks,
-                                 (long long)num_pages, scale, token_scores, stats, s);
+                                 (long long)num_pages, scale,
+                                 score_mode == ETI_SCORE_E ? tok_surp : nullptr, token_scores, stats, s);
     if (st != ETI_OK) return st;
     return eti_launch_prune_finalize(stats, ctx_lens, block_table, (long long)num_pages, B, Hq, Hkv,
-                                     P, max_blocks, theta, B_min, 0, nullptr, nullptr, nullptr,
+                                     P, max_blocks, theta, B_min, score_mode, 0, nullptr, nullptr, nullptr,
                                      keep_mask, kept_idx, kept_cnt, block_score, kept_norm,
                                      err_flags, s);
 }
 
 int eti_score_blocks(const eti_bf16* q, const eti_bf16* k_cache, const int32_t* block_table,
                      const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
-                     int max_blocks, int64_t num_pages, float scale, float* token_scores,
-                     float* block_stats, void* stream) {
+                     int max_blocks, int64_t num_pages, float scale, const float* tok_surp,
+                     float* token_scores, float* block_stats, void* stream) {
     int st = check_attn_shape(B, Hq, Hkv, D, P, max_blocks, num_pages);
     if (st != ETI_OK) return st;
     if (B == 0) return ETI_OK;
     if (!q || !k_cache || !block_table || !ctx_lens || !block_stats) return ETI_ERR_NULL;
     if (!aligned16(q) || !aligned16(k_cache) || !aligned16(block_stats)) return ETI_ERR_ALIGN;
     return eti_launch_score_blocks(q, k_cache, block_table, ctx_lens, B, Hq, Hkv, D, P, max_blocks,
-                                   (long long)num_pages, scale, token_scores,
+                                   (long long)num_pages, scale, tok_surp, token_scores,
                                    reinterpret_cast<float4*>(block_stats), (cudaStream_t)stream);
 }
 
 int eti_prune_blocks(const float* block_stats, const int32_t* block_table, const int32_t* ctx_lens,
                      int B, int Hq, int Hkv, int D, int P, int max_blocks, int64_t num_pages,
-                     const float* theta, int B_min, uint8_t* keep_mask, int32_t* kept_idx,
-                     int32_t* kept_cnt, float* block_score, float* kept_norm, uint32_t* err_flags,
-                     void* stream) {
+                     const float* theta, int B_min, int score_mode, uint8_t* keep_mask,
+                     int32_t* kept_idx, int32_t* kept_cnt, float* block_score, float* kept_norm,
+                     uint32_t* err_flags, void* stream) {
     int st = check_attn_shape(B, Hq, Hkv, D, P, max_blocks, num_pages);
     if (st != ETI_OK) return st;
+    if (score_mode < ETI_SCORE_A || score_mode > ETI_SCORE_M) return ETI_ERR_UNSUPPORTED;
     if (B == 0) return ETI_OK;
     if (!block_stats || !block_table || !ctx_lens || !theta || !keep_mask || !kept_idx ||
         !kept_cnt || !err_flags)
@@ -236,7 +244,7 @@ int eti_prune_blocks(const float* block_stats, const int32_t* block_table, const
     if (!aligned16(block_stats)) return ETI_ERR_ALIGN;
     return eti_launch_prune_finalize(reinterpret_cast<const float4*>(block_stats), ctx_lens,
                                      block_table, (long long)num_pages, B, Hq, Hkv, P, max_blocks,
-                                     theta, B_min, 0, nullptr, nullptr, nullptr, keep_mask, kept_idx,
+                                     theta, B_min, score_mode, 0, nullptr, nullptr, nullptr, keep_mask, kept_idx,
                                      kept_cnt, block_score, kept_norm, err_flags,
                                      (cudaStream_t)stream);
 }
@@ -275,10 +283,11 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
     cudaStream_t s = (cudaStream_t)stream;
     if (!have_scores) {
         st = eti_launch_score_blocks(q, k_cache, block_table, ctx_lens, B, Hq, Hkv, D, P,
-                                     max_blocks, (long long)num_pages, scale, w.scores, w.stats, s);
+                                     max_blocks, (long long)num_pages, scale, nullptr, w.scores,
+                                     w.stats, s);
         if (st != ETI_OK) return st;
         st = eti_launch_prune_finalize(w.stats, ctx_lens, block_table, (long long)num_pages, B, Hq,
-                                       Hkv, P, max_blocks, nullptr, 0, 1, keep_mask,
+                                       Hkv, P, max_blocks, nullptr, 0, ETI_SCORE_A, 1, keep_mask,
                                        have_lists ? kept_idx : nullptr,
                                        have_lists ? kept_cnt : nullptr, nullptr, w.kidx, w.kcnt,
                                        nullptr, w.knorm, nullptr, s);

@@ -162,6 +162,9 @@ struct EtsArgs {
     float* dH;
     float* theta_next;
     float* surprisal;
+    float* surp_store;             // token-surprisal store (score mode E), or null
+    const int64_t* slot_mapping;   // [B] slot of the drawn token in surp_store
+    long long num_slots;
     uint32_t* err;
     int ngroups;          // 4-token groups per row
     long long share;      // groups per CTA of the persistent grid
@@ -367,9 +370,14 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
                                        : a.p.theta_hi;
             a.theta_next[b] = fminf(a.p.theta_user, tmax);
         }
-        if (a.surprisal) {
+        if (a.surprisal || a.surp_store) {
             const float tt = fmaf(row[t.bi], c, -t.mc);
-            a.surprisal[b] = kLn2 * (l2S - tt);
+            const float sp = kLn2 * (l2S - tt);
+            if (a.surprisal) a.surprisal[b] = sp;
+            if (a.surp_store) {
+                const long long slot = a.slot_mapping[b];
+                if (slot >= 0 && slot < a.num_slots) a.surp_store[slot] = sp;
+            }
         }
     }
     a.err[b] = err;
@@ -396,7 +404,8 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
                                    const float* H_target, const eti_ctrl_params* p,
                                    uint64_t seed, uint64_t offset, int32_t* tok, float* H,
                                    float* T_out, float* dH, float* theta_next, float* surprisal,
-                                   uint32_t* err, void* part, cudaStream_t stream) {
+                                   const eti_surp_store* store, uint32_t* err, void* part,
+                                   cudaStream_t stream) {
     using namespace eti;
     if (B == 0) return ETI_OK;
     const int ncta = eti_entropy_ncta();
@@ -411,6 +420,9 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
     a.off_lo = (uint32_t)offset; a.off_hi = (uint32_t)(offset >> 32);
     a.tok = tok; a.H = H; a.T_out = T_out; a.dH = dH; a.theta_next = theta_next;
     a.surprisal = surprisal; a.err = err;
+    a.surp_store = store ? store->store : nullptr;
+    a.slot_mapping = store ? store->slot_mapping : nullptr;
+    a.num_slots = store ? (long long)store->num_slots : 0;
     a.ngroups = (V + 3) / 4;
     const long long total = (long long)B * a.ngroups;
     a.share = (total + ncta - 1) / ncta;
@@ -464,17 +476,20 @@ extern "C" int eti_entropy_temp_sample_noalloc(const float* logits, int B, int V
                                                uint64_t seed, uint64_t offset,
                                                int32_t* tok, float* H, float* T_out,
                                                float* dH, float* theta_next, float* tok_surprisal,
+                                               const eti_surp_store* surp_store,
                                                uint32_t* err_flags, void* stream) {
     if (B < 0 || B > 65535 || V < 1 || ld < V) return ETI_ERR_SHAPE;
     if (B == 0) return ETI_OK;
     if (!logits || !T_in || !H_prev || !tau || !H_target || !params || !tok || !H || !T_out ||
         !err_flags)
         return ETI_ERR_NULL;
+    if (surp_store && (!surp_store->store || !surp_store->slot_mapping)) return ETI_ERR_NULL;
     if (eti_entropy_partial_bytes(B) > kNoAllocScratchBytes) return ETI_ERR_TOO_LARGE;
     void* scratch = nullptr;
     const int st = ets_scratch_address(&scratch);
     if (st != ETI_OK) return st;
     return eti_launch_entropy_temp_sample(logits, B, V, (long long)ld, T_in, H_prev, tau, H_target,
                                           params, seed, offset, tok, H, T_out, dH, theta_next,
-                                          tok_surprisal, err_flags, scratch, (cudaStream_t)stream);
+                                          tok_surprisal, surp_store, err_flags, scratch,
+                                          (cudaStream_t)stream);
 }

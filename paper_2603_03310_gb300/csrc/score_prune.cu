@@ -38,7 +38,9 @@ struct ScoreArgs {
     long long num_pages;
     float scale;
     float* token_scores;   // [B][Hkv][max_blocks][P][g] or null
-    float4* stats;         // [B][Hkv][max_blocks][g]: (m, l, u, 0)
+    float4* stats;         // [B][Hkv][max_blocks][g]: (m, l - 1, u, e) with
+                           // e = sum e^{x-m} s_i when tok_surp is given, else 0
+    const float* tok_surp; // [num_pages][P] stored token surprisal s_i, or null
 };
 
 // Exclusive prefix over sequences of (blocks * Hkv) into shared memory;
@@ -174,6 +176,7 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
     uint4 qf[H][2];
     int q_b = -1, q_kvh = -1;
     float xs[kTiles][4];
+    float ss[kTiles][2];          // stored surprisal of token slots grp, grp + 8
     int i = 0;
     bool timed_out = false;
 #pragma unroll 1
@@ -237,6 +240,15 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
             if (tt == tile)
 #pragma unroll
                 for (int ee = 0; ee < 4; ++ee) xs[tt][ee] = x4[ee];
+        if (a.tok_surp) {
+            // score mode E: the surprisal of each token, paged like the keys
+            const float* sp = a.tok_surp + (long long)e.w * P + tile * 16 + grp;
+            const float s0 = (ok && grp < valid_tok) ? __ldg(sp) : 0.f;
+            const float s1 = (ok && grp + 8 < valid_tok) ? __ldg(sp + 8) : 0.f;
+#pragma unroll
+            for (int tt = 0; tt < kTiles; ++tt)
+                if (tt == tile) { ss[tt][0] = s0; ss[tt][1] = s1; }
+        }
         const long long unit = ((long long)b * a.Hkv + kvh) * a.max_blocks + blk;
         if (a.token_scores) {
             float* ts = a.token_scores + (unit * P + tile * 16) * a.g;
@@ -268,7 +280,7 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
                 // l1 = (sum e^{x-m}) - 1, kept exact: the tokens below the max are
                 // summed and every further token AT the max adds exactly 1, so a
                 // block dominated by one token keeps its small remainder.
-                float l1 = 0.f, u = 0.f, neq = 0.f;
+                float l1 = 0.f, u = 0.f, neq = 0.f, es = 0.f;
                 if (m != -kInf) {
 #pragma unroll
                     for (int tt = 0; tt < kTiles; ++tt) {
@@ -279,6 +291,7 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
                             l1 += d < 0.f ? w : 0.f;
                             neq += d == 0.f ? 1.f : 0.f;
                             u = fmaf(w, fmaxf(d, -1e30f), u);
+                            if (a.tok_surp) es = fmaf(w, ss[tt][ee], es);
                         }
                     }
                 }
@@ -287,10 +300,11 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
                     l1 += __shfl_xor_sync(0xffffffffu, l1, o);
                     u += __shfl_xor_sync(0xffffffffu, u, o);
                     neq += __shfl_xor_sync(0xffffffffu, neq, o);
+                    if (a.tok_surp) es += __shfl_xor_sync(0xffffffffu, es, o);
                 }
                 l1 += neq - 1.f;
                 const int h = 2 * tq + j;
-                if (grp == 0 && h < a.g) a.stats[unit * a.g + h] = make_float4(m, l1, u, 0.f);
+                if (grp == 0 && h < a.g) a.stats[unit * a.g + h] = make_float4(m, l1, u, es);
             }
         }
     }
@@ -321,6 +335,7 @@ struct FinArgs {
     // rule mode (given == 0)
     const float* theta;
     int B_min;
+    int score_mode;         // 0 A: I_i = -log a_i; 1 E: stored surprisal; 2 M: 1
     // given mode: keep set from a list or a mask (or every block)
     int given;
     const uint8_t* given_mask;
@@ -444,7 +459,7 @@ prune_finalize_kernel(const FinArgs a) {
             if (kCache) {
                 sh_m[h * a.max_blocks + j] = s.x;
                 sh_l[h * a.max_blocks + j] = s.y;
-                sh_u[h * a.max_blocks + j] = s.z;
+                sh_u[h * a.max_blocks + j] = a.score_mode == 1 ? s.w : s.z;
             }
             M[h] = fmaxf(M[h], s.x);
         }
@@ -463,7 +478,9 @@ prune_finalize_kernel(const FinArgs a) {
     auto stat = [&](int j, int h) -> float4 {
         if (kCache) return make_float4(sh_m[h * a.max_blocks + j], sh_l[h * a.max_blocks + j],
                                        sh_u[h * a.max_blocks + j], 0.f);
-        return st[j * G + h];
+        float4 v = st[j * G + h];
+        if (a.score_mode == 1) v.z = v.w;   // .z: u (mode A) or sum e^{x-m} s_i (mode E)
+        return v;
     };
 
     if (!a.given) {
@@ -495,7 +512,10 @@ prune_finalize_kernel(const FinArgs a) {
                 Hs[h] = 0.f;
             }
             // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
+            // mode E: I_b = e^{m_b - M} sum e^{x-m_b} s_i / Z; mode M: the block's mass
             auto Ib = [&](float4 s, int h) {
+                if (a.score_mode == 1) return expf(s.x - M[h]) * s.z / Z[h];
+                if (a.score_mode == 2) return expf(s.x - M[h]) * (1.f + s.y) / Z[h];
                 return expf(s.x - M[h]) * ((1.f + s.y) * (lZ[h] + M[h] - s.x) - s.z) / Z[h];
             };
             for (int j = k0; j < k1; ++j)
@@ -785,7 +805,7 @@ prune_finalize_flat_kernel(const FinArgs a) {
         m[k] = -kInf; l1[k] = 0.f; w[k] = 0.f;
         if (h < G && j < nb) {
             const float4 s = st[(long long)j * G + h];
-            m[k] = s.x; l1[k] = s.y; w[k] = s.z;
+            m[k] = s.x; l1[k] = s.y; w[k] = a.score_mode == 1 ? s.w : s.z;
             stale |= (s.x != s.x);              // NaN max: the scoring pass gave up on this block
             Mh[0] = fmaxf(Mh[0], s.x);
         }
@@ -834,7 +854,9 @@ prune_finalize_flat_kernel(const FinArgs a) {
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k)
             if (valid[k]) {
-                w[k] = c[k] * ((1.f + l1[k]) * (lZ + M - m[k]) - w[k]) / Z;
+                if (a.score_mode == 1) w[k] = c[k] * w[k] / Z;                 // E
+                else if (a.score_mode == 2) w[k] = c[k] * (1.f + l1[k]) / Z;   // M
+                else w[k] = c[k] * ((1.f + l1[k]) * (lZ + M - m[k]) - w[k]) / Z;
                 Hs[0] += w[k];
                 l1[k] = (1.f + l1[k]) * c[k];
             }
@@ -989,8 +1011,8 @@ using namespace eti;
 
 int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const int32_t* block_table,
                             const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
-                            int max_blocks, long long num_pages, float scale, float* token_scores,
-                            float4* stats, cudaStream_t stream) {
+                            int max_blocks, long long num_pages, float scale, const float* tok_surp,
+                            float* token_scores, float4* stats, cudaStream_t stream) {
     if (B == 0) return ETI_OK;
     if (num_pages <= 0) {
         // no page can be valid: every sequence with blocks is reported by the
@@ -1001,6 +1023,7 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
     a.q = q; a.k_cache = k_cache; a.block_table = block_table; a.ctx_lens = ctx_lens;
     a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.g = Hq / Hkv; a.max_blocks = max_blocks;
     a.num_pages = num_pages; a.scale = scale; a.token_scores = token_scores; a.stats = stats;
+    a.tok_surp = tok_surp;
     // tile row coordinates are int32 on the device
     if (num_pages * Hkv * P >= (1LL << 31)) return ETI_ERR_UNSUPPORTED;
     CUtensorMap kmap;
@@ -1029,7 +1052,8 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
 
 int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, const int32_t* block_table,
                               long long num_pages, int B, int Hq, int Hkv, int P, int max_blocks,
-                              const float* theta, int B_min, int given, const uint8_t* given_mask,
+                              const float* theta, int B_min, int score_mode, int given,
+                              const uint8_t* given_mask,
                               const int32_t* given_idx, const int32_t* given_cnt, uint8_t* keep_mask,
                               int32_t* kept_idx, int32_t* kept_cnt, float* block_score,
                               float* kept_norm, uint32_t* err, cudaStream_t stream) {
@@ -1037,7 +1061,7 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     FinArgs a;
     a.stats = stats; a.ctx_lens = ctx_lens; a.block_table = block_table; a.num_pages = num_pages;
     a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.g = Hq / Hkv; a.P = P; a.max_blocks = max_blocks;
-    a.theta = theta; a.B_min = B_min; a.given = given; a.given_mask = given_mask;
+    a.theta = theta; a.B_min = B_min; a.score_mode = score_mode; a.given = given; a.given_mask = given_mask;
     a.given_idx = given_idx; a.given_cnt = given_cnt; a.keep_mask = keep_mask;
     a.kept_idx = kept_idx; a.kept_cnt = kept_cnt; a.block_score = block_score;
     a.kept_norm = kept_norm; a.err = err;

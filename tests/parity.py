@@ -111,10 +111,11 @@ def host_kv(kv: dict) -> dict:
 def host_from_gather(sub: dict) -> dict:
     """workloads.gather_sequences output in the host_kv layout."""
     return dict(q=sub["q"], k=sub["k_cache"], v=sub["v_cache"], bt=sub["block_table"],
-                L=sub["ctx_lens"], scale=sub["scale"], num_pages=sub["num_pages"])
+                L=sub["ctx_lens"], scale=sub["scale"], num_pages=sub["num_pages"],
+                pages=sub["pages"])
 
 
-def score_bands(ref: dict, n: dict) -> np.ndarray:
+def score_bands(ref: dict, n: dict, score_mode: int = 0) -> np.ndarray:
     """Per (sequence, kv head, block) bound on |Ibar_gpu - Ibar_exact| from fp32 scores.
 
     The kernel forms x_i = s q.k_i as an fp32 dot product of D bf16 products,
@@ -123,7 +124,9 @@ def score_bands(ref: dict, n: dict) -> np.ndarray:
     Then |da_i / a_i| <= 2 |dx| and, from I_b = sum a_i (-log a_i) and
     H = sum_b I_b,  |dIbar_b| / Ibar_b <= 2 |dx| ((I_b + A_b) / I_b + (H + 1) / H),
     A_b the block's attention mass: the bound is large exactly where one token
-    takes nearly all of a block's attention (I_b << A_b).
+    takes nearly all of a block's attention (I_b << A_b).  In modes E and M the
+    per-token weight does not depend on a_i (s_i >= 0 or 1), so the numerator
+    and the normaliser each move by at most 2 |dx| relative: 4 |dx| in all.
     """
     q = (n["q"].astype(np.uint32) << 16).view(np.float32)           # [B, Hq, D]
     k = (n["k"].astype(np.uint32) << 16).view(np.float32)           # [pages, Hkv, P, D]
@@ -154,7 +157,10 @@ def score_bands(ref: dict, n: dict) -> np.ndarray:
                 H = ref["head_H"][b, h]
                 if H <= 0:
                     continue
-                kappa = (I + A) / np.maximum(I, 1e-300) + (H + 1.0) / H
+                if score_mode == 0:
+                    kappa = (I + A) / np.maximum(I, 1e-300) + (H + 1.0) / H
+                else:
+                    kappa = 2.0
                 nrm = nb * I / H
                 band[b, kvh, :nb] = np.maximum(band[b, kvh, :nb], 2.0 * dx * kappa * nrm)
     return band

@@ -67,18 +67,24 @@ def test_entropy_call_validation(lib):
     f = lib.eti_entropy_temp_sample
     ws = lib.eti_entropy_temp_sample_workspace_size(4, 10)
     assert ws > 0
+    # tok, H, T_out, dH, theta_next, tok_surprisal, surp_store (a host struct), err_flags
+    OUTS = [fake] * 6 + [NULL, fake]
     # bad shapes
-    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -2
-    assert f(fake, 4, 0, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -2
-    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -2
+    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -2
+    assert f(fake, 4, 0, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -2
+    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -2
     # B == 0 is a no-op
-    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, *[NULL] * 7, NULL, 0, NULL) == 0
+    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, *[NULL] * 8, NULL, 0, NULL) == 0
     # required pointers
-    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws, NULL) == -1
-    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, *[fake] * 7, fake, ws, NULL) == -1
+    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -1
+    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, *OUTS, fake, ws, NULL) == -1
+    # a surprisal store needs both of its arrays
+    half = eti.SurpStore(fake, None, 16)
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 6, ctypes.byref(half),
+             fake, fake, ws, NULL) == -1
     # workspace
-    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, NULL, ws, NULL) == -4
-    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 7, fake, ws - 1, NULL) == -4
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL, ws, NULL) == -4
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws - 1, NULL) == -4
 
 
 def test_attention_call_validation(lib):
@@ -90,10 +96,14 @@ def test_attention_call_validation(lib):
     assert need >= 4 * 32 * 512 * 16
     base = dict(B=4, Hq=32, Hkv=8, D=128, P=16, mb=512)
 
-    def call(q=a16, k=a16, B=4, Hq=32, Hkv=8, D=128, Pg=16, mb=512, ws=a16, wsb=None):
+    def call(q=a16, k=a16, B=4, Hq=32, Hkv=8, D=128, Pg=16, mb=512, ws=a16, wsb=None, mode=0,
+             surp=NULL):
         wsb = need if wsb is None else wsb
-        return f(q, k, a16, a16, B, Hq, Hkv, D, Pg, mb, 1000, 0.1, a16, 1,
+        return f(q, k, a16, a16, B, Hq, Hkv, D, Pg, mb, 1000, 0.1, a16, 1, mode, surp,
                  a16, a16, a16, NULL, NULL, NULL, a16, ws, wsb, NULL)
+    assert call(mode=3) == -3                # unknown score mode
+    assert call(mode=-1) == -3
+    assert call(mode=1) == -1                # mode E needs the surprisal store
     assert call(Hq=30) == -2                 # Hq % Hkv
     assert call(Hq=72, Hkv=8) == -3          # g > 8
     assert call(D=96) == -3

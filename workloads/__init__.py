@@ -210,4 +210,4 @@ def gather_sequences(kv: dict, seqs) -> dict:
     vc = kv["v_cache"].index_select(0, idx) if used else kv["v_cache"][:0]
     return dict(q=bf16_bits(kv["q"][seqs]), k_cache=bf16_bits(kc), v_cache=bf16_bits(vc),
                 block_table=new_bt.astype(np.int32), ctx_lens=L.astype(np.int32),
-                num_pages=len(used), scale=kv["scale"])
+                num_pages=len(used), scale=kv["scale"], pages=np.asarray(used, np.int64))
