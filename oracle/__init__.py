@@ -74,6 +74,7 @@ def _load():
             lib.oracle_entropy_row.restype = f64
             lib.oracle_entropy_temp_sample.argtypes = (
                 [P, i32, i64, i64, P, P, P, P, P, u64, u64] + [P] * 9)
+            lib.oracle_topk_entropy.argtypes = [P, i32, i64, i64, P, i64, P, P, P, P]
             lib.oracle_score_prune.argtypes = (
                 [P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, i32, i32, P] + [P] * 8)
             lib.oracle_paged_attention.argtypes = (
@@ -132,6 +133,24 @@ def sample_key(logits_row, T: float, seed: int, offset: int, row: int, x: int) -
 def entropy_row(z, T: float = 1.0) -> float:
     z = _c(z, np.float32)
     return float(_load().oracle_entropy_row(_ptr(z), z.shape[0], float(T)))
+
+
+def topk_entropy(logits, T_in, k: int, V: int | None = None) -> dict:
+    """Top-k entropy H~, tail-corrected H^ and the tail mass of every row.
+
+    logits float32 [B, ld] (the first V columns are the vocabulary); T_in [B].
+    """
+    lib = _load()
+    z = _c(logits, np.float32)
+    B, ld = z.shape
+    V = ld if V is None else int(V)
+    T_in = _c(T_in, np.float32)
+    out = {n: np.empty(B, np.float64) for n in ("H_tilde", "H_hat", "tail_mass")}
+    err = np.empty(B, np.uint32)
+    lib.oracle_topk_entropy(_ptr(z), B, V, ld, _ptr(T_in), int(k), _ptr(out["H_tilde"]),
+                            _ptr(out["H_hat"]), _ptr(out["tail_mass"]), _ptr(err))
+    out["err"] = err
+    return out
 
 
 def entropy_temp_sample(logits, T_in, H_prev, tau_in, H_target, ctrl_params=None,

@@ -236,6 +236,71 @@ double oracle_entropy_row(const float *z, int64_t V, double T) {
 }
 
 /* ------------------------------------------------------------------------ */
+/* Top-k entropy estimators (Section 2.1, "Top-k entropy approximation" and
+ * "Tail-corrected estimator").
+ *
+ * With y = z / T_t, p = softmax(y) and K the first k_eff = min(k, V) tokens
+ * ordered by (y descending, token id ascending):
+ *   p~(x)   = p(x) / sum_{y in K} p(y) on K            (truncated distribution)
+ *   H~      = -sum_{x in K} p~(x) log p~(x)            (0 log 0 := 0)
+ *   m       = sum_{x in K} p(x),   m_bar = 1 - m = sum_{x not in K} p(x)
+ *   H^      = H~ + h(m_bar) + m_bar log(V - k_eff)     (h: binary entropy;
+ *                                                       the last term is 0 when k_eff = V)
+ * tail_mass = m_bar, summed over the tail itself so that a small tail keeps
+ * its relative precision.  Rows with a NaN or +inf logit, with every logit
+ * -inf, or with a temperature that is not a positive finite number set their
+ * error bit and return NaN. */
+typedef struct { double y; int64_t idx; } topk_item;
+
+static int topk_cmp(const void *pa, const void *pb) {
+    const topk_item *a = (const topk_item *)pa, *b = (const topk_item *)pb;
+    if (a->y > b->y) return -1;
+    if (a->y < b->y) return 1;
+    return (a->idx > b->idx) - (a->idx < b->idx);
+}
+
+void oracle_topk_entropy(const float *logits, int B, int64_t V, int64_t ld, const float *T_in,
+                         int64_t k, double *H_tilde, double *H_hat, double *tail_mass,
+                         uint32_t *err) {
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int b = 0; b < B; ++b) {
+        const float *z = logits + (int64_t)b * ld;
+        const double T = (double)T_in[b];
+        uint32_t e = (T > 0.0 && !isinf(T)) ? 0u : ORC_ERR_BAD_TEMP;
+        double M = -INFINITY;
+        for (int64_t x = 0; x < V && !e; ++x) {
+            double zx = (double)z[x];
+            if (isnan(zx) || (isinf(zx) && zx > 0)) e |= ORC_ERR_NONFINITE;
+            else if (zx / T > M) M = zx / T;
+        }
+        if (!e && isinf(M)) e |= ORC_ERR_ALL_NEG_INF;
+        err[b] = e;
+        if (e) { H_tilde[b] = NAN; H_hat[b] = NAN; tail_mass[b] = NAN; continue; }
+        topk_item *it = (topk_item *)malloc(sizeof(topk_item) * (size_t)V);
+        for (int64_t x = 0; x < V; ++x) { it[x].y = (double)z[x] / T; it[x].idx = x; }
+        qsort(it, (size_t)V, sizeof(topk_item), topk_cmp);
+        const int64_t ke = k < V ? k : V;
+        double ZK = 0.0, Zt = 0.0;
+        for (int64_t r = 0; r < V; ++r) {
+            double w = exp(it[r].y - M);
+            if (r < ke) ZK += w; else Zt += w;
+        }
+        double h = 0.0;
+        for (int64_t r = 0; r < ke; ++r) {
+            double pt = exp(it[r].y - M) / ZK;
+            if (pt > 0.0) h -= pt * log(pt);
+        }
+        const double mb = Zt / (ZK + Zt);
+        double hb = 0.0;
+        if (mb > 0.0 && mb < 1.0) hb = -mb * log(mb) - (1.0 - mb) * log1p(-mb);
+        H_tilde[b] = h;
+        tail_mass[b] = mb;
+        H_hat[b] = h + hb + (ke < V ? mb * log((double)(V - ke)) : 0.0);
+        free(it);
+    }
+}
+
+/* ------------------------------------------------------------------------ */
 /* Paged KV cache helpers.  k_cache / v_cache are bf16 bit patterns laid out
  * [num_pages][Hkv][P][D]; block_table is [B][max_blocks]. */
 

@@ -602,3 +602,80 @@ def test_empty_sequences_and_bad_inputs():
     L[1] = w.max_blocks * w.P + 1
     _, err = oracle.paged_attention(n["q"], n["k"], n["v"], bt, L, n["scale"])
     assert err[1] == oracle.ERR_BAD_CTX
+
+
+# ---------------------------------------------------------------------------
+# top-k entropy estimators (Section 2.1)
+
+def test_topk_entropy_grouping_identity_and_upper_bound():
+    """H = h(m_bar) + m H~ + m_bar H_tail exactly (grouping of the entropy over
+    K and its complement), H <= H^ (the tail is at most uniform over V - k
+    tokens), and H~, m_bar, H^ as defined -- p from scipy's softmax."""
+    rng = np.random.default_rng(0)
+    B, V = 6, 300
+    z = (rng.standard_normal((B, V)) * rng.uniform(0.3, 4, (B, 1))).astype(np.float32)
+    z[0, 10:20] = z[0, 9]                      # ties straddling the k-th position
+    T = rng.uniform(0.5, 2.0, B).astype(np.float32)
+    for k in (1, 5, 15, 37, 299, 300, 1000):
+        r = oracle.topk_entropy(z, T, k)
+        for b in range(B):
+            y = z[b].astype(np.float64) / float(T[b])
+            p = special.softmax(y)
+            order = np.lexsort((np.arange(V), -y))       # y desc, token id asc
+            K, tail = order[:min(k, V)], order[min(k, V):]
+            m, mb = p[K].sum(), p[tail].sum()
+            Ht = stats.entropy(p[K] / m)
+            assert abs(r["H_tilde"][b] - Ht) < 1e-12
+            assert abs(r["tail_mass"][b] - mb) < 1e-12
+            H = stats.entropy(p)
+            Htail = stats.entropy(p[tail] / mb) if mb > 0 else 0.0
+            hb = special.entr(mb) + special.entr(1.0 - mb)
+            assert abs(H - (hb + m * Ht + mb * Htail)) < 1e-10
+            assert H <= r["H_hat"][b] + 1e-12
+            want = Ht + hb + (mb * np.log(V - k) if k < V else 0.0)
+            assert abs(r["H_hat"][b] - want) < 1e-10
+
+
+def test_topk_entropy_closed_forms():
+    V = 64
+    T = np.ones(1, np.float32)
+    # uniform logits: H~ = log k, m_bar = 1 - k/V, H^ = log V + m_bar log k
+    z = np.zeros((1, V), np.float32)
+    for k in (1, 8, 63, 64, 100):
+        r = oracle.topk_entropy(z, T, k)
+        ke = min(k, V)
+        mb = 1.0 - ke / V
+        assert abs(r["H_tilde"][0] - np.log(ke)) < 1e-12
+        assert abs(r["tail_mass"][0] - mb) < 1e-12
+        assert abs(r["H_hat"][0] - (np.log(V) + mb * np.log(ke))) < 1e-12
+    # one finite logit: all three are 0
+    z1 = np.full((1, V), -np.inf, np.float32)
+    z1[0, 5] = 2.0
+    r = oracle.topk_entropy(z1, T, 3)
+    assert r["H_tilde"][0] == 0.0 and r["tail_mass"][0] == 0.0 and r["H_hat"][0] == 0.0
+    # V = 2, k = 1: H~ = 0 and m_bar = min(p, 1 - p), so H^ = h(m_bar) = H exactly
+    for a in (-3.0, 0.0, 0.7, 5.0):
+        r = oracle.topk_entropy(np.array([[a, 0.0]], np.float32), T, 1)
+        p = special.expit(float(np.float32(a)))     # the logit the oracle sees
+        assert r["H_tilde"][0] == 0.0
+        assert abs(r["tail_mass"][0] - min(p, 1.0 - p)) < 1e-12
+        assert abs(r["H_hat"][0] - (special.entr(p) + special.entr(1.0 - p))) < 1e-12
+    # k >= V: both estimators are the exact entropy
+    zz = np.random.default_rng(4).standard_normal((3, 50)).astype(np.float32)
+    r = oracle.topk_entropy(zz, np.ones(3, np.float32), 50)
+    for b in range(3):
+        H = oracle.entropy_row(zz[b], 1.0)
+        assert abs(r["H_tilde"][b] - H) < 1e-12 and abs(r["H_hat"][b] - H) < 1e-12
+        assert r["tail_mass"][b] == 0.0
+
+
+def test_topk_entropy_error_rows():
+    z = np.zeros((4, 10), np.float32)
+    z[0, 3] = np.nan
+    z[1, 2] = np.inf
+    z[2] = -np.inf
+    T = np.array([1, 1, 1, 0], np.float32)
+    r = oracle.topk_entropy(z, T, 3)
+    assert list(r["err"]) == [oracle.ERR_NONFINITE, oracle.ERR_NONFINITE, oracle.ERR_ALL_NEG_INF,
+                              oracle.ERR_BAD_TEMP]
+    assert np.isnan(r["H_hat"]).all() and np.isnan(r["H_tilde"]).all()
