@@ -168,6 +168,36 @@ def ncu_traffic(kernel):
     return rec["bytes"] if h.hexdigest() == rec["sha256"] else None
 
 
+def run_estimators(eti, lg, step, prm, w, flush_l2, stream, k=64, reps=50):
+    """Time eti_topk_entropy (L2 flushed before each call) and correlate H~ and H^
+    with the exact entropy of the same rows (Pearson r over the batch)."""
+    B = w.B
+    f32 = torch.float32
+    Ht, Hh, tm = (torch.empty(B, dtype=f32, device=lg["logits"].device) for _ in range(3))
+    err = torch.empty(B, dtype=torch.int32, device=lg["logits"].device)
+    tau = lg["tau"].clone()
+    step.sample(lg["logits"], lg["T_in"], lg["H_prev"], tau, lg["H_target"], params=prm, seed=w.seed)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+    for i in range(reps + 3):
+        flush_l2()
+        if i >= 3:
+            ev[i - 3][0].record(stream)
+        eti.eti_topk_entropy(lg["logits"], lg["T_in"], k, Ht, Hh, err, tail_mass=tm)
+        if i >= 3:
+            ev[i - 3][1].record(stream)
+    torch.cuda.synchronize()
+    ms = statistics.median(e[0].elapsed_time(e[1]) for e in ev)
+    H = step.H.double().cpu().numpy()
+    r_t = float(np.corrcoef(H, Ht.double().cpu().numpy())[0, 1])
+    r_h = float(np.corrcoef(H, Hh.double().cpu().numpy())[0, 1])
+    return {"k": k, "topk_entropy_ms": round(ms, 5),
+            "topk_entropy_gbs": round(B * w.V * 4 / (ms / 1e3) / 1e9, 1),
+            "pearson_r_H_tilde_vs_H": round(r_t, 5), "pearson_r_H_hat_vs_H": round(r_h, 5),
+            "mean_tail_mass": round(float(tm.double().mean().item()), 6),
+            "note": "one CTA per row: radix select of the k-th logit (1 pass from HBM, 3 from L2); "
+                    "the exact entropy + sample pass is in kernels_ms['sample']"}
+
+
 def run_gpu(args):
     import paper_2603_03310_gb300 as eti
 
@@ -291,6 +321,12 @@ def run_gpu(args):
             "traffic_note": "ncu dram read+write per launch of the main kernel (profiles/), "
                             "null if its source changed since the capture"}
 
+    # top-k entropy estimators (Section 2.1) on the same logits: cost next to the
+    # exact pass, and how they track the exact entropy of the step
+    est = None
+    if not args.no_estimators:
+        est = run_estimators(eti, lg, step, prm, w, flush_l2, stream)
+
     # end to end through the public API: host (pinned) inputs -> device -> step -> host results
     e2e = None if args.no_e2e else run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm,
                                            args, device)
@@ -320,6 +356,7 @@ def run_gpu(args):
                               "entropy_sample_partial": 1, "entropy_sample_finalize": 1,
                               "memset (error flags, not a kernel of the library)": 1},
         "e2e": e2e,
+        "estimators": est,
         "wall_s_timed_region": round(wall, 4),
         "clocks": clk.summary(),
     }
@@ -481,6 +518,8 @@ def main(argv=None):
                     help="seconds of oracle work for the CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--no-estimators", action="store_true",
+                    help="skip the top-k entropy estimator line")
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu dram bytes per launch of the dominant kernel, if measured")
     args = ap.parse_args(argv)

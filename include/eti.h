@@ -202,6 +202,23 @@ int eti_entropy_temp_sample_noalloc(const float* logits, int B, int V, int64_t l
                                     uint32_t* err_flags, void* stream);
 
 /*
+ * eti_topk_entropy -- the top-k entropy estimators of Section 2.1, for each
+ * row b with y = z / T_in[b] over the first V entries of row b of `logits`
+ * (fp32, row stride ld >= V), p = softmax(y) and K the first min(k, V) tokens
+ * ordered by (y descending, token id ascending):
+ *   H_tilde[b]   = -sum_{x in K} p~(x) log p~(x),  p~ = p / sum_K p
+ *   tail_mass[b] = sum_{x not in K} p(x)            (= 1 - m_t; nullable)
+ *   H_hat[b]     = H_tilde + h(tail) + tail log(V - k)   (tail-corrected;
+ *                  the last term is 0 when k >= V; h: binary entropy)
+ * err_flags as for eti_entropy_temp_sample (NONFINITE, ALL_NEG_INF,
+ * BAD_TEMP; those rows get NaN).  k >= 1 (k > V is V).  No workspace; one
+ * pass over the logits from HBM and three from L2.
+ */
+int eti_topk_entropy(const float* logits, int B, int V, int64_t ld, const float* T_in, int k,
+                     float* H_tilde, float* H_hat, float* tail_mass, uint32_t* err_flags,
+                     void* stream);
+
+/*
  * Score modes: the reading of "the surprisal associated with the value
  * vector" I(v_i) in the block score of Section 3.2.
  *   ETI_SCORE_A  I(v_i) = -log a_i (attention as a distribution over the

@@ -32,7 +32,7 @@ SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_entropy_temp_sam
            "eti_score_prune_blocks", "eti_score_blocks", "eti_prune_blocks",
            "eti_paged_decode_workspace_size", "eti_paged_decode", "eti_version",
            "eti_status_string", "eti_entropy_temp_sample_noalloc",
-           "eti_entropy_temp_sample_noalloc_max_bytes")
+           "eti_entropy_temp_sample_noalloc_max_bytes", "eti_topk_entropy")
 
 
 class EtiError(RuntimeError):
@@ -76,6 +76,8 @@ def load(path: str | None = None):
         lib.eti_entropy_temp_sample_noalloc.restype = i32
         lib.eti_entropy_temp_sample_noalloc_max_bytes.restype = sz
         lib.eti_entropy_temp_sample.restype = i32
+        lib.eti_topk_entropy.argtypes = [P, i32, i32, i64, P, i32, P, P, P, P, P]
+        lib.eti_topk_entropy.restype = i32
         lib.eti_score_prune_workspace_size.argtypes = [i32] * 6
         lib.eti_score_prune_workspace_size.restype = sz
         lib.eti_score_prune_blocks.argtypes = ([P, P, P, P] + [i32] * 6 + [i64, f32, P, i32, i32, P]
@@ -198,6 +200,22 @@ def eti_entropy_temp_sample_noalloc(logits, T_in, H_prev, tau, H_target, tok, H,
         _dev(tok_surprisal, "tok_surprisal", f32, B), _surp_store(surp_store, slot_mapping, B),
         _dev(err_flags, "err_flags", torch.int32, B), _stream(stream))
     _check(st, "eti_entropy_temp_sample_noalloc")
+
+
+def eti_topk_entropy(logits, T_in, k: int, H_tilde, H_hat, err_flags, tail_mass=None,
+                     V: int | None = None, stream=None):
+    """Top-k entropy H~, tail-corrected H^ and tail mass (Section 2.1); see include/eti.h."""
+    B, ld = logits.shape
+    V = ld if V is None else int(V)
+    if logits.stride(1) != 1 or logits.stride(0) != ld:
+        raise EtiError("logits must be a row-major [B, ld] tensor")
+    f32 = torch.float32
+    st = load().eti_topk_entropy(
+        _dev(logits, "logits", f32), B, V, ld, _dev(T_in, "T_in", f32, B), int(k),
+        _dev(H_tilde, "H_tilde", f32, B), _dev(H_hat, "H_hat", f32, B),
+        _dev(tail_mass, "tail_mass", f32, B), _dev(err_flags, "err_flags", torch.int32, B),
+        _stream(stream))
+    _check(st, "eti_topk_entropy")
 
 
 def _attn_shapes(q, k_cache, block_table):

@@ -14,6 +14,9 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
                                    const eti_surp_store* store, uint32_t* err, void* part,
                                    cudaStream_t stream);
 size_t eti_entropy_partial_bytes(int B);
+int eti_launch_topk_entropy(const float* logits, int B, int V, long long ld, const float* T_in,
+                            int k, float* H_tilde, float* H_hat, float* tail_mass, uint32_t* err,
+                            cudaStream_t stream);
 int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const int32_t* block_table,
                             const int32_t* ctx_lens, int B, int Hq, int Hkv, int D, int P,
                             int max_blocks, long long num_pages, float scale, const float* tok_surp,
@@ -174,6 +177,16 @@ int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
     return eti_launch_entropy_temp_sample(logits, B, V, (long long)ld, T_in, H_prev, tau, H_target,
                                           params, seed, offset, tok, H, T_out, dH, theta_next,
                                           tok_surprisal, surp_store, err_flags, ws, (cudaStream_t)stream);
+}
+
+int eti_topk_entropy(const float* logits, int B, int V, int64_t ld, const float* T_in, int k,
+                     float* H_tilde, float* H_hat, float* tail_mass, uint32_t* err_flags,
+                     void* stream) {
+    if (B < 0 || B > 65535 || V < 1 || ld < V || k < 1) return ETI_ERR_SHAPE;
+    if (B == 0) return ETI_OK;
+    if (!logits || !T_in || !H_tilde || !H_hat || !err_flags) return ETI_ERR_NULL;
+    return eti_launch_topk_entropy(logits, B, V, (long long)ld, T_in, k, H_tilde, H_hat, tail_mass,
+                                   err_flags, (cudaStream_t)stream);
 }
 
 size_t eti_score_prune_workspace_size(int B, int Hq, int Hkv, int D, int P, int max_blocks) {
