@@ -54,7 +54,9 @@ class _Ctrl(ctypes.Structure):
     _fields_ = [("eta", ctypes.c_double), ("sign", ctypes.c_double),
                 ("T_min", ctypes.c_double), ("T_max", ctypes.c_double),
                 ("eps_H", ctypes.c_double), ("H_min", ctypes.c_double),
-                ("theta_user", ctypes.c_double), ("theta_hi", ctypes.c_double)]
+                ("theta_user", ctypes.c_double), ("theta_hi", ctypes.c_double),
+                ("T_cal", ctypes.c_double), ("rho_T", ctypes.c_double),
+                ("dtheta", ctypes.c_double)]
 
 
 def _load():
@@ -73,7 +75,7 @@ def _load():
             lib.oracle_entropy_row.argtypes = [P, i64, f64]
             lib.oracle_entropy_row.restype = f64
             lib.oracle_entropy_temp_sample.argtypes = (
-                [P, i32, i64, i64, P, P, P, P, P, u64, u64] + [P] * 9)
+                [P, i32, i64, i64, P, P, P, P, P, u64, u64] + [P] * 10)
             lib.oracle_topk_entropy.argtypes = [P, i32, i64, i64, P, i64, P, P, P, P]
             lib.oracle_score_prune.argtypes = (
                 [P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, i32, i32, P] + [P] * 8)
@@ -100,7 +102,7 @@ def num_threads() -> int:
 # eta 0.1, restoring sign, T in [0.05, 5], no estimator slack, no entropy
 # floor, no user threshold, theta_max scale 1).
 DEFAULT_CTRL = dict(eta=0.1, sign=-1.0, T_min=0.05, T_max=5.0, eps_H=0.0, H_min=0.0,
-                    theta_user=float("inf"), theta_hi=1.0)
+                    theta_user=float("inf"), theta_hi=1.0, T_cal=1.0, rho_T=0.0, dtheta=0.0)
 
 
 def ctrl(**kw) -> dict:
@@ -154,25 +156,27 @@ def topk_entropy(logits, T_in, k: int, V: int | None = None) -> dict:
 
 
 def entropy_temp_sample(logits, T_in, H_prev, tau_in, H_target, ctrl_params=None,
-                        seed: int = 0, offset: int = 0, V: int | None = None):
+                        seed: int = 0, offset: int = 0, V: int | None = None, theta_prev=None):
     """Entropy / entropic time / temperature / threshold / Gumbel-max sample.
 
-    logits: float32 [B, ld] (the first V columns are the vocabulary).
+    logits: float32 [B, ld] (the first V columns are the vocabulary);
+    theta_prev float32 [B]: the previous thresholds (used by the dtheta guard).
     Returns a dict of numpy arrays (double outputs, int32 tok, uint32 err).
     """
     lib = _load()
     z = _c(logits, np.float32)
     B, ld = z.shape
     V = ld if V is None else V
-    cp = _Ctrl(**(ctrl_params or DEFAULT_CTRL))
+    cp = _Ctrl(**{**DEFAULT_CTRL, **(ctrl_params or {})})
     T_in, H_prev, tau_in, H_target = (_c(a, np.float32) for a in (T_in, H_prev, tau_in, H_target))
+    theta_prev = None if theta_prev is None else _c(theta_prev, np.float32)
     out = {k: np.empty(B, np.float64) for k in
            ("H", "T_out", "dH", "tau", "theta_next", "surprisal", "margin")}
     tok = np.empty(B, np.int32)
     err = np.empty(B, np.uint32)
     lib.oracle_entropy_temp_sample(
         _ptr(z), B, V, ld, _ptr(T_in), _ptr(H_prev), _ptr(tau_in), _ptr(H_target),
-        ctypes.byref(cp), seed, offset, _ptr(tok), _ptr(out["H"]), _ptr(out["T_out"]),
+        ctypes.byref(cp), seed, offset, _ptr(theta_prev), _ptr(tok), _ptr(out["H"]), _ptr(out["T_out"]),
         _ptr(out["dH"]), _ptr(out["tau"]), _ptr(out["theta_next"]), _ptr(out["surprisal"]),
         _ptr(out["margin"]), _ptr(err))
     out["tok"] = tok

@@ -32,6 +32,9 @@
  *   R7  keep iff score >= theta, or the block is among the first
  *       min(B_min, n_b) blocks ordered by (score desc, block index asc).
  *   R8  attention restricted to the kept blocks renormalises over them.
+ *   R9  the Section 5 guards: calibration rescales the logits by 1 / T_cal
+ *       before the step (entropy and draw use z / (T_cal T_t)); the rate
+ *       limits bound |log T_{t+1} - log T_t| and |theta_{t+1} - theta_t|.
  */
 #include <math.h>
 #include <stdint.h>
@@ -139,6 +142,9 @@ typedef struct {
     double H_min;      /* entropy floor for pruning decisions (Section 5) */
     double theta_user; /* user threshold theta_t before the safety floor */
     double theta_hi;   /* scale of theta_max(H) */
+    double T_cal;      /* global calibration temperature (Section 5; reading R9) */
+    double rho_T;      /* bound on |log T_{t+1} - log T_t| per step, 0 = none (Section 5) */
+    double dtheta;     /* bound on |theta_{t+1} - theta_t| per step, 0 = none (Section 5) */
 } oracle_ctrl;
 
 /*
@@ -152,6 +158,11 @@ typedef struct {
  *  theta_max(H) = theta_hi * max(0, 1 - H / log V)               (reading R6)
  *  tok       = argmax_x  z_x/T_t - log(-log u_x)                 (Gumbel-max draw from p)
  *  surprisal = -log p(tok)
+ * Guards of Section 5 (reading R9): the logits are recalibrated by T_cal
+ * before everything above (p from z / (T_cal T_t)); the new temperature is
+ * kept within a factor e^{rho_T} of T_t before the [T_min, T_max] clip; the
+ * new threshold within dtheta of the previous one, theta_prev[b] (a finite
+ * previous threshold only; 0 turns either bound off).
  *
  * Outputs are double.  margin[b] = best key minus second-best key.  Rows with
  * a NaN or +inf logit, with every logit -inf, or with a temperature that is
@@ -161,7 +172,7 @@ typedef struct {
 void oracle_entropy_temp_sample(const float *logits, int B, int64_t V, int64_t ld,
                                 const float *T_in, const float *H_prev, const float *tau_in,
                                 const float *H_target, const oracle_ctrl *cp,
-                                uint64_t seed, uint64_t offset,
+                                uint64_t seed, uint64_t offset, const float *theta_prev,
                                 int32_t *tok, double *H, double *T_out, double *dH,
                                 double *tau_out, double *theta_next, double *surprisal,
                                 double *margin, uint32_t *err) {
@@ -169,7 +180,8 @@ void oracle_entropy_temp_sample(const float *logits, int B, int64_t V, int64_t l
 #pragma omp parallel for schedule(dynamic, 1)
     for (int b = 0; b < B; ++b) {
         const float *z = logits + (int64_t)b * ld;
-        const double T = (double)T_in[b];
+        const double Tt = (double)T_in[b];
+        const double T = Tt * cp->T_cal;          /* calibrated logits at temperature T_t */
         uint32_t e = (T > 0.0 && !isinf(T)) ? 0u : ORC_ERR_BAD_TEMP;
         double m = -INFINITY;
         for (int64_t x = 0; x < V && !e; ++x) {
@@ -180,7 +192,7 @@ void oracle_entropy_temp_sample(const float *logits, int B, int64_t V, int64_t l
         if (!e && isinf(m)) e |= ORC_ERR_ALL_NEG_INF;
         err[b] = e;
         if (e) {
-            tok[b] = -1; H[b] = NAN; dH[b] = NAN; T_out[b] = T;
+            tok[b] = -1; H[b] = NAN; dH[b] = NAN; T_out[b] = Tt;
             tau_out[b] = (double)tau_in[b]; theta_next[b] = 0.0;
             surprisal[b] = NAN; margin[b] = NAN;
             continue;
@@ -213,11 +225,17 @@ void oracle_entropy_temp_sample(const float *logits, int B, int64_t V, int64_t l
         surprisal[b] = -(((double)z[arg] / T - m) - log(S));
         dH[b] = (double)H_prev[b] - h;
         tau_out[b] = (double)tau_in[b] + fmax(0.0, dH[b]);
-        double Tn = T * exp(cp->sign * cp->eta * (h - (double)H_target[b]));
+        double Tn = Tt * exp(cp->sign * cp->eta * (h - (double)H_target[b]));
+        if (cp->rho_T > 0.0) Tn = fmin(Tt * exp(cp->rho_T), fmax(Tt * exp(-cp->rho_T), Tn));
         T_out[b] = fmin(cp->T_max, fmax(cp->T_min, Tn));
         double Heff = fmax(h - cp->eps_H, cp->H_min);
         double tmax = (V > 1) ? cp->theta_hi * fmax(0.0, 1.0 - Heff / logV) : cp->theta_hi;
-        theta_next[b] = fmin(cp->theta_user, tmax);
+        double th = fmin(cp->theta_user, tmax);
+        if (cp->dtheta > 0.0 && theta_prev && isfinite((double)theta_prev[b])) {
+            const double tp = (double)theta_prev[b];
+            th = fmin(tp + cp->dtheta, fmax(tp - cp->dtheta, th));
+        }
+        theta_next[b] = th;
     }
 }
 

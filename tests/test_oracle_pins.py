@@ -679,3 +679,78 @@ def test_topk_entropy_error_rows():
     assert list(r["err"]) == [oracle.ERR_NONFINITE, oracle.ERR_NONFINITE, oracle.ERR_ALL_NEG_INF,
                               oracle.ERR_BAD_TEMP]
     assert np.isnan(r["H_hat"]).all() and np.isnan(r["H_tilde"]).all()
+
+
+# ---------------------------------------------------------------------------
+# guards of Section 5 (reading R9): calibration and rate limits
+
+def _guard_inputs(B=6, V=500, seed=7):
+    rng = np.random.default_rng(seed)
+    z = (rng.standard_normal((B, V)) * rng.uniform(0.3, 5.0, (B, 1))).astype(np.float32)
+    T = np.array([0.5, 1.0, 2.0, 4.0, 1.0, 0.5][:B], np.float32)
+    Hp = rng.uniform(0, np.log(V), B).astype(np.float32)
+    tau = rng.uniform(0, 3, B).astype(np.float32)
+    Ht = np.full(B, 0.5 * np.log(V), np.float32)
+    return z, T, Hp, tau, Ht
+
+
+def test_guard_calibration_is_a_logit_rescale():
+    """T_cal rescales the logits: (T_t, T_cal) gives the entropy, token,
+    surprisal and threshold of (T_t T_cal, 1) exactly (the products are exact
+    here), and T_out(T_t, T_cal) T_cal = T_out(T_t T_cal, 1) with wide clips."""
+    z, T, Hp, tau, Ht = _guard_inputs()
+    c = 1.5
+    wide = dict(T_min=1e-6, T_max=1e6)
+    r1 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, ctrl_params=oracle.ctrl(T_cal=c, **wide), seed=3)
+    r2 = oracle.entropy_temp_sample(z, (T * np.float32(c)).astype(np.float32), Hp, tau, Ht,
+                                    ctrl_params=oracle.ctrl(**wide), seed=3)
+    for k in ("H", "tok", "surprisal", "theta_next", "tau", "dH"):
+        assert np.array_equal(r1[k], r2[k]), k
+    assert np.allclose(r1["T_out"] * c, r2["T_out"], rtol=1e-12)
+    # and calibration moves the entropy the way a temperature does: up with T_cal
+    r3 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, ctrl_params=oracle.ctrl(T_cal=2 * c, **wide), seed=3)
+    assert (r3["H"] > r1["H"]).all()
+
+
+def test_guard_temperature_rate_limit():
+    """|log T_{t+1} - log T_t| <= rho_T: steps inside the bound are unchanged,
+    larger ones end exactly at T_t e^{+-rho_T}; [T_min, T_max] still holds."""
+    z, T, Hp, tau, Ht = _guard_inputs(seed=8)
+    rho = 0.05
+    base = dict(eta=2.0, T_min=1e-6, T_max=1e6)
+    # targets near and far from each row's entropy: steps 2 eta |H - H*| small and large
+    H = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, seed=1)["H"]
+    Ht = (H + np.array([0.001, -0.001, 0.5, -0.5, 0.01, 2.0])).astype(np.float32)
+    r0 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, ctrl_params=oracle.ctrl(**base), seed=1)
+    r1 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, ctrl_params=oracle.ctrl(rho_T=rho, **base), seed=1)
+    step = np.log(r0["T_out"] / T.astype(np.float64))
+    assert (np.abs(step) > rho).any() and (np.abs(step) <= rho).any()   # both branches occur
+    for b in range(len(T)):
+        if abs(step[b]) <= rho:
+            assert r1["T_out"][b] == r0["T_out"][b]
+        else:
+            assert abs(r1["T_out"][b] - float(T[b]) * np.exp(np.sign(step[b]) * rho)) < 1e-12
+    r2 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht,
+                                    ctrl_params=oracle.ctrl(rho_T=rho, eta=2.0, T_min=0.9, T_max=1.1), seed=1)
+    assert ((r2["T_out"] >= 0.9) & (r2["T_out"] <= 1.1)).all()
+    assert np.array_equal(r1["H"], r0["H"]) and np.array_equal(r1["tok"], r0["tok"])
+
+
+def test_guard_threshold_rate_limit():
+    """|theta_{t+1} - theta_t| <= dtheta against a finite previous threshold;
+    an infinite previous threshold (first step) leaves the rule alone."""
+    z, T, Hp, tau, Ht = _guard_inputs(seed=9)
+    d = 0.03
+    r0 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, seed=2)
+    tp = (r0["theta_next"] + np.array([0.0, 0.5, -0.5, 0.01, np.inf, -0.2])).astype(np.float32)
+    r1 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, ctrl_params=oracle.ctrl(dtheta=d), seed=2,
+                                    theta_prev=tp)
+    for b in range(len(T)):
+        want = r0["theta_next"][b]
+        if np.isfinite(tp[b]):
+            want = min(float(tp[b]) + d, max(float(tp[b]) - d, want))
+        assert r1["theta_next"][b] == want
+    assert not np.array_equal(r1["theta_next"], r0["theta_next"])
+    # off (dtheta = 0): theta_prev is ignored
+    r2 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, seed=2, theta_prev=tp)
+    assert np.array_equal(r2["theta_next"], r0["theta_next"])
