@@ -98,6 +98,14 @@ typedef uint16_t eti_bf16;
  *   H_min       entropy floor for pruning decisions (Section 5)   (0)
  *   theta_user  threshold before the safety floor                 (+inf)
  *   theta_hi    scale of theta_max(H) = theta_hi * max(0, 1 - H / log V) (1)
+ *   T_cal       global calibration temperature: the logits are read as
+ *               z / T_cal before everything else (Section 5)       (1)
+ *   rho_T       bound on |log T_out - log T_in| per step, applied before
+ *               the [T_min, T_max] clip; 0 = none (Section 5)        (0)
+ *   dtheta      bound on |theta_next - theta_prev| per step; when > 0,
+ *               theta_next is read first as the previous threshold (in
+ *               place, like tau; a non-finite previous value is not
+ *               bounded); 0 = none (Section 5)                        (0)
  */
 typedef struct {
     float eta;
@@ -108,6 +116,9 @@ typedef struct {
     float H_min;
     float theta_user;
     float theta_hi;
+    float T_cal;
+    float rho_T;
+    float dtheta;
 } eti_ctrl_params;
 
 void eti_ctrl_defaults(eti_ctrl_params* p);
@@ -122,6 +133,8 @@ void eti_ctrl_defaults(eti_ctrl_params* p);
  *   tau[b]    += max(0, dH[b])         (entropic time, in place; Section 2)
  *   T_out[b]   = clip(T_in[b] exp(sign eta (H[b] - H_target[b])), T_min, T_max)
  *                                                                (Section 3.3)
+ *   (with the Section 5 guards of eti_ctrl_params: y = z / (T_cal T_in[b]),
+ *   the rho_T bound on the step of T, the dtheta bound on theta_next)
  *   theta_next[b] = min(theta_user, theta_hi max(0, 1 - max(H - eps_H, H_min) / log V))
  *                  (threshold floor of Section 3.2 with the Section 5 floor;
  *                   theta_hi when V == 1)

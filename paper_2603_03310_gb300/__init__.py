@@ -42,7 +42,8 @@ class EtiError(RuntimeError):
 class CtrlParams(ctypes.Structure):
     """eti_ctrl_params (include/eti.h)."""
     _fields_ = [(n, ctypes.c_float) for n in
-                ("eta", "sign", "T_min", "T_max", "eps_H", "H_min", "theta_user", "theta_hi")]
+                ("eta", "sign", "T_min", "T_max", "eps_H", "H_min", "theta_user", "theta_hi",
+                 "T_cal", "rho_T", "dtheta")]
 
 
 def build(force: bool = False) -> str:

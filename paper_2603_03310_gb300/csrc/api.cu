@@ -136,6 +136,9 @@ void eti_ctrl_defaults(eti_ctrl_params* p) {
     p->H_min = 0.0f;
     p->theta_user = __builtin_huge_valf();
     p->theta_hi = 1.0f;
+    p->T_cal = 1.0f;
+    p->rho_T = 0.0f;
+    p->dtheta = 0.0f;
 }
 
 const char* eti_version(void) { return "libeti 0.1.0 (sm_103a)"; }

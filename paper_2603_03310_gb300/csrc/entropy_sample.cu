@@ -203,7 +203,7 @@ entropy_sample_partial_kernel(const __grid_constant__ EtsArgs a) {
         const int b = (int)(q0 / a.ngroups);
         const int g0 = (int)(q0 - (long long)b * a.ngroups);
         const int g1 = (int)min((long long)a.ngroups, q1 - (long long)b * a.ngroups);
-        const float T = a.T_in[b];
+        const float T = a.T_in[b] * a.p.T_cal;   // calibrated logits at temperature T_t
         const bool bad_T = !(T > 0.f && T < kInf);
         const float c = bad_T ? 0.f : kLog2e / T;
         const float* row = a.logits + (long long)b * a.ld;
@@ -320,7 +320,8 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
     const int lane = threadIdx.x & 31;
     const int b = blockIdx.x * 4 + (threadIdx.x >> 5);
     if (b >= a.B) return;
-    const float T = a.T_in[b];
+    const float Tt = a.T_in[b];
+    const float T = Tt * a.p.T_cal;              // calibrated logits at temperature T_t
     const bool bad_T = !(T > 0.f && T < kInf);
     const float c = bad_T ? 0.f : kLog2e / T;
     const long long lo = (long long)b * a.ngroups, hi = lo + a.ngroups - 1;
@@ -349,7 +350,7 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
     if (err) {
         a.tok[b] = -1;
         a.H[b] = __int_as_float(0x7fc00000);
-        a.T_out[b] = T;
+        a.T_out[b] = Tt;
         if (a.dH) a.dH[b] = __int_as_float(0x7fc00000);
         if (a.theta_next) a.theta_next[b] = 0.f;
         if (a.surprisal) a.surprisal[b] = __int_as_float(0x7fc00000);
@@ -358,7 +359,8 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
         const float H = fmaxf(kLn2 * (l2S - t.U / t.S), 0.f);
         const float dH = a.H_prev[b] - H;
         a.tau[b] = tau_in + fmaxf(dH, 0.f);
-        float Tn = T * expf(a.p.sign * a.p.eta * (H - a.H_target[b]));
+        float Tn = Tt * expf(a.p.sign * a.p.eta * (H - a.H_target[b]));
+        if (a.p.rho_T > 0.f) Tn = fminf(Tt * expf(a.p.rho_T), fmaxf(Tt * expf(-a.p.rho_T), Tn));
         Tn = fminf(a.p.T_max, fmaxf(a.p.T_min, Tn));
         a.tok[b] = t.bi;
         a.H[b] = H;
@@ -368,7 +370,12 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
             const float Heff = fmaxf(H - a.p.eps_H, a.p.H_min);
             const float tmax = a.V > 1 ? a.p.theta_hi * fmaxf(0.f, 1.f - Heff / logf((float)a.V))
                                        : a.p.theta_hi;
-            a.theta_next[b] = fminf(a.p.theta_user, tmax);
+            float th = fminf(a.p.theta_user, tmax);
+            if (a.p.dtheta > 0.f) {
+                const float tp = a.theta_next[b];   // the previous threshold, in place
+                if (isfinite(tp)) th = fminf(tp + a.p.dtheta, fmaxf(tp - a.p.dtheta, th));
+            }
+            a.theta_next[b] = th;
         }
         if (a.surprisal || a.surp_store) {
             const float tt = fmaf(row[t.bi], c, -t.mc);

@@ -29,15 +29,17 @@ MASK_TIE = 1e-5
 ATTN_ABS = 2e-2
 
 
-def run_ets(eti, lg: dict, params=None, seed=0, offset=0, V=None):
-    """Run eti_entropy_temp_sample on the workload's logits; numpy results."""
+def run_ets(eti, lg: dict, params=None, seed=0, offset=0, V=None, theta_prev=None):
+    """Run eti_entropy_temp_sample on the workload's logits; numpy results.
+    theta_prev (numpy [B]) fills theta_next first (read by the dtheta guard)."""
     B = lg["logits"].shape[0]
     dev = lg["logits"].device
     f32, i32 = torch.float32, torch.int32
     tau = lg["tau"].clone()
     out = dict(tok=torch.empty(B, dtype=i32, device=dev), H=torch.empty(B, dtype=f32, device=dev),
                T_out=torch.empty(B, dtype=f32, device=dev), dH=torch.empty(B, dtype=f32, device=dev),
-               theta_next=torch.empty(B, dtype=f32, device=dev),
+               theta_next=(torch.empty(B, dtype=f32, device=dev) if theta_prev is None else
+                           torch.tensor(np.asarray(theta_prev, np.float32), device=dev)),
                surprisal=torch.empty(B, dtype=f32, device=dev),
                err=torch.empty(B, dtype=i32, device=dev))
     ws = torch.empty(eti.entropy_temp_sample_workspace_size(B, V or lg["logits"].shape[1]),
@@ -53,11 +55,11 @@ def run_ets(eti, lg: dict, params=None, seed=0, offset=0, V=None):
     return res
 
 
-def oracle_ets(lg: dict, ctrl=None, seed=0, offset=0, V=None):
+def oracle_ets(lg: dict, ctrl=None, seed=0, offset=0, V=None, theta_prev=None):
     return oracle.entropy_temp_sample(lg["logits"].cpu().numpy(), lg["T_in"].cpu().numpy(),
                                       lg["H_prev"].cpu().numpy(), lg["tau"].cpu().numpy(),
                                       lg["H_target"].cpu().numpy(), ctrl, seed=seed, offset=offset,
-                                      V=V)
+                                      V=V, theta_prev=theta_prev)
 
 
 def _close(a, b, rel, abs_=0.0):

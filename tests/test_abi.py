@@ -55,6 +55,7 @@ def test_ctrl_defaults(lib):
     assert (p.eta, p.sign, p.T_min, p.T_max, p.eps_H, p.H_min, p.theta_hi) == \
         pytest.approx((0.1, -1.0, 0.05, 5.0, 0.0, 0.0, 1.0))
     assert p.theta_user == float("inf")
+    assert (p.T_cal, p.rho_T, p.dtheta) == (1.0, 0.0, 0.0)     # guards off by default
 
 
 NULL = None

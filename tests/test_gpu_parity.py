@@ -79,7 +79,9 @@ def test_entropy_sample_strided_and_unaligned_rows(eti):
 
 
 @pytest.mark.parametrize("kw", [dict(), dict(sign=1.0), dict(eta=0.5, T_min=0.5, T_max=1.5),
-                                dict(eps_H=0.7, H_min=3.0, theta_user=0.4, theta_hi=2.0)])
+                                dict(eps_H=0.7, H_min=3.0, theta_user=0.4, theta_hi=2.0),
+                                dict(T_cal=1.5), dict(T_cal=0.7, eta=0.3),
+                                dict(rho_T=0.05, eta=2.0, T_min=1e-3, T_max=1e3)])
 def test_entropy_sample_controller_params(eti, kw):
     w = workloads.WORKLOADS["tiny"].scaled(B=16, ctx=("list", [1] * 16), seed=11)
     lg = workloads.make_logits(w, DEV)
@@ -88,6 +90,22 @@ def test_entropy_sample_controller_params(eti, kw):
     g = parity.run_ets(eti, lg, params=p, seed=5, offset=1)
     r = parity.oracle_ets(lg, ctrl=c, seed=5, offset=1)
     parity.compare_ets(g, r, lg, seed=5, offset=1)
+
+
+def test_entropy_sample_threshold_rate_limit(eti):
+    """The dtheta guard: theta_next is read as the previous threshold and the
+    new one stays within dtheta of it (non-finite previous values unbounded)."""
+    w = workloads.WORKLOADS["tiny"].scaled(B=16, ctx=("list", [1] * 16), seed=12)
+    lg = workloads.make_logits(w, DEV)
+    base = parity.oracle_ets(lg, seed=3)
+    rng = np.random.default_rng(0)
+    tp = (base["theta_next"] + rng.uniform(-0.1, 0.1, w.B)).astype(np.float32)
+    tp[[2, 9]] = np.inf
+    p, c = _ctrl_pair(eti, dtheta=0.02)
+    g = parity.run_ets(eti, lg, params=p, seed=3, theta_prev=tp)
+    r = parity.oracle_ets(lg, ctrl=c, seed=3, theta_prev=tp)
+    parity.compare_ets(g, r, lg, seed=3)
+    assert (np.abs(g["theta_next"] - tp)[np.isfinite(tp)] <= 0.02 + 1e-6).all()
 
 
 def test_entropy_sample_error_rows(eti):
