@@ -77,6 +77,7 @@ def _load():
             lib.oracle_entropy_temp_sample.argtypes = (
                 [P, i32, i64, i64, P, P, P, P, P, u64, u64] + [P] * 10)
             lib.oracle_topk_entropy.argtypes = [P, i32, i64, i64, P, i64, P, P, P, P]
+            lib.oracle_schedule.argtypes = [P, P, P, i32, i32, P, P, P, i32, i32, P, P, P]
             lib.oracle_score_prune.argtypes = (
                 [P, P, P, P, i32, i32, i32, i32, i32, i32, i64, f64, P, i32, i32, P] + [P] * 8)
             lib.oracle_paged_attention.argtypes = (
@@ -135,6 +136,35 @@ def sample_key(logits_row, T: float, seed: int, offset: int, row: int, x: int) -
 def entropy_row(z, T: float = 1.0) -> float:
     z = _c(z, np.float32)
     return float(_load().oracle_entropy_row(_ptr(z), z.shape[0], float(T)))
+
+
+class _Sched(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_double) for n in ("lambda_", "alpha", "beta", "gamma", "den_min")]
+
+
+DEFAULT_SCHED = dict(lambda_=0.9, alpha=1e-3, beta=1e-3, gamma=1.0, den_min=1e-6)
+
+
+def schedule(dH, ema_in, budget: int, kept_cnt=None, P: int = 16, ctx_lens=None, urgency=None,
+             params=None) -> dict:
+    """Entropy-aware priority pi(s) and the admitted set (Section 3.1, reading R10).
+
+    dH, ema_in, urgency float32 [B]; kept_cnt int32 [B, Hkv]; ctx_lens int32 [B].
+    """
+    lib = _load()
+    dH = _c(dH, np.float32)
+    B = dH.shape[0]
+    ema_in = _c(ema_in, np.float32)
+    kc = None if kept_cnt is None else _c(kept_cnt, np.int32)
+    Hkv = 1 if kc is None else kc.shape[1]
+    cl = None if ctx_lens is None else _c(ctx_lens, np.int32)
+    ur = None if urgency is None else _c(urgency, np.float32)
+    sp = _Sched(**{**DEFAULT_SCHED, **(params or {})})
+    out = dict(ema=np.empty(B), priority=np.empty(B), admit=np.empty(B, np.uint8))
+    lib.oracle_schedule(_ptr(dH), _ptr(ema_in), _ptr(kc), Hkv, int(P), _ptr(cl), _ptr(ur),
+                        ctypes.byref(sp), B, int(budget), _ptr(out["ema"]), _ptr(out["priority"]),
+                        _ptr(out["admit"]))
+    return out
 
 
 def topk_entropy(logits, T_in, k: int, V: int | None = None) -> dict:

@@ -32,6 +32,9 @@
  *   R7  keep iff score >= theta, or the block is among the first
  *       min(B_min, n_b) blocks ordered by (score desc, block index asc).
  *   R8  attention restricted to the kept blocks renormalises over them.
+ *   R10 scheduling priority: E[dH_s] is an exponential moving average of
+ *       max(0, dH_s); C_s, M_s, L_s are kept tokens, context length and a
+ *       caller urgency (Section 3.1 names them without formulas).
  *   R9  the Section 5 guards: calibration rescales the logits by 1 / T_cal
  *       before the step (entropy and draw use z / (T_cal T_t)); the rate
  *       limits bound |log T_{t+1} - log T_t| and |theta_{t+1} - theta_t|.
@@ -251,6 +254,63 @@ double oracle_entropy_row(const float *z, int64_t V, double T) {
         if (p > 0.0) h -= p * log(p);
     }
     return h;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Entropy-aware scheduling priority and admission (Section 3.1, reading R10).
+ *
+ *   E[dH_s] <- lambda E[dH_s] + (1 - lambda) max(0, dH_s)   (the expected
+ *              irreversible entropy reduction, an exponential moving average of
+ *              the reductions that entropic time counts; a NaN dH leaves it)
+ *   C_s = kept tokens per kv head (attention work of the step),
+ *   M_s = context length (KV memory), L_s = caller-given urgency,
+ *   pi(s) = E[dH_s] / max(alpha C_s + beta M_s + gamma L_s, den_min)
+ * and the `budget` sequences of highest pi are admitted (ties to the lower
+ * index; a NaN priority ranks below every number).  kept_cnt, ctx_lens and
+ * urgency may be NULL (the term is 0). */
+typedef struct {
+    double lambda, alpha, beta, gamma, den_min;
+} oracle_sched;
+
+typedef struct { double pi; int idx; } sched_item;
+
+static int sched_cmp(const void *pa, const void *pb) {
+    const sched_item *a = (const sched_item *)pa, *b = (const sched_item *)pb;
+    const int na = isnan(a->pi), nb = isnan(b->pi);
+    if (na != nb) return na - nb;               /* NaN after every number */
+    if (!na) {
+        if (a->pi > b->pi) return -1;
+        if (a->pi < b->pi) return 1;
+    }
+    return (a->idx > b->idx) - (a->idx < b->idx);
+}
+
+void oracle_schedule(const float *dH, const float *ema_in, const int32_t *kept_cnt, int Hkv, int P,
+                     const int32_t *ctx_lens, const float *urgency, const oracle_sched *sp, int B,
+                     int budget, double *ema_out, double *priority, uint8_t *admit) {
+    sched_item *order = (sched_item *)malloc(sizeof(sched_item) * (size_t)(B > 0 ? B : 1));
+    for (int s = 0; s < B; ++s) {
+        const double d = (double)dH[s];
+        double e = (double)ema_in[s];
+        if (!isnan(d)) e = sp->lambda * e + (1.0 - sp->lambda) * fmax(0.0, d);
+        double C = 0.0;
+        if (kept_cnt) {
+            for (int h = 0; h < Hkv; ++h) C += (double)kept_cnt[(int64_t)s * Hkv + h] * P;
+            C /= Hkv;
+        }
+        const double M = ctx_lens ? (double)ctx_lens[s] : 0.0;
+        const double L = urgency ? (double)urgency[s] : 0.0;
+        const double den = fmax(sp->alpha * C + sp->beta * M + sp->gamma * L, sp->den_min);
+        ema_out[s] = e;
+        priority[s] = e / den;
+        order[s].pi = priority[s];
+        order[s].idx = s;
+        admit[s] = 0;
+    }
+    qsort(order, (size_t)B, sizeof(sched_item), sched_cmp);
+    const int n = budget < B ? (budget > 0 ? budget : 0) : B;
+    for (int r = 0; r < n; ++r) admit[order[r].idx] = 1;
+    free(order);
 }
 
 /* ------------------------------------------------------------------------ */

@@ -754,3 +754,78 @@ def test_guard_threshold_rate_limit():
     # off (dtheta = 0): theta_prev is ignored
     r2 = oracle.entropy_temp_sample(z, T, Hp, tau, Ht, seed=2, theta_prev=tp)
     assert np.array_equal(r2["theta_next"], r0["theta_next"])
+
+
+# ---------------------------------------------------------------------------
+# entropy-aware scheduling priority (Section 3.1, reading R10)
+
+def test_schedule_limits_and_closed_forms():
+    rng = np.random.default_rng(5)
+    B = 12
+    dH = rng.normal(0.05, 0.2, B).astype(np.float32)
+    ema = rng.uniform(0, 0.3, B).astype(np.float32)
+    # lambda = 0: the average is the last irreversible reduction; lambda = 1: unchanged
+    r0 = oracle.schedule(dH, ema, 3, params=dict(lambda_=0.0))
+    assert np.array_equal(r0["ema"], np.maximum(dH.astype(np.float64), 0.0))
+    r1 = oracle.schedule(dH, ema, 3, params=dict(lambda_=1.0))
+    assert np.array_equal(r1["ema"], ema.astype(np.float64))
+    # only the urgency term, L = 1, gamma = 1: pi = E[dH]
+    r2 = oracle.schedule(dH, ema, 3, urgency=np.ones(B, np.float32),
+                         params=dict(alpha=0.0, beta=0.0, gamma=1.0))
+    assert np.array_equal(r2["priority"], r2["ema"])
+    # more kept tokens (attention work) strictly lowers the priority of a sequence
+    kc = rng.integers(1, 50, (B, 8)).astype(np.int32)
+    ra = oracle.schedule(dH, ema, 3, kept_cnt=kc)
+    rb = oracle.schedule(dH, ema, 3, kept_cnt=kc + 5)
+    pos = ra["ema"] > 0
+    assert (rb["priority"][pos] < ra["priority"][pos]).all()
+    # Proposition 2: priorities are bounded by max E[dH] / den_min
+    assert (ra["priority"] <= ra["ema"].max() / 1e-6 + 1e-9).all()
+
+
+def test_schedule_admits_the_top_budget():
+    """The admitted set is the first `budget` of (priority desc, index asc),
+    checked against Python's sorted(); ties go to the lower index; NaN last."""
+    rng = np.random.default_rng(6)
+    B = 40
+    dH = rng.normal(0.0, 0.3, B).astype(np.float32)
+    ema = rng.uniform(0, 0.2, B).astype(np.float32)
+    ema[[3, 17, 25]] = 0.125                       # equal priorities
+    dH[[3, 17, 25]] = np.nan                       # (their averages stay as given)
+    ema[30] = np.nan                               # a NaN priority
+    L = np.ones(B, np.float32)
+    for budget in (-1, 0, 1, 5, 20, 39, 40, 100):
+        r = oracle.schedule(dH, ema, budget, urgency=L, params=dict(alpha=0.0, beta=0.0))
+        key = [((1, 0.0) if np.isnan(p) else (0, -p), i) for i, p in enumerate(r["priority"])]
+        want = np.zeros(B, np.uint8)
+        for _, i in sorted(key)[:max(0, min(budget, B))]:
+            want[i] = 1
+        assert np.array_equal(r["admit"], want), budget
+    # equal priorities across the budget's edge: the lower indices go in
+    tie = oracle.schedule(np.full(6, np.nan, np.float32), np.array([0.1, 0.3, 0.3, 0.3, 0.3, 0.2], np.float32),
+                          3, urgency=np.ones(6, np.float32), params=dict(alpha=0.0, beta=0.0))
+    assert list(tie["admit"]) == [0, 1, 1, 1, 0, 0]
+
+
+def test_schedule_no_starvation_when_served_sequences_resolve():
+    """Proposition 3 in a toy run: a served sequence's entropy contracts
+    (H <- 0.7 H + noise), so its reductions and average fade, and with a
+    budget of 2 out of 8 every sequence is served within a bounded time."""
+    rng = np.random.default_rng(7)
+    B, budget, steps = 8, 2, 60
+    H = rng.uniform(2.0, 6.0, B)
+    ema = np.full(B, 0.5, np.float32)
+    dH = np.zeros(B, np.float32)
+    served = np.zeros(B, bool)
+    for t in range(steps):
+        r = oracle.schedule(dH, ema, budget, params=dict(lambda_=0.7, alpha=0.0, beta=0.0, gamma=1.0),
+                            urgency=np.ones(B, np.float32))
+        adm = r["admit"].astype(bool)
+        served |= adm
+        ema = r["ema"].astype(np.float32)
+        newH = np.where(adm, 0.7 * H + rng.normal(0, 0.05, B).clip(-0.1, 0.1), H)
+        dH = np.where(adm, H - newH, np.nan).astype(np.float32)   # waiting sequences observe nothing
+        H = np.maximum(newH, 0.0)
+        if served.all():
+            break
+    assert served.all(), (t, served)
