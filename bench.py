@@ -194,8 +194,30 @@ def run_estimators(eti, lg, step, prm, w, flush_l2, stream, k=64, reps=50):
             "topk_entropy_gbs": round(B * w.V * 4 / (ms / 1e3) / 1e9, 1),
             "pearson_r_H_tilde_vs_H": round(r_t, 5), "pearson_r_H_hat_vs_H": round(r_h, 5),
             "mean_tail_mass": round(float(tm.double().mean().item()), 6),
-            "note": "one CTA per row: radix select of the k-th logit (1 pass from HBM, 3 from L2); "
-                    "the exact entropy + sample pass is in kernels_ms['sample']"}
+            "note": "one CTA per row: the k-th largest thread maximum bounds the k-th logit, the "
+                    "tokens above it are sorted (1 pass from HBM, 1 from L2); the exact entropy + "
+                    "sample pass is kernels_ms['sample']; schedule_ms: Section 3.1 priority and "
+                    "admission of half the batch"}
+
+
+def run_schedule(eti, step, kv, w, stream, reps=50):
+    """Median time of eti_schedule (Section 3.1 priority + admission of half
+    the batch) on the step's entropy flow, kept counts and context lengths."""
+    dev = step.dH.device
+    ema = torch.zeros(w.B, dtype=torch.float32, device=dev)
+    pr = torch.empty(w.B, dtype=torch.float32, device=dev)
+    adm = torch.empty(w.B, dtype=torch.uint8, device=dev)
+    urg = torch.ones(w.B, dtype=torch.float32, device=dev)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+    for i in range(reps + 3):
+        if i >= 3:
+            ev[i - 3][0].record(stream)
+        eti.eti_schedule(step.dH, ema, w.B // 2, pr, adm, kept_cnt=step.kept_cnt, P=w.P,
+                         ctx_lens=kv["ctx_lens"], urgency=urg)
+        if i >= 3:
+            ev[i - 3][1].record(stream)
+    torch.cuda.synchronize()
+    return round(statistics.median(e[0].elapsed_time(e[1]) for e in ev), 5)
 
 
 def run_gpu(args):
@@ -326,6 +348,7 @@ def run_gpu(args):
     est = None
     if not args.no_estimators:
         est = run_estimators(eti, lg, step, prm, w, flush_l2, stream)
+        est["schedule_ms"] = run_schedule(eti, step, kv, w, stream)
 
     # end to end through the public API: host (pinned) inputs -> device -> step -> host results
     e2e = None if args.no_e2e else run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm,

@@ -215,6 +215,38 @@ int eti_entropy_temp_sample_noalloc(const float* logits, int B, int V, int64_t l
                                     uint32_t* err_flags, void* stream);
 
 /*
+ * Entropy-aware scheduling (Section 3.1): the priority
+ *   pi(s) = E[dH_s | S_t] / (alpha C_s + beta M_s + gamma L_s)
+ * with (the paper names the terms without formulas):
+ *   E[dH_s]  an exponential moving average of the irreversible entropy
+ *            reduction max(0, dH_s) that entropic time counts:
+ *            ema[s] <- lambda ema[s] + (1 - lambda) max(0, dH[s]) in place
+ *            (a NaN dH, an error row, leaves it unchanged);
+ *   C_s      attention work: kept tokens per kv head,
+ *            sum_h kept_cnt[s][h] * P / Hkv (0 when kept_cnt is NULL);
+ *   M_s      KV memory: ctx_lens[s] tokens (0 when NULL);
+ *   L_s      urgency[s], the caller's latency risk (0 when NULL);
+ * and the denominator floored at den_min.  The `budget` sequences of highest
+ * priority are admitted: admit_mask[s] = 1 (ties to the lower index, a NaN
+ * priority below every number; budget <= 0 admits none, >= B all).
+ * Parameters (defaults from eti_sched_defaults): lambda 0.9, alpha 1e-3,
+ * beta 1e-3 (per token), gamma 1, den_min 1e-6.  B <= 65535; one CTA.
+ */
+typedef struct {
+    float lambda;
+    float alpha;
+    float beta;
+    float gamma;
+    float den_min;
+} eti_sched_params;
+
+void eti_sched_defaults(eti_sched_params* p);
+
+int eti_schedule(const float* dH, float* ema, const int32_t* kept_cnt, int Hkv, int P,
+                 const int32_t* ctx_lens, const float* urgency, const eti_sched_params* params,
+                 int B, int budget, float* priority, uint8_t* admit_mask, void* stream);
+
+/*
  * eti_topk_entropy -- the top-k entropy estimators of Section 2.1, for each
  * row b with y = z / T_in[b] over the first V entries of row b of `logits`
  * (fp32, row stride ld >= V), p = softmax(y) and K the first min(k, V) tokens

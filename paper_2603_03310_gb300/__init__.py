@@ -32,7 +32,8 @@ SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_entropy_temp_sam
            "eti_score_prune_blocks", "eti_score_blocks", "eti_prune_blocks",
            "eti_paged_decode_workspace_size", "eti_paged_decode", "eti_version",
            "eti_status_string", "eti_entropy_temp_sample_noalloc",
-           "eti_entropy_temp_sample_noalloc_max_bytes", "eti_topk_entropy")
+           "eti_entropy_temp_sample_noalloc_max_bytes", "eti_topk_entropy", "eti_sched_defaults",
+           "eti_schedule")
 
 
 class EtiError(RuntimeError):
@@ -77,6 +78,10 @@ def load(path: str | None = None):
         lib.eti_entropy_temp_sample_noalloc.restype = i32
         lib.eti_entropy_temp_sample_noalloc_max_bytes.restype = sz
         lib.eti_entropy_temp_sample.restype = i32
+        lib.eti_sched_defaults.argtypes = [P]
+        lib.eti_sched_defaults.restype = None
+        lib.eti_schedule.argtypes = [P, P, P, i32, i32, P, P, P, i32, i32, P, P, P]
+        lib.eti_schedule.restype = i32
         lib.eti_topk_entropy.argtypes = [P, i32, i32, i64, P, i32, P, P, P, P, P]
         lib.eti_topk_entropy.restype = i32
         lib.eti_score_prune_workspace_size.argtypes = [i32] * 6
@@ -201,6 +206,35 @@ def eti_entropy_temp_sample_noalloc(logits, T_in, H_prev, tau, H_target, tok, H,
         _dev(tok_surprisal, "tok_surprisal", f32, B), _surp_store(surp_store, slot_mapping, B),
         _dev(err_flags, "err_flags", torch.int32, B), _stream(stream))
     _check(st, "eti_entropy_temp_sample_noalloc")
+
+
+class SchedParams(ctypes.Structure):
+    """eti_sched_params (include/eti.h)."""
+    _fields_ = [(n, ctypes.c_float) for n in ("lambda_", "alpha", "beta", "gamma", "den_min")]
+
+
+def sched_params(**kw) -> SchedParams:
+    """Scheduling parameters: the library defaults, overridden by keywords."""
+    p = SchedParams()
+    load().eti_sched_defaults(ctypes.byref(p))
+    for k, v in kw.items():
+        setattr(p, k, float(v))
+    return p
+
+
+def eti_schedule(dH, ema, budget: int, priority, admit_mask, kept_cnt=None, P: int = 16,
+                 ctx_lens=None, urgency=None, params: SchedParams | None = None, stream=None):
+    """Entropy-aware priority and admission (Section 3.1); see include/eti.h."""
+    B = dH.shape[0]
+    params = params or sched_params()
+    Hkv = kept_cnt.shape[1] if kept_cnt is not None else 1
+    f32, i32 = torch.float32, torch.int32
+    st = load().eti_schedule(
+        _dev(dH, "dH", f32, B), _dev(ema, "ema", f32, B), _dev(kept_cnt, "kept_cnt", i32, B * Hkv),
+        Hkv, int(P), _dev(ctx_lens, "ctx_lens", i32, B), _dev(urgency, "urgency", f32, B),
+        ctypes.byref(params), B, int(budget), _dev(priority, "priority", f32, B),
+        _dev(admit_mask, "admit_mask", torch.uint8, B), _stream(stream))
+    _check(st, "eti_schedule")
 
 
 def eti_topk_entropy(logits, T_in, k: int, H_tilde, H_hat, err_flags, tail_mass=None,

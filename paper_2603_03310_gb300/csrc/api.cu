@@ -14,6 +14,9 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
                                    const eti_surp_store* store, uint32_t* err, void* part,
                                    cudaStream_t stream);
 size_t eti_entropy_partial_bytes(int B);
+int eti_launch_schedule(const float* dH, float* ema, const int32_t* kept_cnt, int Hkv, int P,
+                        const int32_t* ctx_lens, const float* urgency, const eti_sched_params* p,
+                        int B, int budget, float* priority, uint8_t* admit, cudaStream_t stream);
 int eti_launch_topk_entropy(const float* logits, int B, int V, long long ld, const float* T_in,
                             int k, float* H_tilde, float* H_hat, float* tail_mass, uint32_t* err,
                             cudaStream_t stream);
@@ -190,6 +193,25 @@ int eti_topk_entropy(const float* logits, int B, int V, int64_t ld, const float*
     if (!logits || !T_in || !H_tilde || !H_hat || !err_flags) return ETI_ERR_NULL;
     return eti_launch_topk_entropy(logits, B, V, (long long)ld, T_in, k, H_tilde, H_hat, tail_mass,
                                    err_flags, (cudaStream_t)stream);
+}
+
+void eti_sched_defaults(eti_sched_params* p) {
+    if (!p) return;
+    p->lambda = 0.9f;
+    p->alpha = 1e-3f;
+    p->beta = 1e-3f;
+    p->gamma = 1.0f;
+    p->den_min = 1e-6f;
+}
+
+int eti_schedule(const float* dH, float* ema, const int32_t* kept_cnt, int Hkv, int P,
+                 const int32_t* ctx_lens, const float* urgency, const eti_sched_params* params,
+                 int B, int budget, float* priority, uint8_t* admit_mask, void* stream) {
+    if (B < 0 || B > 65535 || (kept_cnt && (Hkv < 1 || P < 1))) return ETI_ERR_SHAPE;
+    if (B == 0) return ETI_OK;
+    if (!dH || !ema || !params || !priority || !admit_mask) return ETI_ERR_NULL;
+    return eti_launch_schedule(dH, ema, kept_cnt, Hkv, P, ctx_lens, urgency, params, B, budget,
+                               priority, admit_mask, (cudaStream_t)stream);
 }
 
 size_t eti_score_prune_workspace_size(int B, int Hq, int Hkv, int D, int P, int max_blocks) {
