@@ -147,7 +147,7 @@ DEFAULT_SCHED = dict(lambda_=0.9, alpha=1e-3, beta=1e-3, gamma=1.0, den_min=1e-6
 
 def schedule(dH, ema_in, budget: int, kept_cnt=None, P: int = 16, ctx_lens=None, urgency=None,
              params=None) -> dict:
-    """Entropy-aware priority pi(s) and the admitted set (Section 3.1, reading R10).
+    """Entropy-aware priority pi(s) and the admitted set (Section 3.1, reading R14).
 
     dH, ema_in, urgency float32 [B]; kept_cnt int32 [B, Hkv]; ctx_lens int32 [B].
     """

@@ -32,12 +32,14 @@
  *   R7  keep iff score >= theta, or the block is among the first
  *       min(B_min, n_b) blocks ordered by (score desc, block index asc).
  *   R8  attention restricted to the kept blocks renormalises over them.
- *   R10 scheduling priority: E[dH_s] is an exponential moving average of
- *       max(0, dH_s); C_s, M_s, L_s are kept tokens, context length and a
- *       caller urgency (Section 3.1 names them without formulas).
- *   R9  the Section 5 guards: calibration rescales the logits by 1 / T_cal
+ *   R13 the Section 5 guards: calibration rescales the logits by 1 / T_cal
  *       before the step (entropy and draw use z / (T_cal T_t)); the rate
  *       limits bound |log T_{t+1} - log T_t| and |theta_{t+1} - theta_t|.
+ *   R14 scheduling priority: E[dH_s] is an exponential moving average of
+ *       max(0, dH_s); C_s, M_s, L_s are kept tokens, context length and a
+ *       caller urgency (Section 3.1 names them without formulas).
+ *   R16 top-k estimators: K is the first k tokens by (y desc, token id asc);
+ *       the tail mass is summed over the complement of K.
  */
 #include <math.h>
 #include <stdint.h>
@@ -145,7 +147,7 @@ typedef struct {
     double H_min;      /* entropy floor for pruning decisions (Section 5) */
     double theta_user; /* user threshold theta_t before the safety floor */
     double theta_hi;   /* scale of theta_max(H) */
-    double T_cal;      /* global calibration temperature (Section 5; reading R9) */
+    double T_cal;      /* global calibration temperature (Section 5; reading R13) */
     double rho_T;      /* bound on |log T_{t+1} - log T_t| per step, 0 = none (Section 5) */
     double dtheta;     /* bound on |theta_{t+1} - theta_t| per step, 0 = none (Section 5) */
 } oracle_ctrl;
@@ -161,7 +163,7 @@ typedef struct {
  *  theta_max(H) = theta_hi * max(0, 1 - H / log V)               (reading R6)
  *  tok       = argmax_x  z_x/T_t - log(-log u_x)                 (Gumbel-max draw from p)
  *  surprisal = -log p(tok)
- * Guards of Section 5 (reading R9): the logits are recalibrated by T_cal
+ * Guards of Section 5 (reading R13): the logits are recalibrated by T_cal
  * before everything above (p from z / (T_cal T_t)); the new temperature is
  * kept within a factor e^{rho_T} of T_t before the [T_min, T_max] clip; the
  * new threshold within dtheta of the previous one, theta_prev[b] (a finite
@@ -257,7 +259,7 @@ double oracle_entropy_row(const float *z, int64_t V, double T) {
 }
 
 /* ------------------------------------------------------------------------ */
-/* Entropy-aware scheduling priority and admission (Section 3.1, reading R10).
+/* Entropy-aware scheduling priority and admission (Section 3.1, reading R14).
  *
  *   E[dH_s] <- lambda E[dH_s] + (1 - lambda) max(0, dH_s)   (the expected
  *              irreversible entropy reduction, an exponential moving average of

@@ -682,7 +682,7 @@ def test_topk_entropy_error_rows():
 
 
 # ---------------------------------------------------------------------------
-# guards of Section 5 (reading R9): calibration and rate limits
+# guards of Section 5 (reading R13): calibration and rate limits
 
 def _guard_inputs(B=6, V=500, seed=7):
     rng = np.random.default_rng(seed)
@@ -757,7 +757,7 @@ def test_guard_threshold_rate_limit():
 
 
 # ---------------------------------------------------------------------------
-# entropy-aware scheduling priority (Section 3.1, reading R10)
+# entropy-aware scheduling priority (Section 3.1, reading R14)
 
 def test_schedule_limits_and_closed_forms():
     rng = np.random.default_rng(5)
