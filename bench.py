@@ -405,9 +405,19 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
     h_res = torch.empty((4, w.B), dtype=torch.float32).pin_memory()
     h_tok = torch.empty(w.B, dtype=torch.int32).pin_memory()
 
+    # The logits (the bulk of the bytes) go up on a copy stream while the
+    # attention half runs; the sampling call waits for them.  The attention
+    # output comes down on the copy stream while the sampling call runs.
+    main = torch.cuda.current_stream()
+    copy = torch.cuda.Stream(device=device)
+    ev_logits = torch.cuda.Event()
+    ev_out = torch.cuda.Event()
+
     def e2e_step(i):
+        with torch.cuda.stream(copy):
+            d_logits.copy_(h_logits, non_blocking=True)
+            ev_logits.record(copy)
         d_q.copy_(h_q, non_blocking=True)
-        d_logits.copy_(h_logits, non_blocking=True)
         d_state.copy_(h_state, non_blocking=True)
         T_in, H_prev, H_tgt, tau, th = d_state[0], d_state[1], d_state[2], d_state[3], d_state[4]
         eti.eti_score_blocks(d_q, kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
@@ -420,15 +430,20 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
                              kept_idx=step.kept_idx, kept_cnt=step.kept_cnt,
                              token_scores=step.token_scores, kept_norm=step.kept_norm,
                              num_pages=kv["num_pages"])
+        ev_out.record(main)
+        with torch.cuda.stream(copy):
+            copy.wait_event(ev_out)
+            h_out.copy_(step.out, non_blocking=True)
+        main.wait_event(ev_logits)
         step.sample(d_logits, T_in.contiguous(), H_prev.contiguous(), tau.contiguous(),
                     H_tgt.contiguous(), params=prm, seed=w.seed, offset=i)
-        h_out.copy_(step.out, non_blocking=True)
         h_tok.copy_(step.tok, non_blocking=True)
         h_res[0].copy_(step.H, non_blocking=True)
         h_res[1].copy_(step.T_out, non_blocking=True)
         h_res[2].copy_(step.theta_next, non_blocking=True)
         h_res[3].copy_(step.surprisal, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
+        main.synchronize()
+        copy.synchronize()
 
     for i in range(args.warmup):
         e2e_step(i)
