@@ -407,13 +407,17 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
 
     # The logits (the bulk of the bytes) go up on a copy stream while the
     # attention half runs; the sampling call waits for them.  The attention
-    # output comes down on the copy stream while the sampling call runs.
+    # output comes down on the copy stream while the sampling call runs.  The
+    # whole step (copies and calls, both streams) is captured once in a CUDA
+    # graph and replayed every step, as a serving loop would; if the capture
+    # is refused the same body runs eagerly.
     main = torch.cuda.current_stream()
     copy = torch.cuda.Stream(device=device)
     ev_logits = torch.cuda.Event()
     ev_out = torch.cuda.Event()
 
-    def e2e_step(i):
+    def body(i, cur):
+        copy.wait_stream(cur)                                  # fork
         with torch.cuda.stream(copy):
             d_logits.copy_(h_logits, non_blocking=True)
             ev_logits.record(copy)
@@ -430,11 +434,11 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
                              kept_idx=step.kept_idx, kept_cnt=step.kept_cnt,
                              token_scores=step.token_scores, kept_norm=step.kept_norm,
                              num_pages=kv["num_pages"])
-        ev_out.record(main)
+        ev_out.record(cur)
         with torch.cuda.stream(copy):
             copy.wait_event(ev_out)
             h_out.copy_(step.out, non_blocking=True)
-        main.wait_event(ev_logits)
+        cur.wait_event(ev_logits)
         step.sample(d_logits, T_in.contiguous(), H_prev.contiguous(), tau.contiguous(),
                     H_tgt.contiguous(), params=prm, seed=w.seed, offset=i)
         h_tok.copy_(step.tok, non_blocking=True)
@@ -442,21 +446,39 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
         h_res[1].copy_(step.T_out, non_blocking=True)
         h_res[2].copy_(step.theta_next, non_blocking=True)
         h_res[3].copy_(step.surprisal, non_blocking=True)
-        main.synchronize()
-        copy.synchronize()
+        cur.wait_stream(copy)                                  # join
 
     for i in range(args.warmup):
-        e2e_step(i)
+        body(i, main)
+        main.synchronize()
+    mode = "cuda graph replay (copies and calls of one step; fixed sampling offset)"
+    graph, gs = None, torch.cuda.Stream(device=device)
+    try:
+        gs.wait_stream(main)
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=gs):
+            body(args.warmup, gs)
+        graph.replay()
+        gs.synchronize()
+    except Exception as ex:                                    # capture refused: eager steps
+        graph = None
+        mode = f"eager (graph capture refused: {type(ex).__name__})"
+        torch.cuda.synchronize()
     times = []
     for i in range(args.steps):
         t0 = time.perf_counter()
-        e2e_step(i)
+        if graph is not None:
+            graph.replay()
+            gs.synchronize()
+        else:
+            body(args.warmup + i, main)
+            main.synchronize()
         times.append(time.perf_counter() - t0)
     s = statistics.mean(times)
     bi = h_q.numel() * 2 + h_logits.numel() * 4 + h_state.numel() * 4
     bo = h_out.numel() * 2 + h_tok.numel() * 4 + h_res.numel() * 4
     return {"value": round(w.B / s, 1), "unit": UNIT, "ms_per_step": round(s * 1e3, 4),
-            "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo)}
+            "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo), "mode": mode}
 
 
 # ---------------------------------------------------------------------------
