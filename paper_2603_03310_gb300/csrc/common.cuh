@@ -55,6 +55,13 @@ __device__ __forceinline__ float fast_ex2(float x) {
     return y;
 }
 
+// 1/x, hardware approximation (MUFU.RCP); 1/0 = +inf.
+__device__ __forceinline__ float fast_rcp(float x) {
+    float y;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 // log2(x), hardware approximation (MUFU.LG2).
 __device__ __forceinline__ float fast_lg2(float x) {
     float y;

@@ -4,20 +4,28 @@
 // threshold (Section 3.2 safety floor, Section 5 entropy floor) and a
 // Gumbel-max draw from p_t, in ONE pass over the fp32 logits.
 //
-// Decomposition: a persistent grid (4 CTAs per SM) in which every CTA takes an
-// equal contiguous share of the row-major list of all rows' 4-token groups,
-// so every SM finishes at the same time whatever B and V are.  Each CTA
-// streams its share with 128-bit loads (the next pair of groups is in flight
-// while the current pair is processed) and keeps, per thread, the online state
+// Decomposition: a persistent grid (4 CTAs of 256 threads per SM) in which
+// every CTA takes an equal contiguous share of the row-major list of all
+// rows' 4-token groups, so every SM finishes at the same time whatever B and
+// V are.  A CTA walks its share one row piece at a time, in steps of two
+// groups per thread (thread t takes groups base + 256 k + t, so its tokens are
+// visited in increasing index order), with the next step's 16-byte loads in
+// flight while the current one is processed.  Each thread keeps the online
+// state
 //     m  = running max of z (raw logit units), mc = m * c,  c = log2(e) / T
-//     S  = sum 2^{t},  t = z c - mc
+//     nt = number of tokens equal to m,  R = sum of 2^{t} over the others,
+//          t = z c - mc,  so that S = sum 2^{t} = nt 2^{t_max} + R
 //     U  = sum 2^{t} * t
 //     race best (r = w / E, index)  for the exponential race below.
 // t is formed with one fma against the rounded mc; that rounding shifts every
-// t of a state by the same amount and cancels exactly in H = ln2 (log2 S - U/S).
-// A CTA writes one partial state per row piece it covered to scratch slot
-// (cta + row); a finalize kernel merges each row's slots in CTA order (a fixed
-// order: results do not depend on timing) and writes the per-row outputs.
+// t of a state by the same amount and cancels exactly in H = ln S - ln2 U / S.
+// Keeping the tokens at the max out of R (one compare and two selects per
+// token) means a near-deterministic row (S = 1 + eps, eps down to 1e-6) keeps
+// eps to full fp32 precision however many tokens a thread sums: no small
+// weight is ever added to a value near 1.  A CTA writes one partial state per
+// row piece it covered to scratch slot (cta + row); a finalize kernel merges
+// each row's slots in CTA order (a fixed order: results do not depend on
+// timing) and writes the per-row outputs.
 //
 // Sampling.  argmax_x y_x - log(-log u_x) is argmax_x w_x / E_x with
 // w_x = exp(y_x - m) and the exponential variate E_x = -log u_x, so the
@@ -30,6 +38,28 @@
 //                the Taylor series of -log(1 - v), whose remainder is below
 //                v^6/7 < 2^-24 / 7 relative.
 // u = (2 (word & 0x7FFFFF) + 1) / 2^24 is formed exactly as 1.m - (1 - 2^-24).
+//
+// Race prefilter.  -log u >= 1 - u, so E2 >= log2(e) v with v = 1 - u, and
+// both evaluations of E2 above stay within 2^-18 (relative) of the true
+// value; a token with w <= rk v, rk = r_lb log2(e) (1 - 2^-16), therefore has
+// w / E2 below r_lb by at least 2^-17 relative and cannot win, where r_lb is
+// any ratio already reached in this row.  Only the tokens that pass evaluate
+// E2 (out of line, in race_group), so the draw is unchanged.  The bound is
+// shared by the whole CTA for its row piece: a thread that reaches a new best
+// publishes lr = log2 r + mc (the ratio in the row's common frame) with a
+// shared-memory atomicMax on the order-preserving key of lr, and every thread
+// folds the published bound into its rk once per step, 2^-10 shaved off for
+// the rounding of lr and of its conversion back.  Before the piece's first
+// race every thread seeds the bound with the exact ratio of its own max token
+// of the first step (one barrier), so that on the benchmark logits only a few
+// dozen tokens per CTA piece reach the exact evaluation.  The test is
+// evaluated as
+//     1.f(~word) < w / rk + (1 - 2^-24) + 2^-21,
+// the left side 1 + v - 2^-24 built from the word's bits with one logic op,
+// the right side one fma against 1/rk.  The 2^-21 slack covers the rounding
+// of the fma and of 1/rk (for w / rk <= 1.6; every token with w / rk > 1
+// passes anyway), so no token that passes w > rk v is rejected; the slack
+// also lets through the tokens with v within 2^-21 of w / rk.
 #include <mutex>
 
 #include "common.cuh"
@@ -66,83 +96,117 @@ __device__ __forceinline__ float exp_variate_log2(uint32_t word) {
     return u > 0.9375f ? series : direct;
 }
 
+// Partial state of a row (piece), 24 bytes.  The frame product mc = m c is
+// not stored: it is recomputed from m and the row's c (always the same
+// rounding) wherever it is needed.
+//   m   max logit seen (raw units); -inf when empty
+//   nt  number of tokens equal to m, each of weight 2^{t_max}, t_max = m c - mc
+//   R   sum of 2^t over the other tokens (t = z c - mc)
+//   U   sum of 2^t t over all tokens
+//   r   race best: w / E in this frame (0 = none);  bi: its token (INT_MAX = none)
+// Keeping the tokens at the max out of R means a near-deterministic row
+// (S = 1 + eps, eps down to 1e-6) keeps eps to full fp32 precision: no small
+// weight is ever added to a value near 1.
 struct RowState {
-    float m;    // max logit seen (raw units)
-    float mc;   // m * c, rounded once
-    float S;    // sum 2^t
-    float U;    // sum 2^t * t
-    float r;    // race best: w / E relative to m (0 = none)
-    int bi;     // race best: token index (INT_MAX = none)
+    float m, nt, R, U, r;
+    int bi;
 };
 
 __device__ __forceinline__ void state_init(RowState& s) {
-    s.m = -kInf; s.mc = -kInf; s.S = 0.f; s.U = 0.f; s.r = 0.f; s.bi = 0x7fffffff;
+    s.m = -kInf; s.nt = 0.f; s.R = 0.f; s.U = 0.f; s.r = 0.f; s.bi = 0x7fffffff;
 }
 
-// Move the state to a new, larger reference max `nm`; returns the factor
-// 2^{mc_old - mc_new} by which every term of the state was scaled.
-__device__ __forceinline__ float state_rebase(RowState& s, float nm, float c) {
+// The state's S = sum 2^t in its own frame.
+__device__ __forceinline__ float state_sum(const RowState& s, float c, float mc) {
+    return fmaf(s.nt, fast_ex2(fmaf(s.m, c, -mc)), s.R);
+}
+
+// Move a thread's state to a new, larger max `nm` (its frame product in
+// `mc`); the tokens at the old max become ordinary terms.  Returns the factor
+// 2^{mc_old - mc_new} by which every earlier term was scaled.
+__device__ __forceinline__ float state_rebase(RowState& s, float& mc, float nm, float c) {
     const float nmc = nm * c;
-    float a = 0.f, d = 0.f;
+    float a = 0.f, d = 0.f, S = 0.f;
     if (s.m != -kInf) {
-        d = s.mc - nmc;              // t_new = t_old + d for every term of the state
+        d = mc - nmc;                            // t_new = t_old + d for every earlier term
         a = fast_ex2(d);
+        S = state_sum(s, c, mc);
     }
-    s.U = a * fmaf(d, s.S, s.U);
-    s.S *= a;
+    s.U = a * fmaf(d, S, s.U);
+    s.R = S * a;
+    s.nt = 0.f;
     s.r *= a;
     s.m = nm;
-    s.mc = nmc;
+    mc = nmc;
     return a;
 }
 
-// Merge partial `o` into `s` (both may be empty).
+// Merge partial `o` into `s` (both may be empty; c is the row's log2(e)/T):
+// the state with the lower max is scaled into the other's frame, where all of
+// its tokens are ordinary terms; equal maxima share the frame.
 __device__ __forceinline__ void state_merge(RowState& s, RowState o, float c) {
     if (o.m == -kInf) return;
     if (s.m == -kInf) { s = o; return; }
-    if (o.m > s.m) {
-        state_rebase(s, o.m, c);
-        // align o to the same rounded reference
-        const float d = o.mc - s.mc;
-        const float a = fast_ex2(d);
-        o.U = a * fmaf(d, o.S, o.U); o.S *= a; o.r *= a;
+    if (o.m > s.m) { const RowState t = s; s = o; o = t; }
+    float orr = o.r;
+    if (o.m == s.m) {
+        s.nt += o.nt;
+        s.R += o.R;
+        s.U += o.U;
     } else {
-        const float d = o.mc - s.mc;
+        const float smc = s.m * c, omc = o.m * c;
+        const float d = omc - smc;               // < 0
         const float a = fast_ex2(d);
-        o.U = a * fmaf(d, o.S, o.U); o.S *= a; o.r *= a;
+        const float So = state_sum(o, c, omc);
+        s.U += a * fmaf(d, So, o.U);
+        s.R = fmaf(So, a, s.R);
+        orr *= a;
     }
-    s.S += o.S;
-    s.U += o.U;
-    if (o.r > s.r || (o.r == s.r && o.bi < s.bi)) { s.r = o.r; s.bi = o.bi; }
+    if (orr > s.r || (orr == s.r && o.bi < s.bi)) { s.r = orr; s.bi = o.bi; }
 }
 
 __device__ __forceinline__ RowState state_shfl_xor(const RowState& s, int o) {
     RowState r;
     r.m = __shfl_xor_sync(0xffffffffu, s.m, o);
-    r.mc = __shfl_xor_sync(0xffffffffu, s.mc, o);
-    r.S = __shfl_xor_sync(0xffffffffu, s.S, o);
+    r.nt = __shfl_xor_sync(0xffffffffu, s.nt, o);
+    r.R = __shfl_xor_sync(0xffffffffu, s.R, o);
     r.U = __shfl_xor_sync(0xffffffffu, s.U, o);
     r.r = __shfl_xor_sync(0xffffffffu, s.r, o);
     r.bi = __shfl_xor_sync(0xffffffffu, s.bi, o);
     return r;
 }
 
-// Race prefilter.  -log u >= 1 - u, so E2 >= log2(e) v with v = 1 - u, and
-// both evaluations of E2 above stay within 2^-18 (relative) of the true
-// value; a token with w <= rk v, rk = r_lb log2(e) (1 - 2^-16), therefore has
-// w / E2 below r_lb by at least 2^-17 relative and cannot win, where r_lb is
-// any ratio already reached in this row (own best, or a bound shared by the
-// warp).  Only the tokens that pass evaluate E2, so the draw is unchanged.
 constexpr float kRaceKappa = 1.4426950408889634f * (1.0f - 1.0f / 65536.0f);
+constexpr float kPassC = 1.000000476837158203125f;    // 1 + 2^-21 >= (1 - 2^-24) + 2^-21 - rounding
 
-// v = 1 - u = (2 (0x7FFFFF - j) + 1) 2^-24 for the word's uniform u, formed exactly
-__device__ __forceinline__ float one_minus_u(uint32_t word) {
-    return __uint_as_float((~word & 0x7FFFFFu) | 0x3F800000u) - __uint_as_float(0x3F7FFFFFu);
+// The exact race over one 4-token group (tokens x0 .. x0 + 3 in order) for the
+// tokens that pass the prefilter against 1/rk = ir.  Kept out of line: it
+// runs for a handful of groups per row piece, and inlined it would cost the
+// straight path its registers and issue slots.
+struct RaceUpd {
+    float r, rk;
+    int bi, pub;
+};
+__device__ __noinline__ RaceUpd race_group(float4 w4, uint4 wd4, float ir, float r, int bi, float rk, int x0) {
+    RaceUpd u{r, rk, bi, 0};
+    const float w[4] = {w4.x, w4.y, w4.z, w4.w};
+    const uint32_t wd[4] = {wd4.x, wd4.y, wd4.z, wd4.w};
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        const float fv = __uint_as_float((~wd[e] & 0x7FFFFFu) | 0x3F800000u);
+        if (fv < fmaf(w[e], ir, kPassC)) {
+            const float E = exp_variate_log2(wd[e]);
+            if (w[e] > u.r * E) {
+                u.r = __fdividef(w[e], E);
+                u.bi = x0 + e;
+                u.rk = fmaxf(u.rk, fminf(u.r * kRaceKappa, 1e38f));
+                ir = fast_rcp(u.rk);
+                u.pub = 1;
+            }
+        }
+    }
+    return u;
 }
-
-constexpr int kEtsThreads = 256;
-constexpr int kEtsPair = 2;     // 4-token groups per thread per pipeline step
-constexpr int kEtsCtasPerSm = 4;
 
 struct EtsArgs {
     const float* logits;
@@ -167,14 +231,28 @@ struct EtsArgs {
     long long num_slots;
     uint32_t* err;
     int ngroups;          // 4-token groups per row
-    long long share;      // groups per CTA of the persistent grid
-    RowState* part;       // [nCTA + B] partial states, slot (cta + row)
+    long long share;      // groups per CTA of the grid
+    RowState* part;       // [grid + B] partial states, slot (cta + row)
 };
+
+constexpr int kEtsThreads = 256;
+constexpr int kEtsWarps = kEtsThreads / 32;
+constexpr int kEtsPair = 2;        // 4-token groups per thread per step
+constexpr int kEtsCtasPerSm = 4;
+constexpr float kFrameMax = 4096.f;   // |mc| above which lr loses the 2^-10 margin
+
+// order-preserving int key of a float (and back); key(-inf) marks "no bound"
+__device__ __forceinline__ int bound_key(float f) {
+    const int b = __float_as_int(f);
+    return b ^ ((b >> 31) & 0x7fffffff);
+}
+__device__ __forceinline__ float bound_unkey(int k) { return __int_as_float(k ^ ((k >> 31) & 0x7fffffff)); }
+constexpr int kNoBound = (int)0x807fffff;   // bound_key(-inf)
 
 template <bool kVec>
 __device__ __forceinline__ void load_group(float (&z)[4], const float* row, int g, int g1, int full_groups,
                                            int V) {
-    if (g < g1 && kVec && g < full_groups) {
+    if (kVec && g < g1 && g < full_groups) {
         const float4 v = ldg_stream_f4(row + 4 * (long long)g);
         z[0] = v.x; z[1] = v.y; z[2] = v.z; z[3] = v.w;
     } else {
@@ -186,19 +264,24 @@ __device__ __forceinline__ void load_group(float (&z)[4], const float* row, int 
     }
 }
 
-// Persistent pass: CTA c takes groups [c*share, (c+1)*share) of the
-// row-major list of all rows' 4-token groups, one row piece at a time.
+// The pass over the logits: CTA c takes groups [c*share, (c+1)*share) of the
+// row-major list of all rows' 4-token groups, one row piece at a time; a
+// piece is walked in steps of kEtsPair groups per thread (thread t takes
+// groups base + k * 256 + t), the next step's 16-byte loads in flight while
+// the current one is processed.
 template <bool kVec>
 __global__ void __launch_bounds__(kEtsThreads, kEtsCtasPerSm)
 entropy_sample_partial_kernel(const __grid_constant__ EtsArgs a) {
     pdl_trigger();
     pdl_wait();
-    __shared__ RowState warp_part[kEtsThreads / 32];
-    const int tid = threadIdx.x;
+    __shared__ RowState warp_part[kEtsWarps];
+    __shared__ int bound;   // the piece's race bound: key of the best lr, or kNoBound
+    const int tid = threadIdx.x, lane = tid & 31;
     const long long total = (long long)a.B * a.ngroups;
     long long q0 = (long long)blockIdx.x * a.share;
     const long long q1 = min(q0 + a.share, total);
     const int full_groups = a.V >> 2;
+    constexpr int step = kEtsPair * kEtsThreads;
     while (q0 < q1) {
         const int b = (int)(q0 / a.ngroups);
         const int g0 = (int)(q0 - (long long)b * a.ngroups);
@@ -207,89 +290,110 @@ entropy_sample_partial_kernel(const __grid_constant__ EtsArgs a) {
         const bool bad_T = !(T > 0.f && T < kInf);
         const float c = bad_T ? 0.f : kLog2e / T;
         const float* row = a.logits + (long long)b * a.ld;
+        if (tid == 0) bound = kNoBound;
+        __syncthreads();
         RowState s;
         state_init(s);
-        float rk = 0.f;              // race prefilter bound, in the state's frame
-        bool shared = false;         // the warp's bound has been folded into rk
-        // every lane of the warp walks this row piece (the same steps), so the
-        // warp may exchange its bound with full-mask shuffles
-        const bool warp_full = g0 + (tid | 31) < g1;
-        if (!bad_T && g0 + tid < g1) {
-            constexpr int step = kEtsPair * kEtsThreads;
+        float mc = -kInf, rk = 0.f, ir = kInf;
+        int seen = kNoBound;
+        if (!bad_T) {
+            const int nsteps = (g1 - g0 + step - 1) / step;   // the same for every thread
             float cur[kEtsPair][4], nxt[kEtsPair][4];
 #pragma unroll
             for (int k = 0; k < kEtsPair; ++k) load_group<kVec>(cur[k], row, g0 + k * kEtsThreads + tid, g1, full_groups, a.V);
-            for (int base = g0; base < g1; base += step) {
-                const bool more = base + step < g1;
-                if (more) {
+            for (int it = 0; it < nsteps; ++it) {
+                const int base = g0 + it * step;
+                if (it + 1 < nsteps) {
 #pragma unroll
                     for (int k = 0; k < kEtsPair; ++k)
                         load_group<kVec>(nxt[k], row, base + step + k * kEtsThreads + tid, g1, full_groups, a.V);
                 }
+                // random words of this step's groups, in one straight block so
+                // that the Philox chains (independent of the state) interleave
+                uint4 rr[kEtsPair];
+#pragma unroll
+                for (int k = 0; k < kEtsPair; ++k)
+                    rr[k] = philox4x32_10(make_uint4((uint32_t)(base + k * kEtsThreads + tid), (uint32_t)b,
+                                                     a.off_lo, a.off_hi), a.rk0, a.rk1);
                 float bm = -kInf;
 #pragma unroll
                 for (int k = 0; k < kEtsPair; ++k)
 #pragma unroll
                     for (int e = 0; e < 4; ++e) bm = fmaxf(bm, cur[k][e]);
-                if (bm == -kInf) {
-                    // every token of the pair is -inf (or NaN): nothing to add and
-                    // nothing to draw, but a NaN must still poison the row
+                if (bm > s.m) {
+                    rk *= state_rebase(s, mc, bm, c);
+                    ir = fast_rcp(rk);
+                }
+                if (it == 0) {
+                    // Seed the piece's race bound before its first race: each
+                    // thread evaluates exactly the ratio of its max token of the
+                    // step (a real token, so a lower bound of the row's best)
+                    // and the CTA keeps the largest.
+                    if (s.m != -kInf && s.m < kInf && fabsf(mc) < kFrameMax) {
+                        uint32_t wd = 0;
+                        bool found = false;
+#pragma unroll
+                        for (int k = 0; k < kEtsPair; ++k) {
+                            const uint32_t w4[4] = {rr[k].x, rr[k].y, rr[k].z, rr[k].w};
+#pragma unroll
+                            for (int e = 0; e < 4; ++e)
+                                if (!found && cur[k][e] == s.m) { wd = w4[e]; found = true; }
+                        }
+                        const float r0 = __fdividef(fast_ex2(fmaf(s.m, c, -mc)), exp_variate_log2(wd));
+                        atomicMax(&bound, bound_key(fast_lg2(r0) + mc));
+                    }
+                    __syncthreads();
+                }
+                if (s.m == -kInf) {
+                    // no finite token yet: nothing to add or draw, but a NaN
+                    // must still poison the row
                     bool nan = false;
 #pragma unroll
                     for (int k = 0; k < kEtsPair; ++k)
 #pragma unroll
-                        for (int e = 0; e < 4; ++e) nan |= (cur[k][e] != cur[k][e]);
-                    if (nan) s.S = __int_as_float(0x7fc00000);
+                        for (int e = 0; e < 4; ++e) nan |= cur[k][e] != cur[k][e];
+                    if (nan) s.R = __int_as_float(0x7fc00000);
                 } else {
-                    if (bm > s.m) rk *= state_rebase(s, bm, c);
-                    // entropy sums for every token, the race prefilter folded into
-                    // one flag; groups past the piece hold -inf (w = 0, never drawn)
-                    float w[kEtsPair][4];
-                    uint32_t word[kEtsPair][4];
-                    bool any = false;
-#pragma unroll
-                    for (int k = 0; k < kEtsPair; ++k) {
-                        const int g = base + k * kEtsThreads + tid;
-                        const uint4 r = philox4x32_10(make_uint4((uint32_t)g, (uint32_t)b, a.off_lo, a.off_hi), a.rk0, a.rk1);
-                        word[k][0] = r.x; word[k][1] = r.y; word[k][2] = r.z; word[k][3] = r.w;
-#pragma unroll
-                        for (int e = 0; e < 4; ++e) {
-                            const float t = fmaf(cur[k][e], c, -s.mc);
-                            w[k][e] = fast_ex2(t);
-                            s.S += w[k][e];
-                            s.U = fmaf(w[k][e], fmaxf(t, -250.f), s.U);   // -inf adds 0; NaN reaches S
-                            any |= w[k][e] > rk * one_minus_u(word[k][e]);
+                    const int kb = *(volatile int*)&bound;
+                    if (kb != seen) {
+                        seen = kb;
+                        if (fabsf(mc) < kFrameMax) {
+                            const float rkb = fminf(fast_ex2(bound_unkey(kb) - mc - 0.0009765625f) * kRaceKappa, 1e38f);
+                            if (rkb > rk) {
+                                rk = rkb;
+                                ir = fast_rcp(rk);
+                            }
                         }
                     }
-                    if (any) {
-                        // rare once rk has grown: the exact race, in token order
 #pragma unroll
-                        for (int k = 0; k < kEtsPair; ++k)
+                    for (int k = 0; k < kEtsPair; ++k) {
+                        float w[4];
+                        const uint32_t wd[4] = {rr[k].x, rr[k].y, rr[k].z, rr[k].w};
+                        bool any = false;
 #pragma unroll
-                            for (int e = 0; e < 4; ++e)
-                                if (w[k][e] > rk * one_minus_u(word[k][e])) {
-                                    const float E = exp_variate_log2(word[k][e]);
-                                    if (w[k][e] > s.r * E) {
-                                        s.r = __fdividef(w[k][e], E);
-                                        s.bi = 4 * (base + k * kEtsThreads + tid) + e;
-                                        rk = fmaxf(rk, s.r * kRaceKappa);
-                                    }
-                                }
+                        for (int e = 0; e < 4; ++e) {
+                            const float t = fmaf(cur[k][e], c, -mc);
+                            w[e] = fast_ex2(t);
+                            s.U = fmaf(w[e], fmaxf(t, -250.f), s.U);   // -inf adds 0; NaN reaches U
+                            const bool at_max = cur[k][e] == s.m;      // the tokens at the max stay out of R
+                            s.nt += at_max ? 1.f : 0.f;
+                            s.R += at_max ? 0.f : w[e];                 // (a NaN lands here)
+                            const float fv = __uint_as_float((~wd[e] & 0x7FFFFFu) | 0x3F800000u);
+                            any |= fv < fmaf(w[e], ir, kPassC);
+                        }
+                        if (any) {
+                            // rare once the bound has formed: the exact race, in token order
+                            const RaceUpd u = race_group(make_float4(w[0], w[1], w[2], w[3]), rr[k], ir, s.r, s.bi,
+                                                         rk, 4 * (base + k * kEtsThreads + tid));
+                            if (u.pub) {
+                                s.r = u.r;
+                                s.bi = u.bi;
+                                rk = u.rk;
+                                ir = fast_rcp(rk);
+                                if (fabsf(mc) < kFrameMax) atomicMax(&bound, bound_key(fast_lg2(s.r) + mc));
+                            }
+                        }
                     }
-                }
-                if (!more) break;
-                if (!shared && warp_full) {
-                    // After the first step, share the best ratio of the warp as
-                    // a bound: lr = log2 r + mc is the ratio in the row's common
-                    // frame, and the 2^-10 shaved off covers the rounding of
-                    // lr and of its conversion back to this state's frame.  The
-                    // cap keeps rk finite, so a later rebase by 0 gives 0.
-                    shared = true;
-                    float lr = s.r > 0.f ? fast_lg2(s.r) + s.mc : -kInf;
-#pragma unroll
-                    for (int o = 16; o > 0; o >>= 1) lr = fmaxf(lr, __shfl_xor_sync(0xffffffffu, lr, o));
-                    if (lr > -kInf && s.m != -kInf)
-                        rk = fmaxf(rk, fminf(fast_ex2(lr - s.mc - 0.0009765625f) * kRaceKappa, 1e38f));
                 }
 #pragma unroll
                 for (int k = 0; k < kEtsPair; ++k)
@@ -297,17 +401,16 @@ entropy_sample_partial_kernel(const __grid_constant__ EtsArgs a) {
                     for (int e = 0; e < 4; ++e) cur[k][e] = nxt[k][e];
             }
         }
-        // CTA reduction of the piece into slot (cta + row)
+        // CTA reduction of the piece into slot (cta + row), in a fixed order
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) state_merge(s, state_shfl_xor(s, o), c);
-        if ((tid & 31) == 0) warp_part[tid >> 5] = s;
+        if (lane == 0) warp_part[tid >> 5] = s;
         __syncthreads();
         if (tid == 0) {
             RowState t = warp_part[0];
-            for (int w = 1; w < kEtsThreads / 32; ++w) state_merge(t, warp_part[w], c);
+            for (int w = 1; w < kEtsWarps; ++w) state_merge(t, warp_part[w], c);
             a.part[blockIdx.x + b] = t;
         }
-        __syncthreads();
         q0 = (long long)b * a.ngroups + g1;
     }
 }
@@ -334,7 +437,7 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
         RowState o2 = state_shfl_xor(s, o);
-        // keep the lower-lane state first so ties resolve to the lower index
+        // keep the lower-lane state first (a fixed order of the sums)
         if (lane & o) { RowState t = o2; o2 = s; s = t; }
         state_merge(s, o2, c);
     }
@@ -344,7 +447,7 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
     uint32_t err = bad_T ? ETI_ERRF_BAD_TEMP : 0u;
     if (!err) {
         if (t.m == -kInf) err = ETI_ERRF_ALL_NEG_INF;
-        else if (t.m == kInf || isnan(t.S) || isnan(t.U)) err = ETI_ERRF_NONFINITE;
+        else if (t.m == kInf || isnan(t.R) || isnan(t.U)) err = ETI_ERRF_NONFINITE;
     }
     const float tau_in = a.tau[b];
     if (err) {
@@ -355,8 +458,12 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
         if (a.theta_next) a.theta_next[b] = 0.f;
         if (a.surprisal) a.surprisal[b] = __int_as_float(0x7fc00000);
     } else {
-        const float l2S = log2f(t.S);
-        const float H = fmaxf(kLn2 * (l2S - t.U / t.S), 0.f);
+        // S = nt 2^{t_max} + R with |t_max| < 2^-10, so 2^{t_max} = 1 + t_max ln2
+        // to well below fp32 precision; ln S = ln nt + log1p(q), q = S / nt - 1
+        const float mc = t.m * c;
+        const float q = fmaf(t.nt, fmaf(t.m, c, -mc) * kLn2, t.R) / t.nt;
+        const float lnS = logf(t.nt) + log1pf(q);
+        const float H = fmaxf(lnS - kLn2 * t.U / (t.nt * (1.f + q)), 0.f);
         const float dH = a.H_prev[b] - H;
         a.tau[b] = tau_in + fmaxf(dH, 0.f);
         float Tn = Tt * expf(a.p.sign * a.p.eta * (H - a.H_target[b]));
@@ -378,8 +485,8 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
             a.theta_next[b] = th;
         }
         if (a.surprisal || a.surp_store) {
-            const float tt = fmaf(row[t.bi], c, -t.mc);
-            const float sp = kLn2 * (l2S - tt);
+            const float tt = fmaf(row[t.bi], c, -mc);
+            const float sp = lnS - kLn2 * tt;
             if (a.surprisal) a.surprisal[b] = sp;
             if (a.surp_store) {
                 const long long slot = a.slot_mapping[b];
@@ -432,8 +539,8 @@ int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long 
     a.num_slots = store ? (long long)store->num_slots : 0;
     a.ngroups = (V + 3) / 4;
     const long long total = (long long)B * a.ngroups;
-    a.share = (total + ncta - 1) / ncta;
     a.part = static_cast<RowState*>(part);
+    a.share = (total + ncta - 1) / ncta;
     const bool vec = (ld % 4 == 0) && ((reinterpret_cast<uintptr_t>(logits) & 15) == 0);
     const cudaError_t e1 = vec ? eti_launch_pdl(entropy_sample_partial_kernel<true>, dim3(ncta), dim3(kEtsThreads), 0, stream, a)
                                : eti_launch_pdl(entropy_sample_partial_kernel<false>, dim3(ncta), dim3(kEtsThreads), 0, stream, a);
