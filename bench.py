@@ -220,6 +220,91 @@ def run_schedule(eti, step, kv, w, stream, reps=50):
     return round(statistics.median(e[0].elapsed_time(e[1]) for e in ev), 5)
 
 
+def run_keep_sweep(eti, device, flush_l2, stream, peak, fracs=(0.1, 0.25, 0.5, 1.0), reps=10):
+    """The long-context step of the paper's sweep (8 sequences, contexts
+    U[32768, 131072]): theta = +inf and B_min = ceil(f * n_b) of the longest
+    sequence, so every sequence keeps its min(B_min, n_b) best blocks.  The
+    decode reads only the kept blocks: its time against the kept fraction is
+    the saving the method buys; the scorer's full read of K is the fixed cost
+    of the rule.  Median of `reps` calls, L2 flushed before each."""
+    w = workloads.WORKLOADS["long_ctx"]
+    kv = workloads.make_kv(w, device)
+    g = w.Hq // w.Hkv
+    st = eti.DecodeStep(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, w.V, device=device)
+    stats = torch.empty((w.B, w.Hkv, w.max_blocks, g, 4), dtype=torch.float32, device=device)
+    shape = (w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks)
+    theta = torch.full((w.B,), float("inf"), dtype=torch.float32, device=device)
+    L = kv["ctx_lens"].cpu().numpy()
+    nb = -(-L // w.P)
+    total = int(nb.sum()) * w.Hkv
+
+    def timed(fn):
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+        for i in range(reps + 2):
+            flush_l2()
+            if i >= 2:
+                ev[i - 2][0].record(stream)
+            fn()
+            if i >= 2:
+                ev[i - 2][1].record(stream)
+        torch.cuda.synchronize()
+        return statistics.median(e[0].elapsed_time(e[1]) for e in ev)
+
+    def score():
+        eti.eti_score_blocks(kv["q"], kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
+                             stats, token_scores=st.token_scores, num_pages=kv["num_pages"])
+
+    def decode():
+        eti.eti_paged_decode(kv["q"], kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
+                             kv["scale"], st.out, st.err_dec, st.ws_dec, kept_idx=st.kept_idx,
+                             kept_cnt=st.kept_cnt, token_scores=st.token_scores,
+                             kept_norm=st.kept_norm, num_pages=kv["num_pages"])
+
+    score_ms = timed(score)
+    # the baseline the rule is measured against: dense decode over every block
+    # (q.K and p.V in one pass, K and V of every block read once)
+    ws_dense = torch.empty(eti.paged_decode_workspace_size(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, False),
+                           dtype=torch.uint8, device=device)
+    out_dense = torch.empty_like(st.out)
+
+    def dense():
+        eti.eti_paged_decode(kv["q"], kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
+                             kv["scale"], out_dense, st.err_dec, ws_dense, num_pages=kv["num_pages"])
+
+    dense_ms = timed(dense)
+    kv_bytes = int(L.sum()) * w.Hkv * w.D * 2 * 2 + 2 * w.B * w.Hq * w.D * 2
+    points = []
+    for f in fracs:
+        B_min = int(math.ceil(f * int(nb.max())))
+
+        def prune():
+            eti.eti_prune_blocks(stats, kv["block_table"], kv["ctx_lens"], shape, theta, B_min, st.keep_mask,
+                                 st.kept_idx, st.kept_cnt, st.err_attn, kept_norm=st.kept_norm,
+                                 num_pages=kv["num_pages"])
+
+        prune_ms = timed(prune)
+        kept = int(st.kept_cnt.sum().item())
+        ms = timed(decode)
+        byt = algorithmic_bytes(w, L, kept)["decode"]
+        step_ms = score_ms + prune_ms + ms
+        points.append({"f": f, "B_min": B_min, "kept_fraction": round(kept / total, 4),
+                       "decode_ms": round(ms, 5), "decode_gbs": round(byt / (ms / 1e3) / 1e9, 1),
+                       "frac": round(byt / (ms / 1e3) / 1e9 / peak, 4), "prune_ms": round(prune_ms, 5),
+                       "attention_ms": round(step_ms, 5), "speedup_vs_dense": round(dense_ms / step_ms, 3)})
+    sbytes = algorithmic_bytes(w, L, 0)["score"]
+    del kv, st, stats, ws_dense, out_dense
+    torch.cuda.empty_cache()
+    return {"workload": f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} D={w.D} P={w.P} "
+                        f"ctx U[{w.ctx[1]},{w.ctx[2]}]",
+            "theta": "+inf", "score_ms": round(score_ms, 5),
+            "score_gbs": round(sbytes / (score_ms / 1e3) / 1e9, 1),
+            "dense_decode_ms": round(dense_ms, 5),
+            "dense_decode_gbs": round(kv_bytes / (dense_ms / 1e3) / 1e9, 1), "points": points,
+            "note": "decode over the kept blocks only (kept V pages + their scores); the scorer "
+                    "reads every key whatever f is; attention_ms = score + prune + decode, against "
+                    "a dense decode that reads K and V of every block"}
+
+
 def run_gpu(args):
     import paper_2603_03310_gb300 as eti
 
@@ -350,6 +435,8 @@ def run_gpu(args):
         est = run_estimators(eti, lg, step, prm, w, flush_l2, stream)
         est["schedule_ms"] = run_schedule(eti, step, kv, w, stream)
 
+    sweep = None if args.no_sweep else run_keep_sweep(eti, device, flush_l2, stream, peak)
+
     # end to end through the public API: host (pinned) inputs -> device -> step -> host results
     e2e = None if args.no_e2e else run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm,
                                            args, device)
@@ -380,6 +467,7 @@ def run_gpu(args):
                               "memset (error flags, not a kernel of the library)": 1},
         "e2e": e2e,
         "estimators": est,
+        "keep_sweep": sweep,
         "wall_s_timed_region": round(wall, 4),
         "clocks": clk.summary(),
     }
@@ -578,6 +666,8 @@ def main(argv=None):
                     help="seconds of oracle work for the CPU baseline")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true", help="skip the host-buffer end-to-end leg")
+    ap.add_argument("--no-sweep", action="store_true",
+                    help="skip the long-context keep-fraction sweep (decode time against kept blocks)")
     ap.add_argument("--no-estimators", action="store_true",
                     help="skip the top-k entropy estimator line")
     ap.add_argument("--traffic", type=float, default=None,

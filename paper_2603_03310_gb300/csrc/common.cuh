@@ -229,6 +229,16 @@ __device__ __forceinline__ int warp_sum_i(int v) {
     return v;
 }
 
+// hist[bin] += 1 for every lane with `on`, one shared-memory atomic per
+// distinct bin of the warp (every lane of the warp must call it together)
+__device__ __forceinline__ void warp_hist_add(int* hist, uint32_t bin, bool on) {
+    const uint32_t act = __ballot_sync(0xffffffffu, on);
+    if (on) {
+        const uint32_t peers = __match_any_sync(act, bin);
+        if ((threadIdx.x & 31) == (uint32_t)(__ffs(peers) - 1)) atomicAdd(hist + bin, __popc(peers));
+    }
+}
+
 __host__ __device__ __forceinline__ int ceil_div(int a, int b) { return (a + b - 1) / b; }
 
 // Blocks of a sequence with context length L (0 for an invalid length, which

@@ -267,6 +267,8 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
         float4 v[kM];
 #pragma unroll
         for (int k = 0; k < kM; ++k) v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+        // four slots' loads in flight at a time (the sums wait on L2 latency)
+#pragma unroll 4
         for (int w = 0; w < nw; ++w) {
 #pragma unroll
             for (int k = 0; k < kM; ++k) {

@@ -27,7 +27,6 @@ namespace eti {
 
 constexpr int kScoreThreads = 256;
 constexpr int kScoreWarps = kScoreThreads / 32;
-constexpr int kFinThreads = 256;
 
 struct ScoreArgs {
     const uint16_t* q;
@@ -350,338 +349,10 @@ struct FinArgs {
     uint32_t* err;          // nullable
 };
 
-template <int N>
-__device__ __forceinline__ void block_reduce_max(float (&v)[N], float* red) {
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int k = 0; k < N; ++k) v[k] = warp_max(v[k]);
-    if (lane == 0)
-        for (int k = 0; k < N; ++k) red[w * N + k] = v[k];
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < N; ++k) {
-        float r = -kInf;
-        for (int i = 0; i < nw; ++i) r = fmaxf(r, red[i * N + k]);
-        v[k] = r;
-    }
-    __syncthreads();
-}
-
-template <int N>
-__device__ __forceinline__ void block_reduce_sum(float (&v)[N], float* red) {
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int k = 0; k < N; ++k) v[k] = warp_sum(v[k]);
-    if (lane == 0)
-        for (int k = 0; k < N; ++k) red[w * N + k] = v[k];
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < N; ++k) {
-        float r = 0.f;
-        for (int i = 0; i < nw; ++i) r += red[i * N + k];
-        v[k] = r;
-    }
-    __syncthreads();
-}
-
-// exclusive block scan of one int per thread; returns the total in *tot
-__device__ __forceinline__ int block_excl_scan(int v, int* red, int* tot) {
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    int x = v;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int y = __shfl_up_sync(0xffffffffu, x, o);
-        if (lane >= o) x += y;
-    }
-    if (lane == 31) red[w] = x;
-    __syncthreads();
-    int ofs = 0, t = 0;
-    for (int i = 0; i < nw; ++i) {
-        if (i < w) ofs += red[i];
-        t += red[i];
-    }
-    __syncthreads();
-    *tot = t;
-    return ofs + x - v;
-}
-
 __device__ __forceinline__ uint32_t order_key(float f) {
     if (f != f) return 0u;
     const uint32_t b = __float_as_uint(f);
     return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
-}
-
-// Shared memory of prune_finalize: block scores / flags, then (when cached)
-// the block stats of the segment, head-major.
-template <int G>
-__host__ __device__ constexpr size_t fin_smem_bytes(int max_blocks, bool cache) {
-    return (size_t)max_blocks * 4 * (cache ? 1 + 3 * G : 1);
-}
-
-template <int G, bool kCache>
-__global__ void __launch_bounds__(kFinThreads)
-prune_finalize_kernel(const FinArgs a) {
-    pdl_trigger();
-    pdl_wait();
-    extern __shared__ __align__(16) float fin_smem[];
-    float* sh_score = fin_smem;                       // [max_blocks]: scores, then keep flags
-    float* sh_m = fin_smem + a.max_blocks;            // [G][max_blocks] (kCache)
-    float* sh_l = sh_m + G * a.max_blocks;
-    float* sh_u = sh_l + G * a.max_blocks;
-    __shared__ float red[(kFinThreads / 32) * 3 * 8];
-    __shared__ int ired[kFinThreads / 32];
-    __shared__ int hist[256];
-    __shared__ int sel_digit, sel_rem;
-    const int seg = blockIdx.x;
-    const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
-    const int tid = threadIdx.x, nt = blockDim.x;
-    const int L = a.ctx_lens[b];
-    const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
-    const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
-    const long long segbase = (long long)seg * a.max_blocks;
-    const int per = (nb + nt - 1) / nt;          // contiguous block range per thread
-    const int j0 = min(tid * per, nb), j1 = min(j0 + per, nb);
-    const float4* st = a.stats + segbase * G;
-
-    // pass 1 (the only pass over global memory when the stats fit in shared
-    // memory): page ids, stats cache, max per head
-    int bad = 0, stale = 0;
-    float M[G];
-#pragma unroll
-    for (int h = 0; h < G; ++h) M[h] = -kInf;
-    for (int j = j0; j < j1; ++j) {
-        const int pg = a.block_table[(long long)b * a.max_blocks + j];
-        bad |= (pg < 0 || (long long)pg >= a.num_pages);
-#pragma unroll
-        for (int h = 0; h < G; ++h) {
-            const float4 s = st[j * G + h];
-            stale |= (s.x != s.x);          // NaN max: the scoring pass gave up on this block
-            if (kCache) {
-                sh_m[h * a.max_blocks + j] = s.x;
-                sh_l[h * a.max_blocks + j] = s.y;
-                sh_u[h * a.max_blocks + j] = a.score_mode == 1 ? s.w : s.z;
-            }
-            M[h] = fmaxf(M[h], s.x);
-        }
-    }
-    const bool bad_page = __syncthreads_or(bad) != 0;
-    const bool timed_out = __syncthreads_or(stale && !bad) != 0;
-    if (a.err && tid == 0) {
-        // err was cleared before this kernel; every kv head ORs in its bits
-        const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page && !bad_ctx ? ETI_ERRF_BAD_PAGE : 0u) |
-                           (timed_out ? ETI_ERRF_TIMEOUT : 0u);
-        if (e) atomicOr(a.err + b, e);
-    }
-    const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
-    const int k0 = min(j0, n), k1 = min(j1, n);
-
-    auto stat = [&](int j, int h) -> float4 {
-        if (kCache) return make_float4(sh_m[h * a.max_blocks + j], sh_l[h * a.max_blocks + j],
-                                       sh_u[h * a.max_blocks + j], 0.f);
-        float4 v = st[j * G + h];
-        if (a.score_mode == 1) v.z = v.w;   // .z: u (mode A) or sum e^{x-m} s_i (mode E)
-        return v;
-    };
-
-    if (!a.given) {
-        if (n > 0) {
-            block_reduce_max<G>(M, red);
-            // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
-            // c_b = e^{m_b - M}: the "1"s of the blocks at the max are counted,
-            // not summed, so log Z = log1p(Z - 1) keeps its relative precision
-            // when one token takes nearly all of the attention.
-            float Zs[2 * G];
-#pragma unroll
-            for (int h = 0; h < 2 * G; ++h) Zs[h] = 0.f;
-            for (int j = k0; j < k1; ++j)
-#pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    const float4 s = stat(j, h);
-                    const bool top = !(s.x < M[h]);
-                    const float cb = top ? 1.f : expf(s.x - M[h]);
-                    Zs[h] += cb * s.y + (top ? 0.f : cb);
-                    Zs[G + h] += top ? 1.f : 0.f;
-                }
-            block_reduce_sum<2 * G>(Zs, red);
-            float lZ[G], Z[G], Hs[G];
-#pragma unroll
-            for (int h = 0; h < G; ++h) {
-                const float zm1 = Zs[h] + (Zs[G + h] - 1.f);
-                lZ[h] = log1pf(zm1);
-                Z[h] = 1.f + zm1;
-                Hs[h] = 0.f;
-            }
-            // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
-            // mode E: I_b = e^{m_b - M} sum e^{x-m_b} s_i / Z; mode M: the block's mass
-            auto Ib = [&](float4 s, int h) {
-                if (a.score_mode == 1) return expf(s.x - M[h]) * s.z / Z[h];
-                if (a.score_mode == 2) return expf(s.x - M[h]) * (1.f + s.y) / Z[h];
-                return expf(s.x - M[h]) * ((1.f + s.y) * (lZ[h] + M[h] - s.x) - s.z) / Z[h];
-            };
-            for (int j = k0; j < k1; ++j)
-#pragma unroll
-                for (int h = 0; h < G; ++h) Hs[h] += Ib(stat(j, h), h);
-            block_reduce_sum<G>(Hs, red);
-            for (int j = k0; j < k1; ++j) {
-                float best = -kInf;
-#pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    const float nrm = Hs[h] > 0.f ? (float)n * Ib(stat(j, h), h) / Hs[h] : 1.f;
-                    best = fmaxf(best, nrm);
-                }
-                sh_score[j] = best;
-            }
-        }
-        __syncthreads();
-        if (a.block_score) {
-            for (int j = tid; j < a.max_blocks; j += nt)
-                a.block_score[segbase + j] = j < n ? sh_score[j] : 0.f;
-        }
-        // B_min budget: the first k blocks by (score desc, index asc)
-        const int k = min(max(a.B_min, 0), n);
-        uint32_t kth = 0xffffffffu;   // keys > kth are selected; `rem` of those == kth
-        int rem = 0;
-        int arg = -1;                 // B_min == 1: the first block of highest score
-        if (k == 1 && n > 1) {
-            float bs = -kInf;
-            int bj = 0x7fffffff;
-            for (int j = k0; j < k1; ++j) {
-                const float v = sh_score[j];
-                if (v > bs || bj == 0x7fffffff) { bs = v; bj = j; }
-            }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                const float ov = __shfl_xor_sync(0xffffffffu, bs, o);
-                const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
-                if (ov > bs || (ov == bs && oj < bj)) { bs = ov; bj = oj; }
-            }
-            if ((tid & 31) == 0) { red[tid >> 5] = bs; ired[tid >> 5] = bj; }
-            __syncthreads();
-            if (tid == 0) {
-                for (int w = 1; w < nt / 32; ++w)
-                    if (red[w] > bs || (red[w] == bs && ired[w] < bj)) { bs = red[w]; bj = ired[w]; }
-                sel_digit = bj;
-            }
-            __syncthreads();
-            arg = sel_digit;
-            __syncthreads();
-        } else if (k > 1 && k < n) {
-            uint32_t prefix = 0, mask = 0;
-            int need = k;
-            for (int digit = 3; digit >= 0; --digit) {
-                const int sh = digit * 8;
-                for (int i = tid; i < 256; i += nt) hist[i] = 0;
-                __syncthreads();
-                for (int j = k0; j < k1; ++j) {
-                    const uint32_t key = order_key(sh_score[j]);
-                    if ((key & mask) == prefix) atomicAdd(&hist[(key >> sh) & 255], 1);
-                }
-                __syncthreads();
-                // bucket where the count from the top reaches `need`
-                if (tid < 32) {
-                    int cnt8[8], s8 = 0;
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) { cnt8[e] = hist[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
-                    int incl = s8;
-#pragma unroll
-                    for (int o = 1; o < 32; o <<= 1) {
-                        const int y = __shfl_up_sync(0xffffffffu, incl, o);
-                        if (tid >= o) incl += y;
-                    }
-                    int above = incl - s8;
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        if (above < need && need <= above + cnt8[e]) {
-                            sel_digit = 255 - (tid * 8 + e);
-                            sel_rem = need - above;
-                        }
-                        above += cnt8[e];
-                    }
-                }
-                __syncthreads();
-                prefix |= (uint32_t)sel_digit << sh;
-                mask |= 255u << sh;
-                need = sel_rem;
-                __syncthreads();
-            }
-            kth = prefix;
-            rem = need;
-        }
-        // flags: threshold or budget (ties at the k-th key go to the lower index)
-        const float th = a.theta[b];
-        int eq = 0;
-        for (int j = k0; j < k1; ++j) eq += (k > 1 && k < n && order_key(sh_score[j]) == kth);
-        int eq_tot;
-        int eq_rank = block_excl_scan(eq, ired, &eq_tot);
-        for (int j = k0; j < k1; ++j) {
-            const float sc = sh_score[j];
-            bool keep = sc >= th || k >= n;
-            if (k == 1) keep |= (j == arg);
-            else if (k > 1 && k < n) {
-                const uint32_t key = order_key(sc);
-                if (key > kth) keep = true;
-                else if (key == kth) { keep |= eq_rank < rem; ++eq_rank; }
-            }
-            sh_score[j] = keep ? 1.f : 0.f;   // scores are no longer needed
-        }
-        __syncthreads();
-    } else {
-        // given keep set
-        for (int j = k0; j < k1; ++j) sh_score[j] = 0.f;
-        __syncthreads();
-        if (a.given_idx) {
-            const int c = min(max(a.given_cnt[seg], 0), a.max_blocks);
-            for (int i = tid; i < c; i += nt) {
-                const int j = a.given_idx[segbase + i];
-                if (j >= 0 && j < n) sh_score[j] = 1.f;
-            }
-        } else {
-            for (int j = k0; j < k1; ++j) sh_score[j] = a.given_mask ? (a.given_mask[segbase + j] ? 1.f : 0.f) : 1.f;
-        }
-        __syncthreads();
-    }
-
-    // compaction (ascending block index)
-    int cnt = 0;
-    for (int j = k0; j < k1; ++j) cnt += sh_score[j] != 0.f;
-    int total;
-    int pos = block_excl_scan(cnt, ired, &total);
-    for (int j = k0; j < k1; ++j)
-        if (sh_score[j] != 0.f) a.kept_idx[segbase + pos++] = j;
-    for (int i = total + tid; i < a.max_blocks; i += nt) a.kept_idx[segbase + i] = -1;
-    if (a.keep_mask)
-        for (int j = tid; j < a.max_blocks; j += nt)
-            a.keep_mask[segbase + j] = (j < n && sh_score[j] != 0.f) ? 1 : 0;
-    if (tid == 0) a.kept_cnt[seg] = total;
-
-    // softmax normaliser over the kept tokens of each query head
-    if (a.kept_norm) {
-        float Mk[G], Lk[G];
-#pragma unroll
-        for (int h = 0; h < G; ++h) { Mk[h] = -kInf; Lk[h] = 0.f; }
-        for (int j = k0; j < k1; ++j)
-            if (sh_score[j] != 0.f)
-#pragma unroll
-                for (int h = 0; h < G; ++h) Mk[h] = fmaxf(Mk[h], stat(j, h).x);
-        block_reduce_max<G>(Mk, red);
-        for (int j = k0; j < k1; ++j)
-            if (sh_score[j] != 0.f)
-#pragma unroll
-                for (int h = 0; h < G; ++h) {
-                    const float4 s = stat(j, h);
-                    Lk[h] += (1.f + s.y) * expf(s.x - Mk[h]);
-                }
-        block_reduce_sum<G>(Lk, red);
-        if (tid < a.g) {
-            float mm = 0.f, ll = 0.f;
-#pragma unroll
-            for (int h = 0; h < G; ++h)
-                if (h == tid) { mm = Mk[h]; ll = Lk[h]; }
-            float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + tid) * 2;
-            kn[0] = mm;
-            kn[1] = ll;
-        }
-    }
 }
 
 // ---------------------------------------------------------------------------
@@ -695,6 +366,8 @@ prune_finalize_kernel(const FinArgs a) {
 // score, so they take the same keep decision; ranks in ascending block order
 // (budget ties, compaction) come from ballots over the head-0 lanes.
 constexpr int kFlatPer = 16;
+constexpr int kWideThreads = 1024;
+constexpr size_t kWideSmemMax = 200 * 1024;   // dynamic shared memory of the cached-term variant
 
 template <int G>
 struct FlatGP { static constexpr int v = G <= 1 ? 1 : G <= 2 ? 2 : G <= 4 ? 4 : 8; };
@@ -917,9 +590,10 @@ prune_finalize_flat_kernel(const FinArgs a) {
             const int sh = digit * 8;
             for (int i = tid; i < 256; i += NT) hist[i] = 0;
             __syncthreads();
-            for (int j = tid; j < n; j += NT) {
-                const uint32_t key = order_key(sh_score[j]);
-                if ((key & mask) == prefix) atomicAdd(&hist[(key >> sh) & 255], 1);
+            for (int j0 = 0; j0 < n; j0 += NT) {      // the same trip count for every lane
+                const int j = j0 + tid;
+                const uint32_t key = j < n ? order_key(sh_score[j]) : 0u;
+                warp_hist_add(hist, (key >> sh) & 255, j < n && (key & mask) == prefix);
             }
             __syncthreads();
             // bucket where the count from the top reaches `need`
@@ -1005,6 +679,313 @@ prune_finalize_flat_kernel(const FinArgs a) {
     }
 }
 
+// ---------------------------------------------------------------------------
+// prune_finalize for segments of any size (and for the given keep sets), one
+// CTA of NT threads per (sequence, kv head), in the flat kernel's layout:
+// thread t owns query head h = t % GP of the blocks r * RB + t / GP + k * JS,
+// k < kFlatPer, in rounds r of RB = JS * kFlatPer blocks.  Every pass walks
+// the rounds and re-reads the block stats (L2-resident after the first
+// pass), so loads are coalesced and nothing of size max_blocks lives in
+// registers; the group scores, then the keep flags, live in shared memory
+// ([max_blocks] floats); the ranks in ascending block order (budget ties,
+// compaction) are ballot scans per round with a running base.
+template <int G, int NT, bool kTerm>
+__global__ void __launch_bounds__(NT)
+prune_finalize_wide_kernel(const FinArgs a) {
+    constexpr int GP = FlatGP<G>::v;
+    constexpr int JS = NT / GP;                  // block stride between a thread's chunks
+    constexpr int RB = JS * kFlatPer;            // blocks per round
+    pdl_trigger();
+    pdl_wait();
+    extern __shared__ __align__(16) float wf_smem[];
+    float* sh = wf_smem;                         // [max_blocks]: group scores, then keep flags
+    // kTerm: [max_blocks * GP] per block-head e^{m_b - M}, then the term I_b
+    // (index j * GP + h: a warp's accesses are consecutive)
+    float* sh_t = wf_smem + a.max_blocks;
+    __shared__ float red[4][2 * 32 * GP];
+    __shared__ int scan[2][kFlatPer * 32 + 1];
+    __shared__ int hist[256];
+    __shared__ int sel_digit, sel_rem;
+    __shared__ float arg_v[32];
+    __shared__ int arg_j[32];
+    const int seg = blockIdx.x;
+    const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int h = lane & (GP - 1);
+    const int jt = tid / GP;
+    const int L = a.ctx_lens[b];
+    const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
+    const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
+    const int nr = (nb + RB - 1) / RB;           // rounds (the same for every thread)
+    const long long segbase = (long long)seg * a.max_blocks;
+    const float4* st = a.stats + segbase * G;
+    auto stat = [&](int j) {
+        float4 v = st[(long long)j * G + h];
+        if (a.score_mode == 1) v.z = v.w;        // .z: u (mode A) or sum e^{x-m} s_i (mode E)
+        return v;
+    };
+
+    int bad = 0;
+    for (int j = tid; j < nb; j += NT) {
+        const int pg = a.block_table[(long long)b * a.max_blocks + j];
+        bad |= (pg < 0 || (long long)pg >= a.num_pages);
+    }
+    int stale = 0;
+    float Mh[1] = {-kInf};
+    for (int r = 0; r < nr; ++r)
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const int j = r * RB + jt + k * JS;
+            if (h < G && j < nb) {
+                const float x = st[(long long)j * G + h].x;
+                stale |= (x != x);               // NaN max: the scoring pass gave up on this block
+                Mh[0] = fmaxf(Mh[0], x);
+            }
+        }
+    const bool bad_page = __syncthreads_or(bad) != 0;
+    const bool timed_out = __syncthreads_or(stale) != 0 && !bad_page;
+    if (a.err && tid == 0) {
+        // err was cleared before this kernel; every kv head ORs in its bits
+        const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page ? ETI_ERRF_BAD_PAGE : 0u) |
+                           (timed_out ? ETI_ERRF_TIMEOUT : 0u);
+        if (e) atomicOr(a.err + b, e);
+    }
+    const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
+    float M = -kInf;
+    if (n > 0) {
+        head_reduce<GP, 1, true>(Mh, red[0]);
+        M = Mh[0];
+    }
+
+    if (!a.given) {
+        if (n > 0) {
+            // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
+            // c_b = e^{m_b - M} (the blocks at the max are counted, not summed)
+            float zs[2] = {0.f, 0.f};
+            for (int r = 0; r < nr; ++r)
+#pragma unroll
+                for (int k = 0; k < kFlatPer; ++k) {
+                    const int j = r * RB + jt + k * JS;
+                    if (h < G && j < n) {
+                        const float4 v = stat(j);
+                        const bool top = !(v.x < M);
+                        const float c = top ? 1.f : expf(v.x - M);
+                        zs[0] += c * v.y + (top ? 0.f : c);
+                        zs[1] += top ? 1.f : 0.f;
+                        if (kTerm) sh_t[j * GP + h] = c;
+                    }
+                }
+            head_reduce<GP, 2, false>(zs, red[1]);
+            const float zm1 = zs[0] + (zs[1] - 1.f);
+            const float lZ = log1pf(zm1), iZ = 1.f / (1.f + zm1);
+            // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
+            auto Ib = [&](float4 v, float c) {
+                if (a.score_mode == 1) return c * v.z * iZ;                 // E
+                if (a.score_mode == 2) return c * (1.f + v.y) * iZ;         // M
+                return c * ((1.f + v.y) * (lZ + M - v.x) - v.z) * iZ;
+            };
+            float Hs[1] = {0.f};
+            for (int r = 0; r < nr; ++r)
+#pragma unroll
+                for (int k = 0; k < kFlatPer; ++k) {
+                    const int j = r * RB + jt + k * JS;
+                    if (h < G && j < n) {
+                        const float4 v = stat(j);
+                        const float t = Ib(v, kTerm ? sh_t[j * GP + h] : (v.x < M ? expf(v.x - M) : 1.f));
+                        if (kTerm) sh_t[j * GP + h] = t;
+                        Hs[0] += t;
+                    }
+                }
+            head_reduce<GP, 1, false>(Hs, red[2]);
+            const float nH = Hs[0] > 0.f ? (float)n / Hs[0] : 0.f;
+            // group score: the largest normalised term over the heads of the block
+            for (int r = 0; r < nr; ++r)
+#pragma unroll
+                for (int k = 0; k < kFlatPer; ++k) {
+                    const int j = r * RB + jt + k * JS;
+                    float sc = -kInf;
+                    if (h < G && j < n) {
+                        float t;
+                        if (kTerm) {
+                            t = sh_t[j * GP + h];
+                        } else {
+                            const float4 v = stat(j);
+                            t = Ib(v, v.x < M ? expf(v.x - M) : 1.f);
+                        }
+                        sc = Hs[0] > 0.f ? t * nH : 1.f;
+                    }
+#pragma unroll
+                    for (int o = 1; o < GP; o <<= 1) sc = fmaxf(sc, __shfl_xor_sync(0xffffffffu, sc, o));
+                    if (h == 0 && j < n) sh[j] = sc;
+                }
+        }
+        __syncthreads();
+        if (a.block_score)
+            for (int j = tid; j < a.max_blocks; j += NT) a.block_score[segbase + j] = j < n ? sh[j] : 0.f;
+
+        // B_min budget: the first kb blocks by (score desc, index asc)
+        const float th = a.theta ? a.theta[b] : kInf;
+        const int kb = min(max(a.B_min, 0), n);
+        int arg = -1;
+        uint32_t kth = 0u;
+        int need = 0;
+        if (kb == 1 && n > 1) {
+            float bs = -kInf;
+            int bj = 0x7fffffff;
+            for (int j = tid; j < n; j += NT) {
+                const float v = sh[j];
+                if (v > bs || bj == 0x7fffffff) { bs = v; bj = j; }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float ov = __shfl_xor_sync(0xffffffffu, bs, o);
+                const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+                if (ov > bs || (ov == bs && oj < bj)) { bs = ov; bj = oj; }
+            }
+            if (lane == 0) { arg_v[tid >> 5] = bs; arg_j[tid >> 5] = bj; }
+            __syncthreads();
+            for (int u = 0; u < NT / 32; ++u)
+                if (arg_v[u] > bs || (arg_v[u] == bs && arg_j[u] < bj)) { bs = arg_v[u]; bj = arg_j[u]; }
+            arg = bj;
+        } else if (kb > 1 && kb < n) {
+            uint32_t prefix = 0, mask = 0;
+            need = kb;
+            for (int digit = 3; digit >= 0; --digit) {
+                const int shf = digit * 8;
+                for (int i = tid; i < 256; i += NT) hist[i] = 0;
+                __syncthreads();
+                for (int j0 = 0; j0 < n; j0 += NT) {  // the same trip count for every lane
+                    const int j = j0 + tid;
+                    const uint32_t key = j < n ? order_key(sh[j]) : 0u;
+                    warp_hist_add(hist, (key >> shf) & 255, j < n && (key & mask) == prefix);
+                }
+                __syncthreads();
+                // bucket where the count from the top reaches `need`
+                if (tid < 32) {
+                    int cnt8[8], s8 = 0;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) { cnt8[e] = hist[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
+                    int incl = s8;
+#pragma unroll
+                    for (int o = 1; o < 32; o <<= 1) {
+                        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                        if (tid >= o) incl += y;
+                    }
+                    int above = incl - s8;
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        if (above < need && need <= above + cnt8[e]) {
+                            sel_digit = 255 - (tid * 8 + e);
+                            sel_rem = need - above;
+                        }
+                        above += cnt8[e];
+                    }
+                }
+                __syncthreads();
+                prefix |= (uint32_t)sel_digit << shf;
+                mask |= 255u << shf;
+                need = sel_rem;
+                __syncthreads();
+            }
+            kth = prefix;
+        }
+        // keep flags: threshold, budget (ties at the k-th key to the lower index)
+        const bool sel = kb > 1 && kb < n;
+        int eq_base = 0;
+        for (int r = 0; r < nr; ++r) {
+            bool eq[kFlatPer], keep[kFlatPer];
+            int eq_pos[kFlatPer];
+#pragma unroll
+            for (int k = 0; k < kFlatPer; ++k) {
+                const int j = r * RB + jt + k * JS;
+                const float sc = j < n ? sh[j] : -kInf;
+                const uint32_t key = order_key(sc);
+                keep[k] = j < n && (sc >= th || kb >= n || j == arg || (sel && key > kth));
+                eq[k] = sel && j < n && key == kth;
+            }
+            if (sel) {
+                const int c = flat_ranks<GP>(eq, eq_pos, scan[r & 1]);
+#pragma unroll
+                for (int k = 0; k < kFlatPer; ++k) keep[k] |= eq[k] && eq_base + eq_pos[k] < need;
+                eq_base += c;
+            }
+            __syncthreads();    // every lane of a block has read its score
+#pragma unroll
+            for (int k = 0; k < kFlatPer; ++k) {
+                const int j = r * RB + jt + k * JS;
+                if (h == 0 && j < n) sh[j] = keep[k] ? 1.f : 0.f;
+            }
+        }
+        __syncthreads();
+    } else {
+        // given keep set: a list, a mask, or every block
+        if (a.given_idx) {
+            for (int j = tid; j < n; j += NT) sh[j] = 0.f;
+            __syncthreads();
+            const int c = min(max(a.given_cnt[seg], 0), a.max_blocks);
+            for (int i = tid; i < c; i += NT) {
+                const int j = a.given_idx[segbase + i];
+                if (j >= 0 && j < n) sh[j] = 1.f;
+            }
+        } else {
+            for (int j = tid; j < n; j += NT) sh[j] = a.given_mask ? (a.given_mask[segbase + j] ? 1.f : 0.f) : 1.f;
+        }
+        __syncthreads();
+    }
+
+    // compaction (ascending block index), round by round
+    int total = 0;
+    for (int r = 0; r < nr; ++r) {
+        bool keep[kFlatPer];
+        int pos[kFlatPer];
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const int j = r * RB + jt + k * JS;
+            keep[k] = j < n && sh[j] != 0.f;
+        }
+        const int c = flat_ranks<GP>(keep, pos, scan[r & 1]);
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const int j = r * RB + jt + k * JS;
+            if (h == 0 && keep[k]) a.kept_idx[segbase + total + pos[k]] = j;
+            if (a.keep_mask && h == 0 && j < n) a.keep_mask[segbase + j] = keep[k] ? 1 : 0;
+        }
+        total += c;
+    }
+    for (int i = total + tid; i < a.max_blocks; i += NT) a.kept_idx[segbase + i] = -1;
+    if (a.keep_mask)
+        for (int j = n + tid; j < a.max_blocks; j += NT) a.keep_mask[segbase + j] = 0;
+    if (tid == 0) a.kept_cnt[seg] = total;
+
+    // softmax normaliser over the kept tokens of each query head
+    if (a.kept_norm) {
+        float Mk[1] = {-kInf};
+        for (int r = 0; r < nr; ++r)
+#pragma unroll
+            for (int k = 0; k < kFlatPer; ++k) {
+                const int j = r * RB + jt + k * JS;
+                if (h < G && j < n && sh[j] != 0.f) Mk[0] = fmaxf(Mk[0], st[(long long)j * G + h].x);
+            }
+        head_reduce<GP, 1, true>(Mk, red[3]);
+        float Lk[1] = {0.f};
+        for (int r = 0; r < nr; ++r)
+#pragma unroll
+            for (int k = 0; k < kFlatPer; ++k) {
+                const int j = r * RB + jt + k * JS;
+                if (h < G && j < n && sh[j] != 0.f) {
+                    const float4 v = st[(long long)j * G + h];
+                    Lk[0] += (1.f + v.y) * expf(v.x - Mk[0]);
+                }
+            }
+        head_reduce<GP, 1, false>(Lk, red[0]);
+        if (tid < GP && h < G) {
+            float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2;
+            kn[0] = Mk[0];
+            kn[1] = Lk[0];
+        }
+    }
+}
+
 }  // namespace eti
 
 using namespace eti;
@@ -1068,9 +1049,6 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     const int grid = B * Hkv;
     cudaError_t e = cudaSuccess;
     if (err && cudaMemsetAsync(err, 0, (size_t)B * sizeof(uint32_t), stream) != cudaSuccess) return ETI_ERR_CUDA;
-    int dev = 0, optin = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     // the flat kernel holds a segment in registers: 16 block-heads a thread
     const int gp = a.g <= 1 ? 1 : a.g <= 2 ? 2 : a.g <= 4 ? 4 : 8;
     const long long flat_need = ((long long)max_blocks * gp + kFlatPer - 1) / kFlatPer;
@@ -1089,11 +1067,13 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
         ETI_FIN_FLAT(GG, 128)                                                               \
         ETI_FIN_FLAT(GG, 256)                                                               \
         ETI_FIN_FLAT(GG, 512)                                                               \
-        const bool cache = fin_smem_bytes<GG>(max_blocks, true) <= (size_t)optin / 2;      \
-        const size_t smem = fin_smem_bytes<GG>(max_blocks, cache);                          \
-        auto k = cache ? prune_finalize_kernel<GG, true> : prune_finalize_kernel<GG, false>; \
+        const size_t smem_t = (size_t)max_blocks * 4 * (1 + gp);                           \
+        const bool term = !given && smem_t <= kWideSmemMax;                                 \
+        auto k = term ? prune_finalize_wide_kernel<GG, kWideThreads, true>                  \
+                      : prune_finalize_wide_kernel<GG, kWideThreads, false>;                \
+        const size_t smem = term ? smem_t : (size_t)max_blocks * 4;                         \
         if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-        e = eti_launch_pdl(k, dim3(grid), dim3(kFinThreads), smem, stream, a);              \
+        e = eti_launch_pdl(k, dim3(grid), dim3(kWideThreads), smem, stream, a);             \
         break;                                                                              \
     }
     switch (a.g) {
