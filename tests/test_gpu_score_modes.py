@@ -183,3 +183,31 @@ def test_fused_surprisal_store(eti, noalloc):
     r = parity.oracle_ets(lg, seed=3, offset=1)
     ok = (e == 0) & (r["tok"] == tok.cpu().numpy())
     assert np.allclose(sp[ok], r["surprisal"][ok], rtol=1e-4, atol=1e-5)
+
+
+@pytest.mark.parametrize("mode,name", [(0, "A")] + MODES)
+def test_score_modes_long_segments(eti, mode, name):
+    """Segments past the register-resident layout (up to 8192 blocks with
+    g = 4): the keep set comes from the wide kernel with its shared-memory
+    cache of the block terms, in all three score modes."""
+    w = workloads.Workload("wl", B=2, Hq=32, Hkv=8, D=128, P=16, V=16, ctx=("list", [40000, 131072]),
+                           seed=21 + mode, hi_frac=0.02)
+    kv = workloads.make_kv(w, DEV)
+    store = _store(kv, seed=3 + mode)
+    th = torch.full((w.B,), 0.9, dtype=torch.float32, device=DEV)
+    got = _score_prune(eti, w, kv, th, 3, mode, store)
+    s = _check(got, parity.host_kv(kv), store.cpu().numpy(), th.cpu().numpy(), 3, mode)
+    print(name, s)
+
+
+def test_prune_long_segment_without_term_cache(eti):
+    """12,500 blocks with g = 4 need more than the 200 KB term cache: the wide
+    kernel recomputes the terms from the stats; a budget select as well."""
+    w = workloads.Workload("wn", B=1, Hq=32, Hkv=8, D=128, P=16, V=16, ctx=("list", [200000]),
+                           seed=31, hi_frac=0.02)
+    assert w.max_blocks * 4 * (1 + 4) > 200 * 1024
+    kv = workloads.make_kv(w, DEV)
+    th = torch.full((w.B,), 1.2, dtype=torch.float32, device=DEV)
+    got = _score_prune(eti, w, kv, th, 700, 0, None)
+    s = _check(got, parity.host_kv(kv), None, th.cpu().numpy(), 700, 0)
+    print(s)
