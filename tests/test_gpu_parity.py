@@ -78,6 +78,18 @@ def test_entropy_sample_strided_and_unaligned_rows(eti):
     parity.compare_ets(g, r, lg2, seed=1, offset=2)
 
 
+@pytest.mark.parametrize("B,V", [(65535, 37), (2, 1000003)])
+def test_entropy_sample_maximum_sizes(eti, B, V):
+    """The largest batch the call accepts (65535 rows, a ragged vocabulary) and
+    a vocabulary of a million tokens: every row against the oracle."""
+    w = workloads.Workload("x", B=B, Hq=1, Hkv=1, D=64, P=16, V=V, ctx=("list", [1] * B), seed=B + V)
+    lg = workloads.make_logits(w, DEV)
+    g = parity.run_ets(eti, lg, seed=5, offset=11)
+    r = parity.oracle_ets(lg, seed=5, offset=11)
+    st = parity.compare_ets(g, r, lg, seed=5, offset=11)
+    print(B, V, st)
+
+
 @pytest.mark.parametrize("kw", [dict(), dict(sign=1.0), dict(eta=0.5, T_min=0.5, T_max=1.5),
                                 dict(eps_H=0.7, H_min=3.0, theta_user=0.4, theta_hi=2.0),
                                 dict(T_cal=1.5), dict(T_cal=0.7, eta=0.3),
