@@ -483,15 +483,27 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
     """Same metric through the public API from pinned host buffers: per step the
     step's inputs (q, logits, per-sequence state, threshold) go host -> device and
     its results (attention output, token, entropy, temperature, threshold) come back."""
-    h_q = kv["q"].cpu().pin_memory()
+    # One byte buffer per direction for the small per-step data, so each
+    # direction costs one copy (a small copy costs ~12 us whatever its size):
+    #   [q | T_in H_prev H_target theta | tau theta_next tok H T_out surprisal err]
+    # goes up as far as tau (q, the state, tau) and comes back from tau on.
+    B = w.B
+    qb = kv["q"].numel() * 2
+    row = B * 4
+    n_in, n_all = qb + 5 * row, qb + 11 * row
+    d_io = torch.zeros(n_all, dtype=torch.uint8, device=device)
+    d_q = d_io[:qb].view(torch.bfloat16).view(kv["q"].shape)
+    rows = d_io[qb:].view(torch.float32).view(11, B)
+    T_in, H_prev, H_tgt, th, tau = rows[0], rows[1], rows[2], rows[3], rows[4]
+    th_next, H_out, T_out, surp = rows[5], rows[7], rows[8], rows[9]
+    tok, err = rows[6].view(torch.int32), rows[10].view(torch.int32)
+    d_io[:qb].view(torch.bfloat16).copy_(kv["q"].reshape(-1))
+    rows[:5].copy_(torch.stack([lg["T_in"], lg["H_prev"], lg["H_target"], theta, lg["tau"]]))
+    h_in = d_io[:n_in].cpu().pin_memory()
+    h_res = torch.empty(n_all - (qb + 4 * row), dtype=torch.uint8).pin_memory()
     h_logits = lg["logits"].cpu().pin_memory()
-    h_state = torch.stack([lg["T_in"], lg["H_prev"], lg["H_target"], lg["tau"], theta]).cpu().pin_memory()
-    d_q = torch.empty_like(kv["q"])
     d_logits = torch.empty_like(lg["logits"])
-    d_state = torch.empty_like(h_state, device=device)
     h_out = torch.empty(step.out.shape, dtype=step.out.dtype).pin_memory()
-    h_res = torch.empty((4, w.B), dtype=torch.float32).pin_memory()
-    h_tok = torch.empty(w.B, dtype=torch.int32).pin_memory()
 
     # The logits (the bulk of the bytes) go up on a copy stream while the
     # attention half runs; the sampling call waits for them.  The attention
@@ -509,12 +521,10 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
         with torch.cuda.stream(copy):
             d_logits.copy_(h_logits, non_blocking=True)
             ev_logits.record(copy)
-        d_q.copy_(h_q, non_blocking=True)
-        d_state.copy_(h_state, non_blocking=True)
-        T_in, H_prev, H_tgt, tau, th = d_state[0], d_state[1], d_state[2], d_state[3], d_state[4]
+        d_io[:n_in].copy_(h_in, non_blocking=True)
         eti.eti_score_blocks(d_q, kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
                              stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
-        eti.eti_prune_blocks(stats, kv["block_table"], kv["ctx_lens"], shape, th.contiguous(), B_min,
+        eti.eti_prune_blocks(stats, kv["block_table"], kv["ctx_lens"], shape, th, B_min,
                              step.keep_mask, step.kept_idx, step.kept_cnt, step.err_attn,
                              kept_norm=step.kept_norm, num_pages=kv["num_pages"])
         eti.eti_paged_decode(d_q, kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
@@ -527,13 +537,10 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
             copy.wait_event(ev_out)
             h_out.copy_(step.out, non_blocking=True)
         cur.wait_event(ev_logits)
-        step.sample(d_logits, T_in.contiguous(), H_prev.contiguous(), tau.contiguous(),
-                    H_tgt.contiguous(), params=prm, seed=w.seed, offset=i)
-        h_tok.copy_(step.tok, non_blocking=True)
-        h_res[0].copy_(step.H, non_blocking=True)
-        h_res[1].copy_(step.T_out, non_blocking=True)
-        h_res[2].copy_(step.theta_next, non_blocking=True)
-        h_res[3].copy_(step.surprisal, non_blocking=True)
+        eti.eti_entropy_temp_sample(d_logits, T_in, H_prev, tau, H_tgt, tok, H_out, T_out, err,
+                                    step.ws_ets, params=prm, seed=w.seed, offset=i,
+                                    theta_next=th_next, tok_surprisal=surp)
+        h_res.copy_(d_io[qb + 4 * row:], non_blocking=True)
         cur.wait_stream(copy)                                  # join
 
     for i in range(args.warmup):
@@ -563,8 +570,8 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
             main.synchronize()
         times.append(time.perf_counter() - t0)
     s = statistics.mean(times)
-    bi = h_q.numel() * 2 + h_logits.numel() * 4 + h_state.numel() * 4
-    bo = h_out.numel() * 2 + h_tok.numel() * 4 + h_res.numel() * 4
+    bi = h_in.numel() + h_logits.numel() * 4
+    bo = h_out.numel() * 2 + h_res.numel()
     return {"value": round(w.B / s, 1), "unit": UNIT, "ms_per_step": round(s * 1e3, 4),
             "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo), "mode": mode}
 
