@@ -269,6 +269,23 @@ def test_standalone_decode_modes(eti, mode):
     assert np.array_equal(err.cpu().numpy().view(np.uint32), rerr)
 
 
+def test_attention_maximum_batch(eti):
+    """The largest batch the attention calls accept (8192 sequences): the
+    scorer's per-sequence prefix no longer leaves room for two CTAs per SM.
+    Ragged contexts of 0 to 100 tokens (empty sequences included), every
+    sequence against the oracle."""
+    B = 8192
+    lens = np.random.default_rng(9).integers(0, 101, B)
+    lens[::97] = 0
+    w = workloads.Workload("mb", B=B, Hq=8, Hkv=2, D=64, P=16, V=16, ctx=("list", [int(x) for x in lens]),
+                           seed=9, hi_frac=0.05)
+    kv = workloads.make_kv(w, DEV)
+    th = torch.full((B,), 0.9, dtype=torch.float32, device=DEV)
+    st = _step(eti, w, kv, th, 2)
+    s = _check_step(st, parity.host_kv(kv), th.cpu().numpy(), 2, w.P)
+    print(s)
+
+
 def test_attention_edge_cases(eti):
     """Empty sequences, a bad page id and a bad context length: error bits and zero outputs."""
     w = workloads.Workload("e", B=4, Hq=8, Hkv=2, D=64, P=16, V=16, ctx=("list", [0, 40, 40, 40]),
