@@ -101,7 +101,9 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
         __syncthreads();
     }
     const int total = carry;
-    const int share = max(1, (total + a.nwarps - 1) / a.nwarps);
+    // at least 32 kept blocks per warp: below that, the pipeline fill and the
+    // merge of many small split parts cost more than the extra warps bring
+    const int share = max(32, (total + a.nwarps - 1) / a.nwarps);
     if (tid == 0) {
         a.cum[a.nseg] = total;
         a.info[0] = total;
