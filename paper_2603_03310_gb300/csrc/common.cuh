@@ -229,6 +229,35 @@ __device__ __forceinline__ int warp_sum_i(int v) {
     return v;
 }
 
+// ---- thread-block clusters (distributed shared memory) ----------------------
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+// Barrier over every thread of every CTA of the cluster (release / acquire:
+// shared-memory writes before it are visible to the cluster after it).
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\t"
+                 "barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Loads from the same shared-memory variable of CTA `rank` of the cluster.
+__device__ __forceinline__ float ld_cluster_f32(const void* p, uint32_t rank) {
+    uint32_t a;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ int ld_cluster_s32(const void* p, uint32_t rank) {
+    uint32_t a;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(smem_u32(p)), "r"(rank));
+    int v;
+    asm volatile("ld.shared::cluster.s32 %0, [%1];" : "=r"(v) : "r"(a) : "memory");
+    return v;
+}
+
 // hist[bin] += 1 for every lane with `on`, one shared-memory atomic per
 // distinct bin of the warp (every lane of the warp must call it together)
 __device__ __forceinline__ void warp_hist_add(int* hist, uint32_t bin, bool on) {

@@ -680,16 +680,26 @@ prune_finalize_flat_kernel(const FinArgs a) {
 }
 
 // ---------------------------------------------------------------------------
-// prune_finalize for segments of any size (and for the given keep sets), one
-// CTA of NT threads per (sequence, kv head), in the flat kernel's layout:
-// thread t owns query head h = t % GP of the blocks r * RB + t / GP + k * JS,
-// k < kFlatPer, in rounds r of RB = JS * kFlatPer blocks.  Every pass walks
-// the rounds and re-reads the block stats (L2-resident after the first
-// pass), so loads are coalesced and nothing of size max_blocks lives in
-// registers; the group scores, then the keep flags, live in shared memory
-// ([max_blocks] floats); the ranks in ascending block order (budget ties,
-// compaction) are ballot scans per round with a running base.
-template <int G, int NT, bool kTerm>
+// prune_finalize for segments of any size (and for the given keep sets), in
+// the flat kernel's layout: thread t owns query head h = t % GP of the blocks
+// r * RB + t / GP + k * JS, k < kFlatPer, in rounds r of RB = JS * kFlatPer
+// blocks.  Every pass walks the rounds and re-reads the block stats
+// (L2-resident after the first pass), so loads are coalesced and nothing of
+// size max_blocks lives in registers; the group scores, then the keep flags,
+// live in shared memory ([max_blocks] floats); with kTerm the term of every
+// block-head too.  Ranks in ascending block order (budget ties, compaction)
+// are ballot scans per round with a running base.
+//
+// A segment is handled by a cluster of kCl CTAs (kCl = 1: one CTA): CTA rank
+// c takes a contiguous run of the rounds.  The per-head reductions, the error
+// flags, the budget histograms and argmax, and the counts that offset the
+// ordered ranks are exchanged through distributed shared memory, each CTA
+// combining all ranks' values in rank order, so every CTA of the cluster
+// holds the same bits.  Cluster barriers sit in code every CTA of the cluster
+// runs the same number of times (it depends on the segment only).
+constexpr int kWideX = 16;    // exchange slots (one per exchange, never reused)
+
+template <int G, int NT, bool kTerm, int kCl>
 __global__ void __launch_bounds__(NT)
 prune_finalize_wide_kernel(const FinArgs a) {
     constexpr int GP = FlatGP<G>::v;
@@ -704,11 +714,16 @@ prune_finalize_wide_kernel(const FinArgs a) {
     float* sh_t = wf_smem + a.max_blocks;
     __shared__ float red[4][2 * 32 * GP];
     __shared__ int scan[2][kFlatPer * 32 + 1];
-    __shared__ int hist[256];
+    __shared__ int hist[2][256];
+    __shared__ int hsum[256];
     __shared__ int sel_digit, sel_rem;
     __shared__ float arg_v[32];
     __shared__ int arg_j[32];
-    const int seg = blockIdx.x;
+    __shared__ float xf[kWideX][2 * GP];         // exchanged per-head values
+    __shared__ int xi[kWideX][2];                // exchanged integers
+    __shared__ int isum[NT / 32];
+    const int cr = kCl > 1 ? (int)cluster_rank() : 0;
+    const int seg = blockIdx.x / kCl;
     const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
     const int tid = threadIdx.x, lane = tid & 31;
     const int h = lane & (GP - 1);
@@ -716,7 +731,9 @@ prune_finalize_wide_kernel(const FinArgs a) {
     const int L = a.ctx_lens[b];
     const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
     const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
-    const int nr = (nb + RB - 1) / RB;           // rounds (the same for every thread)
+    const int nr = (nb + RB - 1) / RB;           // rounds of the segment
+    const int rsplit = (nr + kCl - 1) / kCl;
+    const int r_lo = min(nr, cr * rsplit), r_hi = min(nr, r_lo + rsplit);   // this CTA's rounds
     const long long segbase = (long long)seg * a.max_blocks;
     const float4* st = a.stats + segbase * G;
     auto stat = [&](int j) {
@@ -724,15 +741,60 @@ prune_finalize_wide_kernel(const FinArgs a) {
         if (a.score_mode == 1) v.z = v.w;        // .z: u (mode A) or sum e^{x-m} s_i (mode E)
         return v;
     };
+    int xslot = 0;
+    // sum of one int per thread over the CTA
+    auto block_sum = [&](int v) {
+        v = warp_sum_i(v);
+        if (lane == 0) isum[tid >> 5] = v;
+        __syncthreads();
+        int t = 0;
+        for (int u = 0; u < NT / 32; ++u) t += isum[u];
+        __syncthreads();
+        return t;
+    };
+    // per-head values (head h in every thread): combined over the cluster
+    auto cl_heads = [&](float* v, int N, bool is_max) {
+        if (kCl == 1) return;
+        float* x = xf[xslot++];
+        if (tid < GP)
+            for (int i = 0; i < N; ++i) x[i * GP + tid] = v[i];
+        cluster_sync();
+        for (int i = 0; i < N; ++i) {
+            float r = ld_cluster_f32(&x[i * GP + h], 0);
+            for (int p = 1; p < kCl; ++p) {
+                const float y = ld_cluster_f32(&x[i * GP + h], (uint32_t)p);
+                r = is_max ? fmaxf(r, y) : r + y;
+            }
+            v[i] = r;
+        }
+    };
+    // one integer per CTA: returns the sum over the cluster and, in *below,
+    // the sum over the lower ranks
+    auto cl_count = [&](int v, int* below) {
+        if (kCl == 1) { *below = 0; return v; }
+        int* x = xi[xslot++];
+        if (tid == 0) x[0] = v;
+        cluster_sync();
+        int tot = 0, lo = 0;
+        for (int p = 0; p < kCl; ++p) {
+            const int y = ld_cluster_s32(x, (uint32_t)p);
+            if (p < cr) lo += y;
+            tot += y;
+        }
+        *below = lo;
+        return tot;
+    };
 
+    // page ids of the segment's blocks (split over the cluster), stale stats,
+    // the per-head max
     int bad = 0;
-    for (int j = tid; j < nb; j += NT) {
+    for (int j = cr * NT + tid; j < nb; j += kCl * NT) {
         const int pg = a.block_table[(long long)b * a.max_blocks + j];
         bad |= (pg < 0 || (long long)pg >= a.num_pages);
     }
     int stale = 0;
     float Mh[1] = {-kInf};
-    for (int r = 0; r < nr; ++r)
+    for (int r = r_lo; r < r_hi; ++r)
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k) {
             const int j = r * RB + jt + k * JS;
@@ -742,9 +804,10 @@ prune_finalize_wide_kernel(const FinArgs a) {
                 Mh[0] = fmaxf(Mh[0], x);
             }
         }
-    const bool bad_page = __syncthreads_or(bad) != 0;
-    const bool timed_out = __syncthreads_or(stale) != 0 && !bad_page;
-    if (a.err && tid == 0) {
+    int dummy;
+    const bool bad_page = cl_count(__syncthreads_or(bad) != 0, &dummy) != 0;
+    const bool timed_out = cl_count(__syncthreads_or(stale) != 0, &dummy) != 0 && !bad_page;
+    if (a.err && tid == 0 && cr == 0) {
         // err was cleared before this kernel; every kv head ORs in its bits
         const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page ? ETI_ERRF_BAD_PAGE : 0u) |
                            (timed_out ? ETI_ERRF_TIMEOUT : 0u);
@@ -754,15 +817,17 @@ prune_finalize_wide_kernel(const FinArgs a) {
     float M = -kInf;
     if (n > 0) {
         head_reduce<GP, 1, true>(Mh, red[0]);
+        cl_heads(Mh, 1, true);
         M = Mh[0];
     }
 
+    const int jlo = r_lo * RB, jhi = min(n, r_hi * RB);   // this CTA's blocks of the segment
     if (!a.given) {
         if (n > 0) {
             // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
             // c_b = e^{m_b - M} (the blocks at the max are counted, not summed)
             float zs[2] = {0.f, 0.f};
-            for (int r = 0; r < nr; ++r)
+            for (int r = r_lo; r < r_hi; ++r)
 #pragma unroll
                 for (int k = 0; k < kFlatPer; ++k) {
                     const int j = r * RB + jt + k * JS;
@@ -776,6 +841,7 @@ prune_finalize_wide_kernel(const FinArgs a) {
                     }
                 }
             head_reduce<GP, 2, false>(zs, red[1]);
+            cl_heads(zs, 2, false);
             const float zm1 = zs[0] + (zs[1] - 1.f);
             const float lZ = log1pf(zm1), iZ = 1.f / (1.f + zm1);
             // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
@@ -785,7 +851,7 @@ prune_finalize_wide_kernel(const FinArgs a) {
                 return c * ((1.f + v.y) * (lZ + M - v.x) - v.z) * iZ;
             };
             float Hs[1] = {0.f};
-            for (int r = 0; r < nr; ++r)
+            for (int r = r_lo; r < r_hi; ++r)
 #pragma unroll
                 for (int k = 0; k < kFlatPer; ++k) {
                     const int j = r * RB + jt + k * JS;
@@ -797,9 +863,10 @@ prune_finalize_wide_kernel(const FinArgs a) {
                     }
                 }
             head_reduce<GP, 1, false>(Hs, red[2]);
+            cl_heads(Hs, 1, false);
             const float nH = Hs[0] > 0.f ? (float)n / Hs[0] : 0.f;
             // group score: the largest normalised term over the heads of the block
-            for (int r = 0; r < nr; ++r)
+            for (int r = r_lo; r < r_hi; ++r)
 #pragma unroll
                 for (int k = 0; k < kFlatPer; ++k) {
                     const int j = r * RB + jt + k * JS;
@@ -820,8 +887,10 @@ prune_finalize_wide_kernel(const FinArgs a) {
                 }
         }
         __syncthreads();
-        if (a.block_score)
-            for (int j = tid; j < a.max_blocks; j += NT) a.block_score[segbase + j] = j < n ? sh[j] : 0.f;
+        if (a.block_score) {
+            for (int j = jlo + tid; j < jhi; j += NT) a.block_score[segbase + j] = sh[j];
+            for (int j = n + cr * NT + tid; j < a.max_blocks; j += kCl * NT) a.block_score[segbase + j] = 0.f;
+        }
 
         // B_min budget: the first kb blocks by (score desc, index asc)
         const float th = a.theta ? a.theta[b] : kInf;
@@ -832,7 +901,7 @@ prune_finalize_wide_kernel(const FinArgs a) {
         if (kb == 1 && n > 1) {
             float bs = -kInf;
             int bj = 0x7fffffff;
-            for (int j = tid; j < n; j += NT) {
+            for (int j = jlo + tid; j < jhi; j += NT) {
                 const float v = sh[j];
                 if (v > bs || bj == 0x7fffffff) { bs = v; bj = j; }
             }
@@ -846,25 +915,49 @@ prune_finalize_wide_kernel(const FinArgs a) {
             __syncthreads();
             for (int u = 0; u < NT / 32; ++u)
                 if (arg_v[u] > bs || (arg_v[u] == bs && arg_j[u] < bj)) { bs = arg_v[u]; bj = arg_j[u]; }
+            if (kCl > 1) {
+                const int s = xslot++;
+                if (tid == 0) { xf[s][0] = bs; xi[s][0] = bj; }
+                cluster_sync();
+                bs = -kInf;
+                bj = 0x7fffffff;
+                for (int p = 0; p < kCl; ++p) {
+                    const float ov = ld_cluster_f32(&xf[s][0], (uint32_t)p);
+                    const int oj = ld_cluster_s32(&xi[s][0], (uint32_t)p);
+                    if (oj != 0x7fffffff && (ov > bs || bj == 0x7fffffff || (ov == bs && oj < bj))) { bs = ov; bj = oj; }
+                }
+            }
             arg = bj;
         } else if (kb > 1 && kb < n) {
             uint32_t prefix = 0, mask = 0;
             need = kb;
             for (int digit = 3; digit >= 0; --digit) {
                 const int shf = digit * 8;
-                for (int i = tid; i < 256; i += NT) hist[i] = 0;
+                int* hd = hist[digit & 1];
+                for (int i = tid; i < 256; i += NT) hd[i] = 0;
                 __syncthreads();
-                for (int j0 = 0; j0 < n; j0 += NT) {  // the same trip count for every lane
+                for (int j0 = jlo; j0 < jhi; j0 += NT) {  // the same trip count for every lane
                     const int j = j0 + tid;
-                    const uint32_t key = j < n ? order_key(sh[j]) : 0u;
-                    warp_hist_add(hist, (key >> shf) & 255, j < n && (key & mask) == prefix);
+                    const uint32_t key = j < jhi ? order_key(sh[j]) : 0u;
+                    warp_hist_add(hd, (key >> shf) & 255, j < jhi && (key & mask) == prefix);
+                }
+                if (kCl > 1) {
+                    cluster_sync();
+                    for (int i = tid; i < 256; i += NT) {
+                        int t = 0;
+                        for (int p = 0; p < kCl; ++p) t += ld_cluster_s32(&hd[i], (uint32_t)p);
+                        hsum[i] = t;
+                    }
+                } else {
+                    __syncthreads();
+                    for (int i = tid; i < 256; i += NT) hsum[i] = hd[i];
                 }
                 __syncthreads();
                 // bucket where the count from the top reaches `need`
                 if (tid < 32) {
                     int cnt8[8], s8 = 0;
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) { cnt8[e] = hist[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
+                    for (int e = 0; e < 8; ++e) { cnt8[e] = hsum[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
                     int incl = s8;
 #pragma unroll
                     for (int o = 1; o < 32; o <<= 1) {
@@ -889,10 +982,18 @@ prune_finalize_wide_kernel(const FinArgs a) {
             }
             kth = prefix;
         }
-        // keep flags: threshold, budget (ties at the k-th key to the lower index)
+        // keep flags: threshold, budget (ties at the k-th key to the lower index:
+        // this CTA's ties are ranked after those of the lower ranks)
         const bool sel = kb > 1 && kb < n;
         int eq_base = 0;
-        for (int r = 0; r < nr; ++r) {
+        if (sel) {
+            int eq = 0;
+            for (int j = jlo + tid; j < jhi; j += NT) eq += order_key(sh[j]) == kth;
+            int below;
+            cl_count(block_sum(eq), &below);
+            eq_base = below;
+        }
+        for (int r = r_lo; r < r_hi; ++r) {
             bool eq[kFlatPer], keep[kFlatPer];
             int eq_pos[kFlatPer];
 #pragma unroll
@@ -918,24 +1019,31 @@ prune_finalize_wide_kernel(const FinArgs a) {
         }
         __syncthreads();
     } else {
-        // given keep set: a list, a mask, or every block
+        // given keep set: a list, a mask, or every block (this CTA's blocks)
         if (a.given_idx) {
-            for (int j = tid; j < n; j += NT) sh[j] = 0.f;
+            for (int j = jlo + tid; j < jhi; j += NT) sh[j] = 0.f;
             __syncthreads();
             const int c = min(max(a.given_cnt[seg], 0), a.max_blocks);
             for (int i = tid; i < c; i += NT) {
                 const int j = a.given_idx[segbase + i];
-                if (j >= 0 && j < n) sh[j] = 1.f;
+                if (j >= jlo && j < jhi) sh[j] = 1.f;
             }
         } else {
-            for (int j = tid; j < n; j += NT) sh[j] = a.given_mask ? (a.given_mask[segbase + j] ? 1.f : 0.f) : 1.f;
+            for (int j = jlo + tid; j < jhi; j += NT)
+                sh[j] = a.given_mask ? (a.given_mask[segbase + j] ? 1.f : 0.f) : 1.f;
         }
         __syncthreads();
     }
 
-    // compaction (ascending block index), round by round
-    int total = 0;
-    for (int r = 0; r < nr; ++r) {
+    // compaction (ascending block index), round by round, after the kept
+    // blocks of the lower ranks
+    int total = 0, base = 0;
+    {
+        int cnt = 0;
+        for (int j = jlo + tid; j < jhi; j += NT) cnt += sh[j] != 0.f;
+        total = cl_count(block_sum(cnt), &base);
+    }
+    for (int r = r_lo; r < r_hi; ++r) {
         bool keep[kFlatPer];
         int pos[kFlatPer];
 #pragma unroll
@@ -947,28 +1055,29 @@ prune_finalize_wide_kernel(const FinArgs a) {
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k) {
             const int j = r * RB + jt + k * JS;
-            if (h == 0 && keep[k]) a.kept_idx[segbase + total + pos[k]] = j;
+            if (h == 0 && keep[k]) a.kept_idx[segbase + base + pos[k]] = j;
             if (a.keep_mask && h == 0 && j < n) a.keep_mask[segbase + j] = keep[k] ? 1 : 0;
         }
-        total += c;
+        base += c;
     }
-    for (int i = total + tid; i < a.max_blocks; i += NT) a.kept_idx[segbase + i] = -1;
+    for (int i = total + cr * NT + tid; i < a.max_blocks; i += kCl * NT) a.kept_idx[segbase + i] = -1;
     if (a.keep_mask)
-        for (int j = n + tid; j < a.max_blocks; j += NT) a.keep_mask[segbase + j] = 0;
-    if (tid == 0) a.kept_cnt[seg] = total;
+        for (int j = n + cr * NT + tid; j < a.max_blocks; j += kCl * NT) a.keep_mask[segbase + j] = 0;
+    if (tid == 0 && cr == 0) a.kept_cnt[seg] = total;
 
     // softmax normaliser over the kept tokens of each query head
     if (a.kept_norm) {
         float Mk[1] = {-kInf};
-        for (int r = 0; r < nr; ++r)
+        for (int r = r_lo; r < r_hi; ++r)
 #pragma unroll
             for (int k = 0; k < kFlatPer; ++k) {
                 const int j = r * RB + jt + k * JS;
                 if (h < G && j < n && sh[j] != 0.f) Mk[0] = fmaxf(Mk[0], st[(long long)j * G + h].x);
             }
         head_reduce<GP, 1, true>(Mk, red[3]);
+        cl_heads(Mk, 1, true);
         float Lk[1] = {0.f};
-        for (int r = 0; r < nr; ++r)
+        for (int r = r_lo; r < r_hi; ++r)
 #pragma unroll
             for (int k = 0; k < kFlatPer; ++k) {
                 const int j = r * RB + jt + k * JS;
@@ -978,12 +1087,38 @@ prune_finalize_wide_kernel(const FinArgs a) {
                 }
             }
         head_reduce<GP, 1, false>(Lk, red[0]);
-        if (tid < GP && h < G) {
+        cl_heads(Lk, 1, false);
+        if (tid < GP && h < G && cr == 0) {
             float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2;
             kn[0] = Mk[0];
             kn[1] = Lk[0];
         }
     }
+    // no CTA of the cluster leaves while another may still read its shared memory
+    if (kCl > 1) cluster_sync();
+}
+
+// Launch of the wide kernel for `segs` segments, kCl CTAs per segment
+// (a cluster), with programmatic dependent launch.
+template <int G, bool kTerm, int kCl>
+cudaError_t launch_wide(int segs, size_t smem, cudaStream_t stream, const FinArgs& a) {
+    auto k = prune_finalize_wide_kernel<G, kWideThreads, kTerm, kCl>;
+    if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(segs * kCl);
+    cfg.blockDim = dim3(kWideThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = kCl;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = kCl > 1 ? 2 : 1;
+    return cudaLaunchKernelEx(&cfg, k, a);
 }
 
 }  // namespace eti
@@ -1048,6 +1183,9 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     a.kept_norm = kept_norm; a.err = err;
     const int grid = B * Hkv;
     cudaError_t e = cudaSuccess;
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err && cudaMemsetAsync(err, 0, (size_t)B * sizeof(uint32_t), stream) != cudaSuccess) return ETI_ERR_CUDA;
     // the flat kernel holds a segment in registers: 16 block-heads a thread
     const int gp = a.g <= 1 ? 1 : a.g <= 2 ? 2 : a.g <= 4 ? 4 : 8;
@@ -1069,11 +1207,17 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
         ETI_FIN_FLAT(GG, 512)                                                               \
         const size_t smem_t = (size_t)max_blocks * 4 * (1 + gp);                           \
         const bool term = !given && smem_t <= kWideSmemMax;                                 \
-        auto k = term ? prune_finalize_wide_kernel<GG, kWideThreads, true>                  \
-                      : prune_finalize_wide_kernel<GG, kWideThreads, false>;                \
         const size_t smem = term ? smem_t : (size_t)max_blocks * 4;                         \
-        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-        e = eti_launch_pdl(k, dim3(grid), dim3(kWideThreads), smem, stream, a);             \
+        /* long segments and fewer of them than half the SMs: a pair of CTAs each */       \
+        const bool pair = 2 * grid <= sms && max_blocks > (kWideThreads / gp) * kFlatPer;  \
+        if (pair) {                                                                         \
+            e = term ? launch_wide<GG, true, 2>(grid, smem, stream, a)                      \
+                     : launch_wide<GG, false, 2>(grid, smem, stream, a);                    \
+            if (e == cudaSuccess) break;                                                    \
+            (void)cudaGetLastError();  /* cluster launch refused: one CTA per segment */    \
+        }                                                                                   \
+        e = term ? launch_wide<GG, true, 1>(grid, smem, stream, a)                          \
+                 : launch_wide<GG, false, 1>(grid, smem, stream, a);                        \
         break;                                                                              \
     }
     switch (a.g) {
