@@ -220,6 +220,14 @@ def run_schedule(eti, step, kv, w, stream, reps=50):
     return round(statistics.median(e[0].elapsed_time(e[1]) for e in ev), 5)
 
 
+def ctx_desc(w) -> str:
+    """The workload's context-length distribution, as printed in `config`."""
+    kind = w.ctx[0]
+    if kind == "list":
+        return "ctx " + "/".join(str(x) for x in w.ctx[1])
+    return f"ctx {'log-U' if kind == 'loguniform' else 'U'}[{w.ctx[1]},{w.ctx[2]}]"
+
+
 def run_keep_sweep(eti, device, flush_l2, stream, peak, fracs=(0.1, 0.25, 0.5, 1.0), reps=10):
     """The long-context step of the paper's sweep (8 sequences, contexts
     U[32768, 131072]): theta = +inf and B_min = ceil(f * n_b) of the longest
@@ -295,7 +303,7 @@ def run_keep_sweep(eti, device, flush_l2, stream, peak, fracs=(0.1, 0.25, 0.5, 1
     del kv, st, stats, ws_dense, out_dense
     torch.cuda.empty_cache()
     return {"workload": f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} D={w.D} P={w.P} "
-                        f"ctx U[{w.ctx[1]},{w.ctx[2]}]",
+                        f"{ctx_desc(w)}",
             "theta": "+inf", "score_ms": round(score_ms, 5),
             "score_gbs": round(sbytes / (score_ms / 1e3) / 1e9, 1),
             "dense_decode_ms": round(dense_ms, 5),
@@ -447,7 +455,7 @@ def run_gpu(args):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16/fp32",
         "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
         "config": {"workload": f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} D={w.D} P={w.P} "
-                               f"ctx U[{w.ctx[1]},{w.ctx[2]}] V={w.V}",
+                               f"{ctx_desc(w)} V={w.V}",
                    "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write, then 2x L2 read)",
                    "parallelism": f"replicas x{world} (independent batches)", "B_min": B_min,
                    "theta": "theta_next of the step's own entropy (defaults)",

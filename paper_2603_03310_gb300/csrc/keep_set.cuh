@@ -1,0 +1,114 @@
+// keep_set.cuh -- shared pieces of the keep-set kernels (Section 3.2: block
+// scores, the threshold / budget rule, compaction, the kept-token softmax
+// normaliser): the argument block, the order-preserving key, and the
+// per-head reductions and ranks of the flat layout (thread t owns query head
+// t % GP of its blocks).
+#pragma once
+
+#include "common.cuh"
+
+namespace eti {
+
+struct FinArgs {
+    const float4* stats;
+    const int32_t* ctx_lens;
+    const int32_t* block_table;
+    long long num_pages;
+    int B, Hq, Hkv, g, P, max_blocks;
+    // rule mode (given == 0)
+    const float* theta;
+    int B_min;
+    int score_mode;         // 0 A: I_i = -log a_i; 1 E: stored surprisal; 2 M: 1
+    // given mode: keep set from a list or a mask (or every block)
+    int given;
+    const uint8_t* given_mask;
+    const int32_t* given_idx;
+    const int32_t* given_cnt;
+    // outputs
+    uint8_t* keep_mask;     // nullable
+    int32_t* kept_idx;
+    int32_t* kept_cnt;
+    float* block_score;     // nullable
+    float* kept_norm;       // nullable: [B][Hq][2]
+    uint32_t* err;          // nullable
+};
+
+__device__ __forceinline__ uint32_t order_key(float f) {
+    if (f != f) return 0u;
+    const uint32_t b = __float_as_uint(f);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+constexpr int kFlatPer = 16;
+constexpr int kWideThreads = 1024;
+constexpr size_t kWideSmemMax = 200 * 1024;   // dynamic shared memory of the cached-term variant
+
+template <int G>
+struct FlatGP { static constexpr int v = G <= 1 ? 1 : G <= 2 ? 2 : G <= 4 ? 4 : 8; };
+
+// per-head reduction of N values over the lanes (and warps) of equal h;
+// red holds N * 32 * GP floats and must not be reused before the next barrier
+template <int GP, int N, bool kMax>
+__device__ __forceinline__ void head_reduce(float (&v)[N], float* red) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int o = 16; o >= GP; o >>= 1)
+#pragma unroll
+        for (int i = 0; i < N; ++i) {
+            const float y = __shfl_xor_sync(0xffffffffu, v[i], o);
+            v[i] = kMax ? fmaxf(v[i], y) : v[i] + y;
+        }
+    if (lane < GP)
+#pragma unroll
+        for (int i = 0; i < N; ++i) red[(i * 32 + w) * GP + lane] = v[i];
+    __syncthreads();
+    const int h = lane & (GP - 1);
+#pragma unroll
+    for (int i = 0; i < N; ++i) {
+        float r = kMax ? -kInf : 0.f;
+        for (int u = 0; u < nw; ++u) {
+            const float y = red[(i * 32 + u) * GP + h];
+            r = kMax ? fmaxf(r, y) : r + y;
+        }
+        v[i] = r;
+    }
+}
+
+// Exclusive ranks in ascending block order of the flagged blocks (flags
+// agree across the GP lanes of a block); returns the number flagged.
+// scan holds kFlatPer * 32 + 1 ints.
+template <int GP>
+__device__ __forceinline__ int flat_ranks(const bool (&f)[kFlatPer], int (&pos)[kFlatPer], int* scan) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    const bool lead = (lane & (GP - 1)) == 0;
+    const uint32_t below = (1u << (lane & ~(GP - 1))) - 1u;   // lanes of earlier blocks
+    uint32_t bal[kFlatPer];
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) {
+        bal[k] = __ballot_sync(0xffffffffu, f[k] && lead);
+        if (lane == 0) scan[k * nw + w] = __popc(bal[k]);
+    }
+    __syncthreads();
+    if (w == 0) {
+        // exclusive scan of the (chunk, warp) counts, chunk-major
+        const int E = kFlatPer * nw, per = (E + 31) >> 5;
+        const int e0 = min(lane * per, E), e1 = min(e0 + per, E);
+        int s = 0;
+        for (int e = e0; e < e1; ++e) s += scan[e];
+        int x = s;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        int run = x - s;
+        for (int e = e0; e < e1; ++e) { const int c = scan[e]; scan[e] = run; run += c; }
+        if (lane == 31) scan[E] = x;
+    }
+    __syncthreads();
+#pragma unroll
+    for (int k = 0; k < kFlatPer; ++k) pos[k] = scan[k * nw + w] + __popc(bal[k] & below);
+    return scan[kFlatPer * nw];
+}
+
+}  // namespace eti
