@@ -154,18 +154,30 @@ def algorithmic_bytes(w, L: np.ndarray, kept_blocks: int) -> dict:
     }
 
 
+def source_digest(paths) -> str:
+    """sha256 of the code of these source files: comments and blank lines are
+    left out, so a change of wording is not a change of kernel."""
+    import hashlib
+    import re
+    h = hashlib.sha256()
+    for path in paths:
+        with open(os.path.join(ROOT, path)) as f:
+            for line in f:
+                code = re.sub(r"/\*.*?\*/", "", line).split("//")[0].strip()
+                if code:
+                    h.update(code.encode() + b"\n")
+    return h.hexdigest()
+
+
 def ncu_traffic(kernel):
     """DRAM bytes per launch from the committed ncu record, if the kernel's
-    source is unchanged since that capture (else None)."""
-    import hashlib
+    code is unchanged since that capture (else None)."""
     try:
         rec = json.load(open(os.path.join(ROOT, "profiles", "ncu_traffic.json")))[kernel]
-        h = hashlib.sha256()
-        for path in rec["sources"]:
-            h.update(open(os.path.join(ROOT, path), "rb").read())
+        digest = source_digest(rec["sources"])
     except (OSError, KeyError, TypeError, ValueError):
         return None
-    return rec["bytes"] if h.hexdigest() == rec["sha256"] else None
+    return rec["bytes"] if digest == rec["sha256"] else None
 
 
 def run_estimators(eti, lg, step, prm, w, flush_l2, stream, k=64, reps=50):

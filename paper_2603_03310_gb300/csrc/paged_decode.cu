@@ -17,9 +17,10 @@
 // with the 128-byte swizzle, so the fragment reads below are conflict-free)
 // and a 1-D bulk copy of the tile's scores per stage, completing on the
 // stage's mbarrier; every wait is bounded.  Page ids are resolved 32 blocks at
-// a time, one lane per block, into a small table a batch ahead of use.  p.V runs on bf16 m16n8k16 tensor-core tiles
-// (head_dim = M, query heads = N, tokens = K): V rows are transposed into A
-// fragments with byte permutes, the probabilities form the B fragment.
+// a time, one lane per block, into a small table a batch ahead of use.  p.V
+// runs on bf16 m16n8k16 tensor-core tiles (head_dim = M, query heads = N,
+// tokens = K): each A fragment (V^T, 16 x 16) is one ldmatrix.x4.trans from
+// the swizzled stage, the probabilities form the B fragment.
 // A segment that lies inside one warp's range is written straight to `out`;
 // otherwise the warp's part goes to partial slot (warp + segment), and the
 // warp that closes the segment's ticket last adds its slots in warp order

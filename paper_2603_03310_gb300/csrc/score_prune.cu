@@ -3,15 +3,17 @@
 // score_blocks (the HBM-bound pass): every key page chunk (page, kv head) is
 // read exactly once.  Warps walk a flattened list of (sequence, kv head,
 // block) units, each warp taking an equal contiguous share (no idle tail);
-// a unit is P/16 tiles of 16 tokens x D.  Each tile is loaded straight into
-// registers with 128-bit streaming loads in the A-fragment order of a bf16
-// m16n8k16 tensor-core tile (tokens = M, query heads of the GQA group = N,
-// head_dim = K; the K index is permuted identically in the key and query
-// fragments, so a thread's 16-byte load feeds two MMAs), and the next tile's
-// loads are issued before the current tile is consumed.  Per block and query
-// head it emits the stats (m_b, l_b, u_b) = (max x, sum e^{x-m_b},
-// sum e^{x-m_b}(x-m_b)) and, optionally, the scaled scores x_i themselves so
-// the decode pass never reads a key page again.
+// a unit is P/16 tiles of 16 tokens x D.  Each warp streams its tiles through
+// a private ring of shared-memory stages filled by the Tensor Memory
+// Accelerator (one lane issues 2-D tiled copies of 64-element boxes with the
+// 128-byte swizzle, completing on the stage's mbarrier; every wait is
+// bounded and a stage that never arrives is reported as a timeout).  q.k^T
+// runs on bf16 m16n8k16 tensor-core tiles (tokens = M, query heads of the
+// GQA group = N, head_dim = K) read conflict-free from the swizzled stage.
+// Per block and query head it emits the stats (m_b, l_b - 1, u_b, e_b) =
+// (max x, sum e^{x-m_b} - 1 kept exact, sum e^{x-m_b}(x-m_b), and for score
+// mode E sum e^{x-m_b} s_i) and, optionally, the scaled scores x_i
+// themselves so the decode pass never reads a key page again.
 //
 // prune_finalize (one CTA per (sequence, kv head)): with M = max_b m_b and
 // Z = sum_b l_b e^{m_b - M}, the block term of the attention entropy is
@@ -20,7 +22,9 @@
 // over the block stats (both bracket terms are >= 0, so no cancellation).
 // Then the normalised group score, the threshold, the B_min budget (radix
 // select, ties to the lower block index), compaction, and the kept-token
-// softmax normaliser (max, sum) that the decode pass uses.
+// softmax normaliser (max, sum) that the decode pass uses.  This file holds
+// the flat kernel (a segment held in registers); longer segments and the
+// given keep sets of a standalone decode go to prune_wide.cu.
 #include "common.cuh"
 #include "keep_set.cuh"
 
