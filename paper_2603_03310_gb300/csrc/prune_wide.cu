@@ -148,6 +148,7 @@ prune_finalize_wide_kernel(const FinArgs a) {
     }
 
     const int jlo = r_lo * RB, jhi = min(n, r_hi * RB);   // this CTA's blocks of the segment
+    int kbase = 0;                               // kept blocks listed so far (one-CTA rule mode)
     if (!a.given) {
         if (n > 0) {
             // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
@@ -336,6 +337,19 @@ prune_finalize_wide_kernel(const FinArgs a) {
                 for (int k = 0; k < kFlatPer; ++k) keep[k] |= eq[k] && eq_base + eq_pos[k] < need;
                 eq_base += c;
             }
+            if (kCl == 1) {
+                // one CTA: the ranks of this round follow those of the rounds
+                // before it, so the kept list is written here
+                int pos[kFlatPer];
+                const int c = flat_ranks<GP>(keep, pos, scan[(r + 1) & 1]);
+#pragma unroll
+                for (int k = 0; k < kFlatPer; ++k) {
+                    const int j = r * RB + jt + k * JS;
+                    if (h == 0 && keep[k]) a.kept_idx[segbase + kbase + pos[k]] = j;
+                    if (a.keep_mask && h == 0 && j < n) a.keep_mask[segbase + j] = keep[k] ? 1 : 0;
+                }
+                kbase += c;
+            }
             __syncthreads();    // every lane of a block has read its score
 #pragma unroll
             for (int k = 0; k < kFlatPer; ++k) {
@@ -362,14 +376,15 @@ prune_finalize_wide_kernel(const FinArgs a) {
     }
 
     // compaction (ascending block index), round by round, after the kept
-    // blocks of the lower ranks
-    int total = 0, base = 0;
-    {
+    // blocks of the lower ranks (one-CTA rule mode: done with the flags)
+    const bool listed = kCl == 1 && !a.given;
+    int total = kbase, base = 0;
+    if (!listed) {
         int cnt = 0;
         for (int j = jlo + tid; j < jhi; j += NT) cnt += sh[j] != 0.f;
         total = cl_count(block_sum(cnt), &base);
     }
-    for (int r = r_lo; r < r_hi; ++r) {
+    for (int r = listed ? r_hi : r_lo; r < r_hi; ++r) {
         bool keep[kFlatPer];
         int pos[kFlatPer];
 #pragma unroll
