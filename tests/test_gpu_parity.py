@@ -286,6 +286,45 @@ def test_attention_maximum_batch(eti):
     print(s)
 
 
+@pytest.mark.parametrize("mode", ["dense", "mask", "lists"])
+def test_standalone_decode_long_segments(eti, mode):
+    """eti_paged_decode without precomputed scores on segments of up to 8192
+    blocks: its internal keep-set pass takes the wide kernel on a pair of CTAs
+    per segment; dense, from a mask, from lists."""
+    w = workloads.Workload("dl", B=2, Hq=32, Hkv=8, D=128, P=16, V=16, ctx=("list", [40000, 131072]),
+                           seed=17, hi_frac=0.02)
+    kv = workloads.make_kv(w, DEV)
+    n = parity.host_kv(kv)
+    rng = np.random.default_rng(3)
+    mask = (rng.random((w.B, w.Hkv, w.max_blocks)) < 0.3).astype(np.uint8)
+    for b, L in enumerate(n["L"]):
+        mask[b, :, -(-int(L) // w.P):] = 0
+    out = torch.empty((w.B, w.Hq, w.D), dtype=torch.bfloat16, device=DEV)
+    err = torch.empty(w.B, dtype=torch.int32, device=DEV)
+    ws = torch.empty(eti.paged_decode_workspace_size(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, False),
+                     dtype=torch.uint8, device=DEV)
+    kw = {}
+    if mode == "mask":
+        kw["keep_mask"] = torch.from_numpy(mask).to(DEV)
+    elif mode == "lists":
+        idx = np.full(mask.shape, -1, np.int32)
+        cnt = mask.sum(-1).astype(np.int32)
+        for b in range(w.B):
+            for h in range(w.Hkv):
+                nz = np.nonzero(mask[b, h])[0]
+                rng.shuffle(nz)                       # any order is accepted
+                idx[b, h, :len(nz)] = nz
+        kw["kept_idx"] = torch.from_numpy(idx).to(DEV)
+        kw["kept_cnt"] = torch.from_numpy(cnt).to(DEV)
+    eti.eti_paged_decode(kv["q"], kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
+                         kv["scale"], out, err, ws, num_pages=kv["num_pages"], **kw)
+    torch.cuda.synchronize()
+    ref, rerr = oracle.paged_attention(n["q"], n["k"], n["v"], n["bt"], n["L"], n["scale"],
+                                       None if mode == "dense" else mask, num_pages=n["num_pages"])
+    print(mode, parity.compare_attention(out.float().cpu().numpy(), ref))
+    assert np.array_equal(err.cpu().numpy().view(np.uint32), rerr)
+
+
 def test_attention_edge_cases(eti):
     """Empty sequences, a bad page id and a bad context length: error bits and zero outputs."""
     w = workloads.Workload("e", B=4, Hq=8, Hkv=2, D=64, P=16, V=16, ctx=("list", [0, 40, 40, 40]),
