@@ -211,3 +211,26 @@ def test_prune_long_segment_without_term_cache(eti):
     got = _score_prune(eti, w, kv, th, 700, 0, None)
     s = _check(got, parity.host_kv(kv), None, th.cpu().numpy(), 700, 0)
     print(s)
+
+
+@pytest.mark.parametrize("B_min", [3000, 5000])
+def test_budget_ties_across_a_cluster(eti, B_min):
+    """q = 0 gives every full block the same stats, hence bitwise-equal group
+    scores: with theta = +inf the kept blocks of every head are exactly blocks
+    0..B_min-1, whichever CTA of the pair holds them (8192 blocks: the
+    segment is split between two CTAs at block 4096, so B_min = 5000 takes
+    all of the first CTA's blocks and the first 904 of the second's)."""
+    w = workloads.Workload("tie", B=1, Hq=32, Hkv=8, D=128, P=16, V=16, ctx=("list", [131072]), seed=41,
+                           hi_frac=0.0)
+    kv = workloads.make_kv(w, DEV)
+    kv["q"].zero_()
+    th = torch.full((w.B,), float("inf"), dtype=torch.float32, device=DEV)
+    got = _score_prune(eti, w, kv, th, B_min, 0, None)
+    want = np.zeros((w.B, w.Hkv, w.max_blocks), np.uint8)
+    want[:, :, :B_min] = 1
+    assert np.array_equal(got["keep_mask"], want)
+    assert (got["kept_cnt"] == B_min).all()
+    assert np.array_equal(got["kept_idx"][:, :, :B_min], np.broadcast_to(np.arange(B_min), (w.B, w.Hkv, B_min)))
+    assert (got["kept_idx"][:, :, B_min:] == -1).all()
+    sc = got["block_score"][0, :, :8192]
+    assert (sc == sc[:, :1]).all()                  # every block the same score, bit for bit
