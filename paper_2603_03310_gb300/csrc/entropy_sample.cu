@@ -4,11 +4,11 @@
 // threshold (Section 3.2 safety floor, Section 5 entropy floor) and a
 // Gumbel-max draw from p_t, in ONE pass over the fp32 logits.
 //
-// Decomposition: a persistent grid (4 CTAs of 256 threads per SM) in which
+// Decomposition: a persistent grid (8 CTAs of 128 threads per SM) in which
 // every CTA takes an equal contiguous share of the row-major list of all
 // rows' 4-token groups, so every SM finishes at the same time whatever B and
 // V are.  A CTA walks its share one row piece at a time, in steps of two
-// groups per thread (thread t takes groups base + 256 k + t, so its tokens are
+// groups per thread (thread t takes groups base + 128 k + t, so its tokens are
 // visited in increasing index order), with the next step's 16-byte loads in
 // flight while the current one is processed.  Each thread keeps the online
 // state
@@ -235,10 +235,10 @@ struct EtsArgs {
     RowState* part;       // [grid + B] partial states, slot (cta + row)
 };
 
-constexpr int kEtsThreads = 256;
+constexpr int kEtsThreads = 128;
 constexpr int kEtsWarps = kEtsThreads / 32;
 constexpr int kEtsPair = 2;        // 4-token groups per thread per step
-constexpr int kEtsCtasPerSm = 4;
+constexpr int kEtsCtasPerSm = 8;
 constexpr float kFrameMax = 4096.f;   // |mc| above which lr loses the 2^-10 margin
 
 // order-preserving int key of a float (and back); key(-inf) marks "no bound"
