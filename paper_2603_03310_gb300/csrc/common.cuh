@@ -55,6 +55,27 @@ __device__ __forceinline__ float fast_ex2(float x) {
     return y;
 }
 
+// Whether any page id row[j], j = first, first + stride, ... < n, lies
+// outside [0, num_pages).  Eight loads per thread are issued before any is
+// tested, so a long row costs a few memory round trips, not one per id.
+__device__ __forceinline__ bool any_bad_page(const int32_t* row, int first, int stride, int n,
+                                             long long num_pages) {
+    constexpr int kU = 8;
+    bool bad = false;
+    for (int j0 = first; j0 < n; j0 += kU * stride) {
+        int pg[kU];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            const int j = j0 + u * stride;
+            pg[u] = j < n ? __ldg(row + j) : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < kU; ++u)
+            bad |= j0 + u * stride < n && (pg[u] < 0 || (long long)pg[u] >= num_pages);
+    }
+    return bad;
+}
+
 // 1/x, hardware approximation (MUFU.RCP); 1/0 = +inf.
 __device__ __forceinline__ float fast_rcp(float x) {
     float y;

@@ -429,6 +429,14 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
     const float c = bad_T ? 0.f : kLog2e / T;
     const long long lo = (long long)b * a.ngroups, hi = lo + a.ngroups - 1;
     const int c0 = (int)(lo / a.share), c1 = (int)(hi / a.share);
+    // the per-row inputs of the epilogue, loaded while the slots are merged
+    float tau_in = 0.f, H_prev = 0.f, H_tgt = 0.f, th_prev = 0.f;
+    if (lane == 0) {
+        tau_in = a.tau[b];
+        H_prev = a.H_prev[b];
+        H_tgt = a.H_target[b];
+        if (a.theta_next && a.p.dtheta > 0.f) th_prev = a.theta_next[b];
+    }
     // lane l merges slots c0 + l, c0 + l + 32, ... in order, then the lanes merge
     // in a fixed tree: the result does not depend on timing
     RowState s;
@@ -449,7 +457,6 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
         if (t.m == -kInf) err = ETI_ERRF_ALL_NEG_INF;
         else if (t.m == kInf || isnan(t.R) || isnan(t.U)) err = ETI_ERRF_NONFINITE;
     }
-    const float tau_in = a.tau[b];
     if (err) {
         a.tok[b] = -1;
         a.H[b] = __int_as_float(0x7fc00000);
@@ -464,9 +471,9 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
         const float q = fmaf(t.nt, fmaf(t.m, c, -mc) * kLn2, t.R) / t.nt;
         const float lnS = logf(t.nt) + log1pf(q);
         const float H = fmaxf(lnS - kLn2 * t.U / (t.nt * (1.f + q)), 0.f);
-        const float dH = a.H_prev[b] - H;
+        const float dH = H_prev - H;
         a.tau[b] = tau_in + fmaxf(dH, 0.f);
-        float Tn = Tt * expf(a.p.sign * a.p.eta * (H - a.H_target[b]));
+        float Tn = Tt * expf(a.p.sign * a.p.eta * (H - H_tgt));
         if (a.p.rho_T > 0.f) Tn = fminf(Tt * expf(a.p.rho_T), fmaxf(Tt * expf(-a.p.rho_T), Tn));
         Tn = fminf(a.p.T_max, fmaxf(a.p.T_min, Tn));
         a.tok[b] = t.bi;
@@ -479,7 +486,7 @@ entropy_sample_finalize_kernel(const EtsArgs a) {
                                        : a.p.theta_hi;
             float th = fminf(a.p.theta_user, tmax);
             if (a.p.dtheta > 0.f) {
-                const float tp = a.theta_next[b];   // the previous threshold, in place
+                const float tp = th_prev;   // the previous threshold, in place
                 if (isfinite(tp)) th = fminf(tp + a.p.dtheta, fmaxf(tp - a.p.dtheta, th));
             }
             a.theta_next[b] = th;

@@ -38,6 +38,7 @@ namespace eti {
 constexpr int kDecWarps = 8;
 constexpr int kDecThreads = kDecWarps * 32;
 constexpr int kPlanThreads = 1024;
+constexpr int kPlanSmemSeg = 4096;   // segments whose prefix the plan keeps in shared memory
 
 // --------------------------------------------------------------------------
 // plan: prefix of kept counts, the per-warp share, each warp's first
@@ -67,16 +68,13 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
         const int L = a.ctx_lens[b];
         const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
         const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
-        int bad = 0;
-        for (int j = lane; j < nb; j += 32) {
-            const int pg = a.block_table[(long long)b * a.max_blocks + j];
-            bad |= (pg < 0 || (long long)pg >= a.num_pages);
-        }
-        bad = __any_sync(0xffffffffu, bad);
+        const bool bad = __any_sync(0xffffffffu, any_bad_page(a.block_table + (long long)b * a.max_blocks,
+                                                              lane, 32, nb, a.num_pages));
         if (lane == 0) a.err[b] = bad_ctx ? ETI_ERRF_BAD_CTX : (bad ? ETI_ERRF_BAD_PAGE : 0u);
         return;
     }
     __shared__ int wsum[kPlanThreads / 32];
+    __shared__ int scum[kPlanSmemSeg + 1];   // cum[0 .. kPlanSmemSeg], kept for the second loop
     int carry = 0;
     for (int base = 0; base < a.nseg; base += kPlanThreads) {
         const int s = base + tid;
@@ -97,6 +95,7 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
         if (s < a.nseg) {
             a.cum[s] = carry + ofs + x - v;
             a.ticket[s] = 0;
+            if (s <= kPlanSmemSeg) scum[s] = carry + ofs + x - v;
         }
         carry += tot;
         __syncthreads();
@@ -106,6 +105,7 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
     // merge of many small split parts cost more than the extra warps bring
     const int share = max(32, (total + a.nwarps - 1) / a.nwarps);
     if (tid == 0) {
+        if (a.nseg <= kPlanSmemSeg) scum[a.nseg] = total;
         a.cum[a.nseg] = total;
         a.info[0] = total;
         a.info[1] = share;
@@ -113,7 +113,8 @@ __global__ void __launch_bounds__(kPlanThreads) decode_plan_kernel(const PlanArg
     for (int c = tid; c < a.nwarps; c += kPlanThreads) a.warp_seg[c] = a.nseg;
     __syncthreads();
     for (int s = tid; s < a.nseg; s += kPlanThreads) {
-        const int lo = a.cum[s], hi = a.cum[s + 1];
+        const int lo = s + 1 <= kPlanSmemSeg ? scum[s] : a.cum[s];
+        const int hi = s + 1 <= kPlanSmemSeg ? scum[s + 1] : a.cum[s + 1];
         if (hi <= lo) continue;
         const int c0 = (lo + share - 1) / share, c1 = min((hi + share - 1) / share, a.nwarps);
         for (int c = c0; c < c1; ++c) a.warp_seg[c] = s;

@@ -113,11 +113,8 @@ prune_finalize_wide_kernel(const FinArgs a) {
 
     // page ids of the segment's blocks (split over the cluster), stale stats,
     // the per-head max
-    int bad = 0;
-    for (int j = cr * NT + tid; j < nb; j += kCl * NT) {
-        const int pg = a.block_table[(long long)b * a.max_blocks + j];
-        bad |= (pg < 0 || (long long)pg >= a.num_pages);
-    }
+    const int bad = any_bad_page(a.block_table + (long long)b * a.max_blocks, cr * NT + tid, kCl * NT, nb,
+                                 a.num_pages);
     int stale = 0;
     float Mh[1] = {-kInf};
     for (int r = r_lo; r < r_hi; ++r)

@@ -364,11 +364,7 @@ prune_finalize_flat_kernel(const FinArgs a) {
     const long long segbase = (long long)seg * a.max_blocks;
     const float4* st = a.stats + segbase * G;
 
-    int bad = 0;
-    for (int j = tid; j < nb; j += NT) {
-        const int pg = a.block_table[(long long)b * a.max_blocks + j];
-        bad |= (pg < 0 || (long long)pg >= a.num_pages);
-    }
+    const int bad = any_bad_page(a.block_table + (long long)b * a.max_blocks, tid, NT, nb, a.num_pages);
     float m[kFlatPer], l1[kFlatPer], w[kFlatPer];   // w: u_b, then the block term I_b
     int stale = 0;
     float Mh[1] = {-kInf};
@@ -420,24 +416,25 @@ prune_finalize_flat_kernel(const FinArgs a) {
             }
         head_reduce<GP, 2, false>(zs, red[1]);
         const float zm1 = zs[0] + (zs[1] - 1.f);
-        const float lZ = log1pf(zm1), Z = 1.f + zm1;
+        const float lZ = log1pf(zm1), iZ = 1.f / (1.f + zm1);
         // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
         // (l1 becomes (1 + l1_b) e^{m_b - M}, the block's share of Z)
         float Hs[1] = {0.f};
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k)
             if (valid[k]) {
-                if (a.score_mode == 1) w[k] = c[k] * w[k] / Z;                 // E
-                else if (a.score_mode == 2) w[k] = c[k] * (1.f + l1[k]) / Z;   // M
-                else w[k] = c[k] * ((1.f + l1[k]) * (lZ + M - m[k]) - w[k]) / Z;
+                if (a.score_mode == 1) w[k] = c[k] * w[k] * iZ;                 // E
+                else if (a.score_mode == 2) w[k] = c[k] * (1.f + l1[k]) * iZ;   // M
+                else w[k] = c[k] * ((1.f + l1[k]) * (lZ + M - m[k]) - w[k]) * iZ;
                 Hs[0] += w[k];
                 l1[k] = (1.f + l1[k]) * c[k];
             }
         head_reduce<GP, 1, false>(Hs, red[2]);
+        const float nH = Hs[0] > 0.f ? (float)n / Hs[0] : 0.f;
         // group score: the largest normalised term over the heads of the block
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k) {
-            float s = valid[k] ? (Hs[0] > 0.f ? (float)n * w[k] / Hs[0] : 1.f) : -kInf;
+            float s = valid[k] ? (Hs[0] > 0.f ? w[k] * nH : 1.f) : -kInf;
 #pragma unroll
             for (int o = 1; o < GP; o <<= 1) s = fmaxf(s, __shfl_xor_sync(0xffffffffu, s, o));
             score[k] = s;
@@ -559,17 +556,23 @@ prune_finalize_flat_kernel(const FinArgs a) {
             if (valid[k] && keep[k]) Mk[0] = fmaxf(Mk[0], m[k]);
         head_reduce<GP, 1, true>(Mk, red[3]);
         float Lk[1] = {0.f};
+        if (Mk[0] == M) {
 #pragma unroll
-        for (int k = 0; k < kFlatPer; ++k)
-            if (valid[k] && keep[k]) {
-                if (Mk[0] == M) {
-                    Lk[0] += l1[k];
-                } else {
-                    // the largest logit's block was pruned: rescale from the stats
+            for (int k = 0; k < kFlatPer; ++k)
+                if (valid[k] && keep[k]) Lk[0] += l1[k];
+        } else {
+            // the largest logit's block was pruned: rescale from the stats
+            // (a rolled loop: this path is rare and its code stays small)
+            uint32_t kk = 0;
+#pragma unroll
+            for (int k = 0; k < kFlatPer; ++k) kk |= (valid[k] && keep[k]) ? 1u << k : 0u;
+#pragma unroll 1
+            for (int k = 0; k < kFlatPer; ++k)
+                if ((kk >> k) & 1u) {
                     const float4 s = st[(long long)(jt + k * JS) * G + h];
                     Lk[0] += (1.f + s.y) * expf(s.x - Mk[0]);
                 }
-            }
+        }
         head_reduce<GP, 1, false>(Lk, red[0]);
         if (tid < GP && h < G) {
             float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2;
