@@ -480,11 +480,10 @@ def run_gpu(args):
         "entropy_sample_gbs": round(achieved["sample"], 1),
         "attention_tbs": round((abytes["score"] + abytes["decode"]) /
                                ((mean_ms["score"] + mean_ms["prune"] + mean_ms["decode"]) / 1e3) / 1e12, 3),
-        "gpu_launches": 6 * args.steps,
-        "launches_per_step": {"score_blocks": 1, "prune_finalize": 1, "decode_plan": 1,
-                              "paged_decode": 1,
-                              "entropy_sample_partial": 1, "entropy_sample_finalize": 1,
-                              "memset (error flags, not a kernel of the library)": 1},
+        "gpu_launches": 7 * args.steps,
+        "launches_per_step": {"score_blocks": 1, "clear_words (keep-set error words)": 1,
+                              "prune_finalize": 1, "decode_plan": 1, "paged_decode": 1,
+                              "entropy_sample_partial": 1, "entropy_sample_finalize": 1},
         "e2e": e2e,
         "estimators": est,
         "keep_sweep": sweep,

@@ -328,6 +328,17 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
 }
 
 // ---------------------------------------------------------------------------
+// Zeroes the per-sequence error words before the keep-set kernel ORs its bits
+// in (every kv head of a sequence adds its own).  A kernel, not a memset: a
+// memset node in a captured CUDA graph cost about 30 us per replay here, and
+// after a kernel the keep-set kernel keeps its programmatic launch overlap.
+__global__ void __launch_bounds__(256) clear_words_kernel(uint32_t* w, int n) {
+    pdl_trigger();
+    pdl_wait();
+    for (int i = blockIdx.x * 256 + threadIdx.x; i < n; i += gridDim.x * 256) w[i] = 0u;
+}
+
+// ---------------------------------------------------------------------------
 // prune_finalize for segments of up to 16 * NT block-heads, one CTA of NT
 // threads per (sequence, kv head).  Flat layout: with GP the power of two
 // >= G, thread t owns query head h = t % GP of the blocks j = t / GP +
@@ -649,7 +660,15 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    if (err && cudaMemsetAsync(err, 0, (size_t)B * sizeof(uint32_t), stream) != cudaSuccess) return ETI_ERR_CUDA;
+    if (err) {
+        // a plain launch (it waits for the kernel before it, as a memset
+        // would); the keep-set kernel then overlaps its own launch with it
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((B + 255) / 256);
+        cfg.blockDim = dim3(256);
+        cfg.stream = stream;
+        if (cudaLaunchKernelEx(&cfg, clear_words_kernel, err, B) != cudaSuccess) return ETI_ERR_CUDA;
+    }
     // the flat kernel holds a segment in registers: 16 block-heads a thread
     const int gp = a.g <= 1 ? 1 : a.g <= 2 ? 2 : a.g <= 4 ? 4 : 8;
     const long long flat_need = ((long long)max_blocks * gp + kFlatPer - 1) / kFlatPer;
