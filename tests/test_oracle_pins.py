@@ -6,6 +6,7 @@ torch's scaled-dot-product attention, Triton's Philox), or a statistical law
 (the Gumbel-max theorem).  CPU only.
 """
 import math
+import os
 
 import numpy as np
 import pytest
@@ -247,6 +248,18 @@ def test_threshold_floor():
 
 # ----------------------------------------------------------------------------
 # Sampler: Philox4x32-10 and the Gumbel-max draw
+
+def test_philox_known_answers():
+    """The published Philox4x32-10 known-answer values (tests/golden, cited there):
+    zero counter and key, all-ones counter and key, and the digits-of-pi case."""
+    path = os.path.join(os.path.dirname(__file__), "golden", "philox4x32_10_kat.txt")
+    rows = [l for l in open(path).read().splitlines() if l.strip() and not l.startswith("#")]
+    assert len(rows) == 3
+    for row in rows:
+        ctr, key, want = ([int(w, 16) for w in part.split()] for part in row.split("|"))
+        got = oracle.philox4x32_10(np.array(ctr, np.uint32), np.array(key, np.uint32)).reshape(-1)
+        assert [int(x) for x in got] == want, row
+
 
 def test_philox_matches_tritons_independent_implementation():
     """Triton's Philox4x32-10 (run by its CPU interpreter) on random counters and 64-bit keys."""
