@@ -400,8 +400,10 @@ def run_gpu(args):
         import torch.distributed as dist
         dist.barrier()
     torch.cuda.synchronize()
-    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-    clock_log = os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")
+    clock_log = None
+    if args.clock_log:
+        clock_log = args.clock_log.replace("{rank}", str(rank))
+        os.makedirs(os.path.dirname(os.path.abspath(clock_log)), exist_ok=True)
     with ClockSampler(local, clock_log) as clk:
         t0 = time.perf_counter()
         for i in range(args.steps):
@@ -696,6 +698,9 @@ def main(argv=None):
                     help="skip the long-context keep-fraction sweep (decode time against kept blocks)")
     ap.add_argument("--no-estimators", action="store_true",
                     help="skip the top-k entropy estimator line")
+    ap.add_argument("--clock-log", default=None,
+                    help="also write the raw nvidia-smi clock samples of the timed region to this "
+                         "CSV file ({rank} is replaced by the rank)")
     ap.add_argument("--traffic", type=float, default=None,
                     help="ncu dram bytes per launch of the dominant kernel, if measured")
     args = ap.parse_args(argv)
