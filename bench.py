@@ -574,8 +574,8 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=gs):
             body(args.warmup, gs)
-        graph.replay()
-        gs.synchronize()
+        graph.replay()                 # on the current stream, like every replay below
+        torch.cuda.synchronize()
     except Exception as ex:                                    # capture refused: eager steps
         graph = None
         mode = f"eager (graph capture refused: {type(ex).__name__})"
@@ -584,8 +584,10 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
     for i in range(args.steps):
         t0 = time.perf_counter()
         if graph is not None:
+            # replay() launches on the current stream (not the capture stream):
+            # wait for the whole device, so each step's results are on the host
             graph.replay()
-            gs.synchronize()
+            torch.cuda.synchronize()
         else:
             body(args.warmup + i, main)
             main.synchronize()
