@@ -68,7 +68,7 @@ typedef uint16_t eti_bf16;
 #define ETI_OK               0
 #define ETI_ERR_NULL        (-1)  /* a required pointer is NULL */
 #define ETI_ERR_SHAPE       (-2)  /* a size is out of range or inconsistent */
-#define ETI_ERR_UNSUPPORTED (-3)  /* a valid shape this build does not implement */
+#define ETI_ERR_UNSUPPORTED (-3)  /* a valid shape this library does not implement */
 #define ETI_ERR_WORKSPACE   (-4)  /* ws is NULL or smaller than *_workspace_size() */
 #define ETI_ERR_CUDA        (-5)  /* a kernel launch failed (cudaGetLastError) */
 #define ETI_ERR_ALIGN       (-6)  /* a bf16 tensor is not 16-byte aligned */

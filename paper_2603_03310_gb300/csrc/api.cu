@@ -151,7 +151,7 @@ const char* eti_status_string(int s) {
         case ETI_OK: return "ok";
         case ETI_ERR_NULL: return "a required pointer is NULL";
         case ETI_ERR_SHAPE: return "a size is out of range or inconsistent";
-        case ETI_ERR_UNSUPPORTED: return "shape not supported by this build";
+        case ETI_ERR_UNSUPPORTED: return "shape not supported by this library";
         case ETI_ERR_WORKSPACE: return "workspace missing or too small";
         case ETI_ERR_CUDA: return "CUDA launch failed";
         case ETI_ERR_ALIGN: return "a bf16 tensor is not 16-byte aligned";
