@@ -135,3 +135,105 @@ def test_binding_refuses_cpu_tensors(lib):
         eti.eti_entropy_temp_sample(x, x[:, 0], x[:, 0], x[:, 0], x[:, 0],
                                     torch.zeros(2, dtype=torch.int32), x[:, 0], x[:, 0],
                                     torch.zeros(2, dtype=torch.int32), torch.zeros(64, dtype=torch.uint8))
+
+
+def test_status_strings_cover_every_code(lib):
+    for s in (-7,):
+        assert "scratch" in lib.eti_status_string(s).decode()
+    assert lib.eti_status_string(-99).decode() == "unknown status"
+
+
+def test_topk_call_validation(lib):
+    P = ctypes.c_void_p
+    fake = P(256)
+    f = lib.eti_topk_entropy
+
+    def call(logits=fake, B=4, V=10, ld=10, T=fake, k=3, Ht=fake, Hh=fake, tail=fake, err=fake):
+        return f(logits, B, V, ld, T, k, Ht, Hh, tail, err, NULL)
+    assert call(B=-1) == -2
+    assert call(B=65536) == -2
+    assert call(V=0) == -2
+    assert call(ld=9) == -2                  # rows overlap
+    assert call(k=0) == -2
+    assert call(B=0, logits=NULL, T=NULL, Ht=NULL, Hh=NULL, err=NULL) == 0
+    for name in ("logits", "T", "Ht", "Hh", "err"):
+        assert call(**{name: NULL}) == -1, name
+
+
+def test_schedule_call_validation(lib):
+    P = ctypes.c_void_p
+    fake = P(256)
+    prm = eti.sched_params()
+    f = lib.eti_schedule
+
+    def call(dH=fake, ema=fake, kept=NULL, Hkv=8, Pg=16, L=NULL, urg=NULL, p=ctypes.byref(prm),
+             B=4, budget=2, pri=fake, adm=fake):
+        return f(dH, ema, kept, Hkv, Pg, L, urg, p, B, budget, pri, adm, NULL)
+    assert call(B=-1) == -2
+    assert call(B=65536) == -2
+    assert call(kept=fake, Hkv=0) == -2      # kept counts need the kv-head count
+    assert call(kept=fake, Pg=0) == -2       # ... and the page size
+    assert call(B=0, dH=NULL, ema=NULL, p=NULL, pri=NULL, adm=NULL) == 0
+    for name in ("dH", "ema", "p", "pri", "adm"):
+        assert call(**{name: NULL}) == -1, name
+
+
+def test_score_and_prune_call_validation(lib):
+    P = ctypes.c_void_p
+    a16, bad = P(4096), P(4100)
+
+    def score(q=a16, k=a16, bt=a16, L=a16, B=4, Hq=32, Hkv=8, D=128, Pg=16, mb=512, pages=1000,
+              stats=a16):
+        return lib.eti_score_blocks(q, k, bt, L, B, Hq, Hkv, D, Pg, mb, pages, 0.1, NULL, NULL,
+                                    stats, NULL)
+    assert score(B=-1) == -2
+    assert score(pages=-1) == -2
+    assert score(Hq=12, Hkv=8) == -2
+    assert score(D=256) == -3
+    assert score(B=0, q=NULL, k=NULL, bt=NULL, L=NULL, stats=NULL) == 0
+    for name in ("q", "k", "bt", "L", "stats"):
+        assert score(**{name: NULL}) == -1, name
+    for name in ("q", "k", "stats"):
+        assert score(**{name: bad}) == -6, name
+
+    def prune(stats=a16, bt=a16, L=a16, B=4, Hq=32, Hkv=8, D=128, Pg=16, mb=512, pages=1000,
+              theta=a16, mode=0, mask=a16, kidx=a16, kcnt=a16, err=a16):
+        return lib.eti_prune_blocks(stats, bt, L, B, Hq, Hkv, D, Pg, mb, pages, theta, 1, mode,
+                                    mask, kidx, kcnt, NULL, NULL, err, NULL)
+    assert prune(mb=0) == -2
+    assert prune(mb=40000) == -3
+    assert prune(Pg=64) == -3
+    assert prune(mode=3) == -3
+    assert prune(B=0, stats=NULL, bt=NULL, L=NULL, theta=NULL, mask=NULL, kidx=NULL, kcnt=NULL,
+                 err=NULL) == 0
+    for name in ("stats", "bt", "L", "theta", "mask", "kidx", "kcnt", "err"):
+        assert prune(**{name: NULL}) == -1, name
+    assert prune(stats=bad) == -6
+
+
+def test_noalloc_call_validation(lib):
+    # every refusal below comes before the library looks up its scratch
+    # array on a device, so it runs without a GPU
+    P = ctypes.c_void_p
+    fake = P(256)
+    prm = eti.ctrl_params()
+    f = lib.eti_entropy_temp_sample_noalloc
+    OUTS = [fake] * 6 + [NULL, fake]
+    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -2
+    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -2
+    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, *[NULL] * 8, NULL) == 0
+    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -1
+    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, *OUTS, NULL) == -1
+    # the largest batch whose scratch fits is accepted by the size check; one
+    # more row than the array holds is refused with ETI_ERR_TOO_LARGE
+    cap = lib.eti_entropy_temp_sample_noalloc_max_bytes()
+    lo, hi = 1, 65535
+    if lib.eti_entropy_temp_sample_workspace_size(hi, 4) <= cap:
+        pytest.skip("every batch fits the fixed scratch on this device")
+    while hi - lo > 1:
+        mid = (lo + hi) // 2
+        if lib.eti_entropy_temp_sample_workspace_size(mid, 4) <= cap:
+            lo = mid
+        else:
+            hi = mid
+    assert f(fake, hi, 4, 4, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -7
