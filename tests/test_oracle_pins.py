@@ -397,6 +397,29 @@ def test_block_scores_sum_to_attention_entropy():
             assert abs(r["head_A"][b, h].sum() - 1.0) < 1e-12
 
 
+def test_mode_A_group_score_from_torch_attention():
+    """Reading R4 + R5 + R6: the normalised score of block b for kv head k is
+    max over the g query heads of the group of n_b * I_b^(h) / sum_b' I_b'^(h),
+    with I_b^(h) = sum_{i in b} -a_i log a_i (torch softmax, fp64); checked on
+    g = 4 with ragged last blocks, so a mean over heads, a dropped n_b or a
+    normalisation by the block count fails it."""
+    w, kv, n = _small_kv(B=3, Hq=8, Hkv=2, lens=(37, 64, 5), seed=31)
+    r = oracle.score_prune(n["q"], n["k"], n["bt"], n["L"], n["scale"], np.zeros(w.B), 1)
+    g = w.Hq // w.Hkv
+    for b in range(w.B):
+        nb = -(-int(n["L"][b]) // w.P)
+        per_head = np.empty((w.Hq, nb))
+        for h in range(w.Hq):
+            a = _torch_attention(n, b, h, g)
+            t = special.entr(a)
+            I = np.array([t[j * w.P:(j + 1) * w.P].sum() for j in range(nb)])
+            per_head[h] = nb * I / I.sum() if I.sum() > 0 else 1.0
+        grouped = per_head.reshape(w.Hkv, g, nb)
+        assert np.allclose(r["block_score"][b, :, :nb], grouped.max(axis=1), rtol=1e-10, atol=1e-12)
+        # the heads of a group disagree, so a mean or a single head would fail
+        assert nb == 1 or not np.allclose(grouped.max(axis=1), grouped.mean(axis=1))
+
+
 def test_uniform_attention_closed_form():
     """q = 0: a_i = 1/L, so I_b = (t_b/L) log L and Ibar_b = n_b t_b / L."""
     w, kv, n = _small_kv(lens=(37, 64, 5, 16), B=4)
