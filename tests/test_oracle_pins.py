@@ -246,6 +246,24 @@ def test_threshold_floor():
         assert abs(_ets(z, **kw)["theta_next"][0] - want) < 1e-12
 
 
+def test_threshold_limits_and_monotonicity():
+    """Section 3.2 / Section 5: a flat distribution (H = log V) prunes nothing
+    (theta = 0 keeps every block), a certain one (H = 0) gets the full
+    theta_hi, and the threshold never rises as the entropy rises (heating the
+    same logits raises H, Section 2.1)."""
+    V = 512
+    assert _ets(np.zeros(V))["theta_next"][0] == pytest.approx(0.0, abs=1e-12)
+    z = np.full(V, -np.inf, np.float32)
+    z[3] = 1.0
+    assert _ets(z, theta_hi=1.5)["theta_next"][0] == 1.5
+    rng = np.random.default_rng(19)
+    z = (rng.standard_normal(V) * 3).astype(np.float32)
+    th = [_ets(z, T=T)["theta_next"][0] for T in np.geomspace(0.05, 50, 30)]
+    Hs = [_ets(z, T=T)["H"][0] for T in np.geomspace(0.05, 50, 30)]
+    assert all(b > a for a, b in zip(Hs, Hs[1:]))
+    assert all(b <= a for a, b in zip(th, th[1:])) and th[0] > 0.5 > th[-1]
+
+
 # ----------------------------------------------------------------------------
 # Sampler: Philox4x32-10 and the Gumbel-max draw
 
