@@ -11,10 +11,13 @@ vocabulary 128,256) with seeded synthetic inputs.
 
 Prints ONE JSON line (rank 0).  Timing: W warm-up steps, then K timed steps;
 before every step a buffer of twice the L2 size is written and another one
-read (L2 flush, write-backs settled outside the timed region); each
-kernel call is bracketed by CUDA events on the launching stream and the step
-time is the sum of its calls.  `value` = sequences decoded per second per
-layer step over all ranks (each rank decodes its own batch: weak scaling).
+read (L2 flush, write-backs settled outside the timed region); each timed
+step is bracketed by one pair of CUDA events on the launching stream (no
+event between its calls, so each kernel keeps its programmatic launch overlap
+with the one before), and a separate pass with an event between calls gives
+the per-kernel times behind `roofline`.  `value` = sequences decoded per
+second per layer step over all ranks (each rank decodes its own batch: weak
+scaling).
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload (the paper has no reference implementation).

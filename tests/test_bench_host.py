@@ -1,0 +1,114 @@
+"""Host logic of bench.py that decides what the JSON line reports (CPU only).
+
+The clock summary decides whether a run is kept (a thermal or hardware
+slowdown rejects it), the source digest decides whether the committed ncu
+traffic still describes the kernel that ran, and the byte accounting is the
+numerator of every roofline fraction.  None of this needs a GPU.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import bench
+import workloads
+
+
+def _line(sm, mx=2070, reasons=("Not Active",) * 4, power=900.0):
+    hw, hwt, swt, cap = reasons
+    return f"0, {sm}, {mx}, {power}, 0x0000000000000000, {hw}, {hwt}, {swt}, {cap}"
+
+
+def test_clock_summary_median_max_and_reasons():
+    c = bench.ClockSampler(0)
+    c.lines = [_line(2070), _line(1995), _line(2070),
+               _line(1900, reasons=("Not Active", "Not Active", "Not Active", "Active")),
+               "garbage", "0, [N/A], 2070, 1.0, 0x0, Not Active, Not Active, Not Active, Not Active"]
+    s = c.summary()
+    assert s["sm_mhz"] == 2032.5 and s["sm_max_mhz"] == 2070.0 and s["samples"] == 4
+    assert s["reasons"] == ["sw_power_cap"]
+    c.lines = [_line(1200, reasons=("Active", "Not Active", "Active", "Not Active"))]
+    assert c.summary()["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"]
+    c.lines = []
+    assert c.summary() is None
+
+
+def test_clock_sampler_without_nvidia_smi(monkeypatch, tmp_path):
+    # no nvidia-smi on the host: the sampler is a no-op and reports nothing
+    monkeypatch.setenv("PATH", str(tmp_path))
+    log = tmp_path / "clocks.csv"
+    with bench.ClockSampler(0, str(log)) as c:
+        pass
+    assert c.summary() is None and not log.exists()
+
+
+def test_source_digest_ignores_comments_not_code(tmp_path):
+    a = tmp_path / "a.cu"
+    a.write_text("int f(int x) {\n    return x + 1;  // add one\n}\n")
+    d0 = bench.source_digest([str(a)])
+    a.write_text("/* header */\n\nint f(int x) {\n    return x + 1;  // plus one\n}\n")
+    assert bench.source_digest([str(a)]) == d0
+    a.write_text("int f(int x) {\n    return x + 2;\n}\n")
+    assert bench.source_digest([str(a)]) != d0
+
+
+def test_ncu_traffic_record_matches_the_committed_kernels():
+    rec = json.load(open(os.path.join(bench.ROOT, "profiles", "ncu_traffic.json")))
+    kernels = [k for k in rec if not k.startswith("_")]
+    assert {"score_blocks", "paged_decode", "entropy_sample_partial"} <= set(kernels)
+    for k in kernels:
+        for p in rec[k]["sources"]:
+            assert os.path.exists(os.path.join(bench.ROOT, p)), p
+        got = bench.ncu_traffic(k)
+        # a record is either current (its bytes) or stale (None), never wrong
+        assert got in (rec[k]["bytes"], None)
+    assert bench.ncu_traffic("no_such_kernel") is None
+
+
+def test_algorithmic_bytes_of_the_step():
+    w = workloads.WORKLOADS["llama3_8b"]
+    L = workloads.ctx_lengths(w)
+    nb = -(-L // w.P)
+    g = w.Hq // w.Hkv
+    kept = int(nb.sum()) * w.Hkv // 2
+    b = bench.algorithmic_bytes(w, L, kept)
+    # every key of every sequence once (bf16), per kv head
+    keys = sum(int(l) * w.Hkv * w.D * 2 for l in L)
+    assert b["score"] > keys and b["score"] - keys < 0.25 * keys      # + q, scores, stats
+    # the decode reads only the kept V pages (and their scores): half kept,
+    # about half of all V
+    allv = sum(int(n) * w.P * w.Hkv * (w.D * 2 + g * 4) for n in nb)
+    assert abs(b["decode"] - allv / 2) < w.B * w.Hq * w.D * 2 + 1
+    assert b["sample"] == w.B * w.V * 4
+    assert 0 < b["prune"] < b["score"] / 10
+    # the keep-all decode bytes scale linearly with the kept blocks
+    b2 = bench.algorithmic_bytes(w, L, 2 * kept)
+    assert b2["decode"] - b["decode"] == b["decode"] - bench.algorithmic_bytes(w, L, 0)["decode"]
+
+
+def test_aggregate_counts_every_rank_over_the_slowest():
+    v, slow = bench.aggregate([0.010, 0.012, 0.011, 0.009], 64)
+    assert slow == 0.012 and v == pytest.approx(4 * 64 / 0.012)
+    assert bench.max_over_ranks(3.5, 1, None) == 3.5
+
+
+def test_shards_are_independent_batches_of_the_same_shape():
+    w = workloads.WORKLOADS["llama3_8b"]
+    shards = [bench.shard_workload(w, r) for r in range(4)]
+    assert shards[0] == w
+    assert len({s.seed for s in shards}) == 4
+    assert all((s.B, s.Hq, s.Hkv, s.D, s.P, s.V, s.ctx) == (w.B, w.Hq, w.Hkv, w.D, w.P, w.V, w.ctx)
+               for s in shards)
+    Ls = [workloads.ctx_lengths(s) for s in shards]
+    assert not np.array_equal(Ls[0], Ls[1])
+
+
+def test_warmup_is_at_least_three(monkeypatch):
+    seen = {}
+    monkeypatch.setattr(bench, "run_gpu", lambda a: seen.update(gpu=a))
+    monkeypatch.setattr(bench, "run_reference", lambda a: seen.update(ref=a))
+    bench.main(["--steps", "5", "--warmup", "1"])
+    assert seen["gpu"].warmup == 3 and seen["gpu"].steps == 5
+    bench.main(["--impl", "reference", "--steps", "2", "--warmup", "0"])
+    assert seen["ref"].impl == "reference" and seen["ref"].warmup == 0
