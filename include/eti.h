@@ -35,6 +35,9 @@
  *  - Supported shapes: head_dim D in {64, 128}; page size P in {16, 32};
  *    Hq % Hkv == 0 with group size g = Hq / Hkv <= 8; 1 <= max_blocks <= 32768;
  *    B <= 65535 (entropy/sample) or 8192 (attention calls); 1 <= V.
+ *    Attention calls also need B * Hkv * max_blocks <= 2^30 and
+ *    num_pages * Hkv * P < 2^31 (block counts and cache rows are 32-bit
+ *    indices on the device); larger shapes return ETI_ERR_UNSUPPORTED.
  *    q, k_cache, v_cache, token_scores and the decode output must be 16-byte
  *    aligned.
  *

@@ -72,6 +72,7 @@ namespace {
 
 constexpr int kMaxB = 8192;
 constexpr int kMaxBlocks = 32768;
+constexpr long long kMaxUnits = 1LL << 30;   // B * Hkv * max_blocks
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15) == 0; }
 size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -83,6 +84,11 @@ int check_attn_shape(int B, int Hq, int Hkv, int D, int P, int max_blocks, long 
     if (Hq / Hkv > 8 || max_blocks > kMaxBlocks) return ETI_ERR_UNSUPPORTED;
     if (!((D == 64 || D == 128) && (P == 16 || P == 32))) return ETI_ERR_UNSUPPORTED;
     if ((long long)max_blocks * P > 0x7fffffffLL) return ETI_ERR_SHAPE;
+    // the kernels count (sequence, kv head, block) units and their prefix
+    // sums in 32-bit ints, and a TMA row coordinate (page * Hkv + head) * P
+    // is a signed 32-bit value
+    if ((long long)B * Hkv * max_blocks > kMaxUnits) return ETI_ERR_UNSUPPORTED;
+    if (num_pages > 0x7fffffffLL / ((long long)Hkv * P)) return ETI_ERR_UNSUPPORTED;
     return ETI_OK;
 }
 

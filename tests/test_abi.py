@@ -117,6 +117,15 @@ def test_attention_call_validation(lib):
     assert call(ws=NULL) == -4
     assert call(wsb=need - 1) == -4
     assert call(B=0, ws=NULL) == 0
+    # 32-bit device indices: unit counts B*Hkv*max_blocks and cache rows
+    # num_pages*Hkv*P are bounded even where each size alone is allowed
+    assert call(B=8192, Hq=32, Hkv=8, mb=32768) == -3
+    assert call(B=8192, Hq=32, Hkv=8, mb=16384, q=NULL) == -1   # 2^30 units: accepted
+    assert f(a16, a16, a16, a16, 4, 32, 8, 128, 16, 512, (1 << 31) // (8 * 16) + 1, 0.1, a16, 1, 0,
+             NULL, a16, a16, a16, NULL, NULL, NULL, a16, a16, need, NULL) == -3
+    assert f(a16, a16, a16, a16, 4, 32, 8, 128, 16, 512, (1 << 31) // (8 * 16) - 1, 0.1, a16, 1, 0,
+             NULL, a16, a16, a16, NULL, NULL, NULL, a16, NULL, need, NULL) == -4
+    assert lib.eti_score_prune_workspace_size(8192, 32, 8, 128, 16, 32768) == 0
     # decode: workspace sizes grow when the scores must be recomputed
     with_s = lib.eti_paged_decode_workspace_size(4, 32, 8, 128, 16, 512, 1)
     without = lib.eti_paged_decode_workspace_size(4, 32, 8, 128, 16, 512, 0)
