@@ -25,6 +25,7 @@ STATUS = {0: "ok", -1: "null pointer", -2: "bad shape", -3: "unsupported shape",
           -4: "workspace too small", -5: "CUDA launch failed", -6: "misaligned tensor",
           -7: "too large for the fixed scratch"}
 ERRF_BAD_PAGE, ERRF_BAD_CTX, ERRF_NONFINITE, ERRF_ALL_NEG_INF, ERRF_BAD_TEMP = 1, 2, 4, 8, 16
+ERRF_TIMEOUT = 32
 
 # C-ABI symbols declared in include/eti.h
 SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_entropy_temp_sample_workspace_size",

@@ -246,3 +246,11 @@ def test_noalloc_call_validation(lib):
         else:
             hi = mid
     assert f(fake, hi, 4, 4, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -7
+
+
+def test_binding_constants_match_the_header():
+    txt = open(os.path.join(ROOT, "include", "eti.h")).read()
+    for name, val in re.findall(r"#define ETI_(ERRF_\w+)\s+(0x[0-9a-fA-F]+)u", txt):
+        assert getattr(eti, name) == int(val, 16), name
+    for name, val in re.findall(r"#define ETI_(OK|ERR_\w+)\s+\(?(-?\d+)\)?", txt):
+        assert int(val) in eti.STATUS, name
