@@ -254,3 +254,47 @@ def test_binding_constants_match_the_header():
         assert getattr(eti, name) == int(val, 16), name
     for name, val in re.findall(r"#define ETI_(OK|ERR_\w+)\s+\(?(-?\d+)\)?", txt):
         assert int(val) in eti.STATUS, name
+
+
+C_CLIENT = r"""
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+#include "eti.h"
+
+int main(void) {
+    eti_ctrl_params p;
+    eti_sched_params s;
+    eti_ctrl_defaults(&p);
+    eti_sched_defaults(&s);
+    if (p.sign != -1.0f || !isinf(p.theta_user) || s.lambda != 0.9f) return 2;
+    if (strstr(eti_version(), "libeti") == NULL) return 3;
+    if (eti_status_string(ETI_ERR_TOO_LARGE)[0] == 0) return 4;
+    if (eti_score_prune_workspace_size(4, 32, 8, 128, 16, 512) == 0) return 5;
+    if (eti_score_prune_workspace_size(4, 30, 8, 128, 16, 512) != 0) return 6;
+    /* an argument error is reported before anything is enqueued */
+    if (eti_entropy_temp_sample(NULL, 4, 10, 10, NULL, NULL, NULL, NULL, &p, 0, 0, NULL, NULL,
+                                NULL, NULL, NULL, NULL, NULL, NULL, NULL, 0, NULL) != ETI_ERR_NULL)
+        return 7;
+    printf("ok %s\n", eti_version());
+    return 0;
+}
+"""
+
+
+def test_header_is_plain_c_and_links(lib, tmp_path):
+    import shutil, subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    src = tmp_path / "client.c"
+    src.write_text(C_CLIENT)
+    exe = tmp_path / "client"
+    libdir = os.path.dirname(eti.LIB_PATH)
+    p = subprocess.run([cc, "-std=c99", "-Wall", "-Werror", "-pedantic", str(src),
+                        "-I", os.path.join(ROOT, "include"), "-L", libdir, "-l:libeti.so",
+                        "-Wl,-rpath," + libdir, "-lm", "-o", str(exe)],
+                       capture_output=True, text=True)
+    assert p.returncode == 0, p.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
+    assert r.returncode == 0 and r.stdout.startswith("ok libeti"), (r.returncode, r.stdout, r.stderr)
