@@ -112,3 +112,27 @@ def test_warmup_is_at_least_three(monkeypatch):
     assert seen["gpu"].warmup == 3 and seen["gpu"].steps == 5
     bench.main(["--impl", "reference", "--steps", "2", "--warmup", "0"])
     assert seen["ref"].impl == "reference" and seen["ref"].warmup == 0
+
+
+def test_reference_arm_runs_on_rank_zero_only(monkeypatch, capsys):
+    # under torchrun the other ranks exit without work and print nothing
+    monkeypatch.setenv("RANK", "1")
+    monkeypatch.setenv("WORLD_SIZE", "2")
+    import argparse
+    args = argparse.Namespace(workload="tiny", steps=3, warmup=3, cpu_budget=1.0)
+    assert bench.run_reference(args) is None
+    assert capsys.readouterr().out == ""
+
+
+def test_reference_arm_line_on_the_tiny_step(monkeypatch, capsys, oracle_lib):
+    monkeypatch.setenv("RANK", "0")
+    monkeypatch.setenv("WORLD_SIZE", "1")
+    bench.main(["--impl", "reference", "--workload", "tiny", "--steps", "3", "--warmup", "3",
+                "--cpu-budget", "2"])
+    line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["metric"] == bench.METRIC
+    assert line["value"] > 0 and line["unit"] == bench.UNIT and line["higher_is_better"] is True
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["cores"] >= 1
+    assert line["e2e"] == {"value": line["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
