@@ -152,6 +152,9 @@ void eti_ctrl_defaults(eti_ctrl_params* p);
  * [B].  T_out may alias T_in.
  * Row errors (NaN/+inf logit, all -inf, bad T_in) give tok = -1, H = dH =
  * surprisal = NaN, T_out = T_in, theta_next = 0 (prune nothing), tau unchanged.
+ * The row is computed in fp32 on z * log2(e) / (T_cal T_in): a row where that
+ * product overflows (|z| / (T_cal T_in) above about 2.36e38, or T_cal T_in
+ * below about 4.2e-39) is reported as ETI_ERRF_NONFINITE as well.
  * Workspace: eti_entropy_temp_sample_workspace_size(B, V) bytes (partial
  * reductions of the row pieces; no initial contents required).
  */
