@@ -599,7 +599,15 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
     bi = h_in.numel() + h_logits.numel() * 4
     bo = h_out.numel() * 2 + h_res.numel()
     return {"value": round(w.B / s, 1), "unit": UNIT, "ms_per_step": round(s * 1e3, 4),
-            "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo), "mode": mode}
+            "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo), "mode": mode,
+            "l2": "not flushed: every step uploads its logits and reads "
+                  f"{(key_bytes(w, kv) / 1e9):.2f} GB of keys plus the kept values, more than the L2"}
+
+
+def key_bytes(w, kv) -> int:
+    """Bytes of the key pages a step reads (every block of every sequence)."""
+    L = kv["ctx_lens"].cpu().numpy()
+    return int((-(-L // w.P)).sum()) * w.Hkv * w.P * w.D * 2
 
 
 # ---------------------------------------------------------------------------

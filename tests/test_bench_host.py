@@ -136,3 +136,14 @@ def test_reference_arm_line_on_the_tiny_step(monkeypatch, capsys, oracle_lib):
     assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["cores"] >= 1
     assert line["e2e"] == {"value": line["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
                            "d2h_bytes_per_step": 0}
+
+
+def test_e2e_working_set_exceeds_l2():
+    # the end-to-end leg runs without an L2 flush: the keys alone that a step
+    # of the benchmark workload reads are several times the 129 MB L2
+    import torch
+    w = workloads.WORKLOADS["llama3_8b"]
+    L = workloads.ctx_lengths(w)
+    kb = bench.key_bytes(w, {"ctx_lens": torch.from_numpy(L)})
+    assert kb >= int(L.sum()) * w.Hkv * w.D * 2
+    assert kb > 4 * 129 * 2 ** 20
