@@ -120,3 +120,75 @@ def test_step_writes_stay_inside_their_buffers(case):
         assert torch.equal(a, b), n
     if case != "gqa4_d128_p16":
         assert got["err_attn"].cpu().tolist()[2] != 0 and got["err_ets"].cpu().tolist()[3] != 0
+
+
+def _estimator_and_scheduler(eti, lg, B, dev, guarded):
+    """eti_topk_entropy and eti_schedule on guarded (or plain) output buffers."""
+    f32, i32, u8 = torch.float32, torch.int32, torch.uint8
+    spec = {"H_tilde": f32, "H_hat": f32, "tail_mass": f32, "err": i32, "priority": f32,
+            "admit": u8, "ema": f32}
+    gs, t = {}, {}
+    for n, dt in spec.items():
+        if guarded:
+            gs[n] = Guarded((B,), dt, dev)
+            t[n] = gs[n].t
+        else:
+            t[n] = torch.empty(B, dtype=dt, device=dev)
+    t["ema"].copy_(torch.linspace(0.0, 0.5, B, device=dev))
+    _topk(eti, lg, t)
+    _sched(eti, lg, t, B, dev)
+    torch.cuda.synchronize()
+    return {n: v.clone() for n, v in t.items()}, gs
+
+
+def _topk(eti, lg, t):
+    eti.eti_topk_entropy(lg["logits"], lg["T_in"], 64, t["H_tilde"], t["H_hat"], t["err"],
+                         tail_mass=t["tail_mass"])
+
+
+def _sched(eti, lg, t, B, dev):
+    dH = (lg["H_prev"] - 1.0).contiguous()
+    kept = (torch.arange(B * 4, device=dev) % 50).to(torch.int32).view(B, 4)
+    ctx = (torch.arange(B, device=dev) * 37 % 4000).to(torch.int32)
+    urg = torch.ones(B, dtype=torch.float32, device=dev)
+    eti.eti_schedule(dH, t["ema"], B // 2, t["priority"], t["admit"], kept_cnt=kept, P=16,
+                     ctx_lens=ctx, urgency=urg)
+
+
+def test_estimator_and_scheduler_calls_reach_the_device_check():
+    # the calls the GPU test below makes are well formed: with host tensors
+    # they get as far as the binding's device check
+    import paper_2603_03310_gb300 as eti
+    w = workloads.WORKLOADS["llama3_8b"].scaled(B=5, V=300)
+    lg = workloads.make_logits(w, "cpu")
+    t = {n: Guarded((w.B,), dt, "cpu").t for n, dt in
+         (("H_tilde", torch.float32), ("H_hat", torch.float32), ("tail_mass", torch.float32),
+          ("err", torch.int32), ("priority", torch.float32), ("admit", torch.uint8),
+          ("ema", torch.float32))}
+    with pytest.raises(eti.EtiError, match="CUDA tensor"):
+        _topk(eti, lg, t)
+    with pytest.raises(eti.EtiError, match="CUDA tensor"):
+        _sched(eti, lg, t, w.B, "cpu")
+
+
+@pytest.mark.gpu
+def test_estimator_and_scheduler_writes_stay_inside_their_buffers():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2603_03310_gb300 as eti
+    eti.build()
+    eti.load()
+    w = workloads.WORKLOADS["llama3_8b"].scaled(B=37, V=5003)
+    lg = workloads.make_logits(w, "cuda:0")
+    lg["logits"][4, 7] = float("nan")                      # an error row
+    plain, _ = _estimator_and_scheduler(eti, lg, w.B, "cuda:0", guarded=False)
+    got, gs = _estimator_and_scheduler(eti, lg, w.B, "cuda:0", guarded=True)
+    bad = [n for n, g in gs.items() if not g.intact()]
+    assert not bad, f"writes outside the buffer extent: {bad}"
+    for n, a in plain.items():
+        a, b = a.cpu(), got[n].cpu()
+        if a.dtype == torch.float32:
+            assert torch.equal(torch.isnan(a), torch.isnan(b)), n
+            a, b = torch.nan_to_num(a), torch.nan_to_num(b)
+        assert torch.equal(a, b), n
+    assert got["err"].cpu().tolist()[4] != 0
