@@ -65,6 +65,17 @@ def aggregate(per_rank_step_s: list[float], B: int) -> tuple[float, float]:
     return B * len(per_rank_step_s) / slowest, slowest
 
 
+def aggregate_e2e(e2e: dict, B: int, world: int, device) -> dict:
+    """The end-to-end figure for the whole job: every rank's sequences over the
+    slowest rank's step, and every rank's copies (unchanged at one rank)."""
+    if world == 1:
+        return e2e
+    s = max_over_ranks(e2e["ms_per_step"] / 1e3, world, device)
+    return dict(e2e, value=round(B * world / s, 1), ms_per_step=round(s * 1e3, 4),
+                h2d_bytes_per_step=e2e["h2d_bytes_per_step"] * world,
+                d2h_bytes_per_step=e2e["d2h_bytes_per_step"] * world)
+
+
 def max_over_ranks(x: float, world: int, device) -> float:
     if world == 1:
         return x
@@ -465,6 +476,8 @@ def run_gpu(args):
     # end to end through the public API: host (pinned) inputs -> device -> step -> host results
     e2e = None if args.no_e2e else run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm,
                                            args, device)
+    if e2e is not None:
+        e2e = aggregate_e2e(e2e, w.B, world, device)
 
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,

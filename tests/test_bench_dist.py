@@ -1,6 +1,7 @@
 """Multi-rank logic of bench.py on CPU with gloo, world size 2: every rank
 decodes its own batch (independent sequences, no data-path collective), the
-step time is the max over ranks and the throughput counts every rank's batch."""
+step time is the max over ranks and the throughput counts every rank's batch;
+the end-to-end figure is aggregated the same way."""
 import os
 import socket
 
@@ -28,8 +29,11 @@ def _worker(rank, world, port, q):
     slowest = bench.max_over_ranks(step_s, w, torch.device("cpu"))
     value, _ = bench.aggregate([slowest] * w, wl.B)
     L = workloads.ctx_lengths(wl)
+    e2e = bench.aggregate_e2e({"value": 0.0, "unit": "tokens/s", "ms_per_step": 0.3 + 0.1 * r,
+                               "h2d_bytes_per_step": 100, "d2h_bytes_per_step": 7},
+                              wl.B, w, torch.device("cpu"))
     dist.barrier()
-    q.put((r, wl.seed, slowest, value, L.tolist()))
+    q.put((r, wl.seed, slowest, value, L.tolist(), e2e))
     dist.destroy_process_group()
 
 
@@ -44,7 +48,11 @@ def test_two_rank_weak_scaling_logic():
     for p in ps:
         p.join(timeout=60)
         assert p.exitcode == 0
-    (r0, s0, t0, v0, L0), (r1, s1, t1, v1, L1) = res
+    (r0, s0, t0, v0, L0, e0), (r1, s1, t1, v1, L1, e1) = res
     assert s0 != s1 and L0 != L1                  # independent batches
     assert t0 == t1 == pytest.approx(0.020)       # max over ranks
     assert v0 == v1 == pytest.approx(2 * 64 / 0.020)
+    # end to end: both ranks' sequences over the slower rank's 0.4 ms step
+    assert e0 == e1
+    assert e0["ms_per_step"] == pytest.approx(0.4) and e0["value"] == pytest.approx(2 * 64 / 0.4e-3, rel=1e-6)
+    assert (e0["h2d_bytes_per_step"], e0["d2h_bytes_per_step"]) == (200, 14)

@@ -147,3 +147,9 @@ def test_e2e_working_set_exceeds_l2():
     kb = bench.key_bytes(w, {"ctx_lens": torch.from_numpy(L)})
     assert kb >= int(L.sum()) * w.Hkv * w.D * 2
     assert kb > 4 * 129 * 2 ** 20
+
+
+def test_e2e_at_one_rank_is_reported_as_measured():
+    e = {"value": 123.0, "unit": "tokens/s", "ms_per_step": 0.5, "h2d_bytes_per_step": 9,
+         "d2h_bytes_per_step": 3, "mode": "x"}
+    assert bench.aggregate_e2e(e, 64, 1, None) is e
