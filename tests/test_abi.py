@@ -298,3 +298,20 @@ def test_header_is_plain_c_and_links(lib, tmp_path):
     assert p.returncode == 0, p.stderr
     r = subprocess.run([str(exe)], capture_output=True, text=True, timeout=60)
     assert r.returncode == 0 and r.stdout.startswith("ok libeti"), (r.returncode, r.stdout, r.stderr)
+
+
+def test_readme_c_example_compiles(tmp_path):
+    # the decode-step example in the README is compiled against include/eti.h
+    import shutil, subprocess
+    cc = shutil.which("gcc") or shutil.which("cc")
+    if cc is None:
+        pytest.skip("no C compiler")
+    txt = open(os.path.join(ROOT, "README.md")).read()
+    blocks = re.findall(r"```c\n(.*?)```", txt, flags=re.S)
+    assert len(blocks) == 1 and "decode_step" in blocks[0]
+    src = tmp_path / "example.c"
+    src.write_text(blocks[0])
+    p = subprocess.run([cc, "-std=c99", "-Wall", "-Wextra", "-Werror", "-pedantic", "-c", str(src),
+                        "-I", os.path.join(ROOT, "include"), "-o", str(tmp_path / "example.o")],
+                       capture_output=True, text=True)
+    assert p.returncode == 0, p.stderr
