@@ -168,6 +168,31 @@ def algorithmic_bytes(w, L: np.ndarray, kept_blocks: int) -> dict:
     }
 
 
+def kept_attention_mass(stats: torch.Tensor, keep_mask: torch.Tensor, ctx_lens: torch.Tensor,
+                        P: int) -> dict:
+    """Share of each query head's attention (softmax over all of its sequence's
+    tokens) that falls in the kept blocks, from the scorer's block stats
+    [B][Hkv][max_blocks][g][(m, l - 1, u, e)] and the keep mask: with
+    l_b = 1 + (l - 1), Z = sum_b l_b e^{m_b - M} over the sequence's blocks and
+    the kept share = the same sum over the kept blocks / Z.  Sequences without
+    tokens are left out.  A diagnostic of reading A, whose block score can be
+    small for a block holding one dominant token."""
+    B, Hkv, mb, g, _ = stats.shape
+    nb = (ctx_lens.to(torch.int64) + P - 1) // P
+    valid = (torch.arange(mb, device=stats.device)[None, :] < nb[:, None])[:, None, :, None]
+    m = stats[..., 0].double()
+    ok = valid & torch.isfinite(m)
+    M = torch.where(ok, m, torch.full_like(m, -math.inf)).amax(dim=2, keepdim=True)
+    w = torch.where(ok, (1.0 + stats[..., 1].double()) * torch.exp(m - M), torch.zeros_like(m))
+    Z = w.sum(dim=2)
+    kept = keep_mask.to(torch.bool)[..., None] & ok
+    frac = torch.where(kept, w, torch.zeros_like(w)).sum(dim=2) / Z
+    frac = frac[(nb > 0)[:, None, None].expand_as(frac) & torch.isfinite(frac)]
+    if frac.numel() == 0:
+        return {"mean": None, "min": None}
+    return {"mean": round(float(frac.mean()), 5), "min": round(float(frac.min()), 5)}
+
+
 def source_digest(paths) -> str:
     """sha256 of the code of these source files: comments and blank lines are
     left out, so a change of wording is not a change of kernel."""
@@ -438,6 +463,12 @@ def run_gpu(args):
         one_step(evb[i], offset=args.warmup + args.steps + i)
     torch.cuda.synchronize()
     per = {n: [evb[i][j].elapsed_time(evb[i][j + 1]) for i in range(nb)] for j, n in enumerate(names)}
+    # share of the attention the keep set retains (outside the timed region;
+    # a diagnostic never fails the run)
+    try:
+        kept_mass = kept_attention_mass(stats, step.keep_mask, kv["ctx_lens"], w.P)
+    except Exception as ex:
+        kept_mass = {"error": f"{type(ex).__name__}: {ex}"}
     ms_local = statistics.mean(step_ms)
     ms = max_over_ranks(ms_local, world, device)
     value, _ = aggregate([ms / 1e3] * world, w.B)
@@ -505,6 +536,7 @@ def run_gpu(args):
         "e2e": e2e,
         "estimators": est,
         "keep_sweep": sweep,
+        "kept_attention_mass": kept_mass,
         "wall_s_timed_region": round(wall, 4),
         "clocks": clk.summary(),
     }

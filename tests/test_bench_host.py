@@ -153,3 +153,46 @@ def test_e2e_at_one_rank_is_reported_as_measured():
     e = {"value": 123.0, "unit": "tokens/s", "ms_per_step": 0.5, "h2d_bytes_per_step": 9,
          "d2h_bytes_per_step": 3, "mode": "x"}
     assert bench.aggregate_e2e(e, 64, 1, None) is e
+
+
+def test_kept_attention_mass_matches_the_oracle(oracle_lib):
+    # block stats in the scorer's layout, formed in fp64 from the same bf16
+    # inputs; the oracle's per-block attention masses summed over its keep set
+    # give the expected share for every query head
+    import math
+    import torch
+    oracle = oracle_lib
+    w = workloads.Workload("km", B=4, Hq=8, Hkv=2, D=64, P=16, V=16,
+                           ctx=("list", [37, 0, 200, 16]), seed=71, hi_frac=0.2)
+    kv = workloads.make_kv(w, "cpu")
+    g, mb = w.Hq // w.Hkv, w.max_blocks
+    qb, kb = workloads.bf16_bits(kv["q"]), workloads.bf16_bits(kv["k_cache"])
+    bt, L = kv["block_table"].numpy(), kv["ctx_lens"].numpy()
+    ref = oracle.score_prune(qb, kb, bt, L, kv["scale"], np.full(w.B, 0.9), 2, want_heads=True)
+    q = kv["q"].double()
+    stats = torch.full((w.B, w.Hkv, mb, g, 4), float("nan"), dtype=torch.float32)  # unwritten
+    for b in range(w.B):
+        nb = -(-int(L[b]) // w.P)
+        for j in range(nb):
+            n = min(w.P, int(L[b]) - j * w.P)
+            k = kv["k_cache"][int(bt[b, j])].double()[:, :n]            # [Hkv, n, D]
+            for h in range(w.Hq):
+                x = (k[h // g] @ q[b, h]) * kv["scale"]
+                m = x.max()
+                stats[b, h // g, j, h % g, 0] = float(m)
+                stats[b, h // g, j, h % g, 1] = float(torch.exp(x - m).sum() - 1.0)
+    keep = torch.from_numpy(ref["keep_mask"])
+    got = bench.kept_attention_mass(stats, keep, kv["ctx_lens"], w.P)
+    want = []
+    for b in range(w.B):
+        if L[b] == 0:
+            continue
+        for h in range(w.Hq):
+            kept = ref["keep_mask"][b, h // g].astype(bool)
+            want.append(ref["head_A"][b, h][kept].sum())
+    assert got["mean"] == pytest.approx(float(np.mean(want)), abs=2e-5)
+    assert got["min"] == pytest.approx(float(np.min(want)), abs=2e-5)
+    assert 0 < got["min"] <= got["mean"] <= 1
+    # keeping every block keeps all of the attention
+    full = bench.kept_attention_mass(stats, torch.ones_like(keep), kv["ctx_lens"], w.P)
+    assert full["mean"] == pytest.approx(1.0, abs=1e-6) and full["min"] == pytest.approx(1.0, abs=1e-6)
