@@ -271,6 +271,11 @@ def run_schedule(eti, step, kv, w, stream, reps=50):
     return round(statistics.median(e[0].elapsed_time(e[1]) for e in ev), 5)
 
 
+def workload_desc(w) -> str:
+    """The workload as `config.workload` names it (both arms print the same)."""
+    return f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} D={w.D} P={w.P} {ctx_desc(w)} V={w.V}"
+
+
 def ctx_desc(w) -> str:
     """The workload's context-length distribution, as printed in `config`."""
     kind = w.ctx[0]
@@ -515,8 +520,7 @@ def run_gpu(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16/fp32",
         "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
-        "config": {"workload": f"{w.name}: B={w.B} Hq={w.Hq} Hkv={w.Hkv} D={w.D} P={w.P} "
-                               f"{ctx_desc(w)} V={w.V}",
+        "config": {"workload": workload_desc(w),
                    "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write, then 2x L2 read)",
                    "parallelism": f"replicas x{world} (independent batches)", "B_min": B_min,
                    "theta": "theta_next of the step's own entropy (defaults)",
@@ -734,7 +738,8 @@ def run_reference(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(s * 1e3, 3),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
-        "config": {"workload": f"{w.name} (oracle sample)", "global_batch": len(seqs)},
+        "config": {"workload": workload_desc(w), "global_batch": w.B,
+                   "oracle_sample": f"{len(seqs)} of {w.B} sequences per step"},
         "cpu_baseline": {"value": v, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

@@ -132,6 +132,8 @@ def test_reference_arm_line_on_the_tiny_step(monkeypatch, capsys, oracle_lib):
     line = json.loads(capsys.readouterr().out.strip().splitlines()[-1])
     assert line["impl"] == "reference" and line["metric"] == bench.METRIC
     assert line["value"] > 0 and line["unit"] == bench.UNIT and line["higher_is_better"] is True
+    assert line["config"]["workload"] == bench.workload_desc(workloads.WORKLOADS["tiny"])
+    assert line["config"]["workload"].startswith("tiny: B=4 Hq=8 Hkv=8 D=64 P=16")
     cb = line["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["value"] == line["value"] and cb["cores"] >= 1
     assert line["e2e"] == {"value": line["value"], "unit": bench.UNIT, "h2d_bytes_per_step": 0,
