@@ -74,9 +74,12 @@ typedef uint16_t eti_bf16;
 #define ETI_ERR_UNSUPPORTED (-3)  /* a valid shape this library does not implement */
 #define ETI_ERR_WORKSPACE   (-4)  /* ws is NULL or smaller than *_workspace_size() */
 #define ETI_ERR_CUDA        (-5)  /* a kernel launch failed (cudaGetLastError) */
-#define ETI_ERR_ALIGN       (-6)  /* a bf16 tensor is not 16-byte aligned */
+#define ETI_ERR_TIMEOUT     (-6)  /* reserved: no call returns it.  Calls never wait on the
+                                     host; a device-side wait that gives up is reported per
+                                     sequence by ETI_ERRF_TIMEOUT in err_flags */
 #define ETI_ERR_TOO_LARGE   (-7)  /* the problem needs more than the fixed scratch of
                                      eti_entropy_temp_sample_noalloc */
+#define ETI_ERR_ALIGN       (-8)  /* a bf16 tensor is not 16-byte aligned */
 
 /* per-sequence data error bits written to err_flags */
 #define ETI_ERRF_BAD_PAGE     0x1u  /* a block_table entry is outside [0, num_pages) */
@@ -86,6 +89,11 @@ typedef uint16_t eti_bf16;
 #define ETI_ERRF_BAD_TEMP     0x10u /* T_in is not a positive finite number */
 #define ETI_ERRF_TIMEOUT      0x20u /* a device-side wait for a tile copy gave up (the
                                        sequence's results are not valid) */
+#define ETI_ERRF_DRAIN        0x40u /* with TIMEOUT: after the wait gave up, a tile copy
+                                       already issued did not land within the drain
+                                       limit either, so it may still write shared
+                                       memory after its CTA exited: treat the device
+                                       as suspect, not only the sequence */
 
 /*
  * Controller parameters (Section 3.3 temperature law, Section 3.2 safety
@@ -155,8 +163,13 @@ void eti_ctrl_defaults(eti_ctrl_params* p);
  * The row is computed in fp32 on z * log2(e) / (T_cal T_in): a row where that
  * product overflows (|z| / (T_cal T_in) above about 2.36e38, or T_cal T_in
  * below about 4.2e-39) is reported as ETI_ERRF_NONFINITE as well.
- * Workspace: eti_entropy_temp_sample_workspace_size(B, V) bytes (partial
- * reductions of the row pieces; no initial contents required).
+ * offset_dev: NULL, or a device uint64 that replaces `offset`: the call reads
+ * the counter from it and, once every row is drawn, stores counter + 1 back,
+ * so that a captured CUDA graph draws fresh numbers at every replay.  Calls
+ * that share one offset_dev word must not overlap on the GPU.
+ * Workspace: eti_entropy_temp_sample_workspace_size(B, V) bytes, 4-byte
+ * aligned (row tickets and partial reductions of the row pieces; no initial
+ * contents required: the call zeroes its tickets itself).
  */
 size_t eti_entropy_temp_sample_workspace_size(int B, int V);
 
@@ -178,7 +191,7 @@ typedef struct {
 int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
                             const float* T_in, const float* H_prev, float* tau,
                             const float* H_target, const eti_ctrl_params* params,
-                            uint64_t seed, uint64_t offset,
+                            uint64_t seed, uint64_t offset, uint64_t* offset_dev,
                             int32_t* tok, float* H, float* T_out,
                             float* dH, float* theta_next, float* tok_surprisal,
                             const eti_surp_store* surp_store,
@@ -198,23 +211,25 @@ int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
  * on every GPU that loads the library, kept until the process exits).  It
  * never calls cudaMalloc, cudaFree or any allocating routine.
  *  - The first call on a device looks up that array's device address
- *    (cudaGetSymbolAddress) with the device current, once per device; make
- *    that first call before any stream capture.
+ *    (cudaGetSymbolAddress) with the device current, once per device (and
+ *    again if the device's current context changes, e.g. after
+ *    cudaDeviceReset); make that first call before any stream capture.
  *  - Every call on a device shares the one array and it keeps the previous
- *    call's contents; nothing in it needs to start at zero, because every
- *    entry a call reads was written earlier by the same call.  Calls whose
- *    execution overlaps on the GPU (other streams, or several host threads)
- *    race on the array: serialise them.
+ *    call's contents; nothing in it needs to start at zero: each call first
+ *    clears the row tickets it uses (a small kernel in the same stream), and
+ *    every other entry it reads was written earlier by the same call.  Calls
+ *    whose execution overlaps on the GPU (other streams, or several host
+ *    threads) race on the array: serialise them.
  *  - A problem whose scratch (eti_entropy_temp_sample_workspace_size(B, V))
  *    exceeds the array returns ETI_ERR_TOO_LARGE and enqueues nothing; at
- *    152 SMs the limit is about 9,700 sequences, whatever V is.
+ *    152 SMs the limit is about 14,500 sequences, whatever V is.
  */
 size_t eti_entropy_temp_sample_noalloc_max_bytes(void);
 
 int eti_entropy_temp_sample_noalloc(const float* logits, int B, int V, int64_t ld,
                                     const float* T_in, const float* H_prev, float* tau,
                                     const float* H_target, const eti_ctrl_params* params,
-                                    uint64_t seed, uint64_t offset,
+                                    uint64_t seed, uint64_t offset, uint64_t* offset_dev,
                                     int32_t* tok, float* H, float* T_out,
                                     float* dH, float* theta_next, float* tok_surprisal,
                                     const eti_surp_store* surp_store,
@@ -377,6 +392,21 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
                      const float* token_scores, const float* kept_norm,
                      eti_bf16* out, uint32_t* err_flags,
                      void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * eti_set_wait_limit -- a diagnostic setting, not part of the method (the
+ * paper has no counterpart): the number of polls after which a device-side
+ * wait for a tile copy (in the scoring pass and in the decode pass) gives up
+ * and reports ETI_ERRF_TIMEOUT for the sequences it serves.  It applies to
+ * every call launched afterwards from this process, on every device; it is
+ * the one setting of this library that outlives a call.  polls < 0 restores
+ * the default (2^20 polls, far beyond any copy's latency).  0 makes every
+ * such wait give up at once, which drives the error path without anything
+ * being stuck: the copies already issued are still waited for, with the
+ * default limit, before the kernel exits (ETI_ERRF_DRAIN if even that wait
+ * gives up).  Returns the previous limit.
+ */
+int64_t eti_set_wait_limit(int64_t polls);
 
 /* Version string and a readable name for a status code. */
 const char* eti_version(void);

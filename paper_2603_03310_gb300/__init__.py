@@ -22,10 +22,10 @@ _lib = None
 
 ETI_OK = 0
 STATUS = {0: "ok", -1: "null pointer", -2: "bad shape", -3: "unsupported shape",
-          -4: "workspace too small", -5: "CUDA launch failed", -6: "misaligned tensor",
-          -7: "too large for the fixed scratch"}
+          -4: "workspace too small", -5: "CUDA launch failed", -6: "device wait gave up (reserved)",
+          -7: "too large for the fixed scratch", -8: "misaligned tensor"}
 ERRF_BAD_PAGE, ERRF_BAD_CTX, ERRF_NONFINITE, ERRF_ALL_NEG_INF, ERRF_BAD_TEMP = 1, 2, 4, 8, 16
-ERRF_TIMEOUT = 32
+ERRF_TIMEOUT, ERRF_DRAIN = 32, 64
 
 # C-ABI symbols declared in include/eti.h
 SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_entropy_temp_sample_workspace_size",
@@ -34,7 +34,7 @@ SYMBOLS = ("eti_ctrl_defaults", "eti_entropy_temp_sample", "eti_entropy_temp_sam
            "eti_paged_decode_workspace_size", "eti_paged_decode", "eti_version",
            "eti_status_string", "eti_entropy_temp_sample_noalloc",
            "eti_entropy_temp_sample_noalloc_max_bytes", "eti_topk_entropy", "eti_sched_defaults",
-           "eti_schedule")
+           "eti_schedule", "eti_set_wait_limit")
 
 
 class EtiError(RuntimeError):
@@ -72,10 +72,12 @@ def load(path: str | None = None):
         lib.eti_status_string.restype = ctypes.c_char_p
         lib.eti_entropy_temp_sample_workspace_size.argtypes = [i32, i32]
         lib.eti_entropy_temp_sample_workspace_size.restype = sz
-        lib.eti_entropy_temp_sample.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64,
+        lib.eti_entropy_temp_sample.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64, P,
                                                 P, P, P, P, P, P, P, P, P, sz, P]
-        lib.eti_entropy_temp_sample_noalloc.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64,
+        lib.eti_entropy_temp_sample_noalloc.argtypes = [P, i32, i32, i64, P, P, P, P, P, u64, u64, P,
                                                         P, P, P, P, P, P, P, P, P]
+        lib.eti_set_wait_limit.argtypes = [i64]
+        lib.eti_set_wait_limit.restype = i64
         lib.eti_entropy_temp_sample_noalloc.restype = i32
         lib.eti_entropy_temp_sample_noalloc_max_bytes.restype = sz
         lib.eti_entropy_temp_sample.restype = i32
@@ -105,6 +107,13 @@ def load(path: str | None = None):
 
 def version() -> str:
     return load().eti_version().decode()
+
+
+def set_wait_limit(polls: int) -> int:
+    """Diagnostic: polls before a device-side tile wait gives up (< 0: the
+    default); applies to later calls of this process.  Returns the previous
+    limit (see eti_set_wait_limit in include/eti.h)."""
+    return int(load().eti_set_wait_limit(int(polls)))
 
 
 def ctrl_params(**kw) -> CtrlParams:
@@ -166,8 +175,10 @@ def _surp_store(surp_store, slot_mapping, B):
 def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, err_flags, ws,
                             params: CtrlParams | None = None, seed: int = 0, offset: int = 0,
                             dH=None, theta_next=None, tok_surprisal=None, V: int | None = None,
-                            surp_store=None, slot_mapping=None, stream=None):
-    """Half (a) of the step; see include/eti.h.  logits fp32 [B, ld]."""
+                            surp_store=None, slot_mapping=None, offset_dev=None, stream=None):
+    """Half (a) of the step; see include/eti.h.  logits fp32 [B, ld]; offset_dev:
+    an int64 CUDA tensor of one element that replaces `offset` and is advanced
+    by one after the call's draws."""
     B, ld = logits.shape
     V = ld if V is None else int(V)
     if logits.stride(1) != 1 or logits.stride(0) != ld:
@@ -178,6 +189,7 @@ def eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, tok, H, T_out, 
         _dev(logits, "logits", f32), B, V, ld, _dev(T_in, "T_in", f32, B),
         _dev(H_prev, "H_prev", f32, B), _dev(tau, "tau", f32, B), _dev(H_target, "H_target", f32, B),
         ctypes.byref(params), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+        _dev(offset_dev, "offset_dev", torch.int64, 1),
         _dev(tok, "tok", i32, B), _dev(H, "H", f32, B), _dev(T_out, "T_out", f32, B),
         _dev(dH, "dH", f32, B), _dev(theta_next, "theta_next", f32, B),
         _dev(tok_surprisal, "tok_surprisal", f32, B), _surp_store(surp_store, slot_mapping, B),
@@ -190,7 +202,7 @@ def eti_entropy_temp_sample_noalloc(logits, T_in, H_prev, tau, H_target, tok, H,
                                     params: CtrlParams | None = None, seed: int = 0,
                                     offset: int = 0, dH=None, theta_next=None, tok_surprisal=None,
                                     V: int | None = None, surp_store=None, slot_mapping=None,
-                                    stream=None):
+                                    offset_dev=None, stream=None):
     """eti_entropy_temp_sample without a workspace (fixed library scratch); see include/eti.h."""
     B, ld = logits.shape
     V = ld if V is None else int(V)
@@ -202,6 +214,7 @@ def eti_entropy_temp_sample_noalloc(logits, T_in, H_prev, tau, H_target, tok, H,
         _dev(logits, "logits", f32), B, V, ld, _dev(T_in, "T_in", f32, B),
         _dev(H_prev, "H_prev", f32, B), _dev(tau, "tau", f32, B), _dev(H_target, "H_target", f32, B),
         ctypes.byref(params), int(seed) & (2 ** 64 - 1), int(offset) & (2 ** 64 - 1),
+        _dev(offset_dev, "offset_dev", torch.int64, 1),
         _dev(tok, "tok", i32, B), _dev(H, "H", f32, B), _dev(T_out, "T_out", f32, B),
         _dev(dH, "dH", f32, B), _dev(theta_next, "theta_next", f32, B),
         _dev(tok_surprisal, "tok_surprisal", f32, B), _surp_store(surp_store, slot_mapping, B),
@@ -399,12 +412,12 @@ class DecodeStep:
                          kept_norm=self.kept_norm, num_pages=num_pages, stream=stream)
 
     def sample(self, logits, T_in, H_prev, tau, H_target, params=None, seed=0, offset=0, V=None,
-               stream=None):
+               offset_dev=None, stream=None):
         eti_entropy_temp_sample(logits, T_in, H_prev, tau, H_target, self.tok, self.H, self.T_out,
                                 self.err_ets, self.ws_ets, params=params, seed=seed, offset=offset,
                                 dH=self.dH,
                                 theta_next=self.theta_next, tok_surprisal=self.surprisal,
-                                V=V, stream=stream)
+                                V=V, offset_dev=offset_dev, stream=stream)
 
 
 def default_scale(D: int) -> float:

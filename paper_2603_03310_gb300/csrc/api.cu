@@ -1,6 +1,7 @@
 // api.cu -- the extern "C" boundary of libeti: argument validation, workspace
 // layout and the launch sequence of each entry point.  Declarations and the
 // full contract are in include/eti.h.
+#include <atomic>
 #include <cstring>
 
 #include "common.cuh"
@@ -9,9 +10,10 @@
 int eti_launch_entropy_temp_sample(const float* logits, int B, int V, long long ld,
                                    const float* T_in, const float* H_prev, float* tau,
                                    const float* H_target, const eti_ctrl_params* p,
-                                   uint64_t seed, uint64_t offset, int32_t* tok, float* H,
-                                   float* T_out, float* dH, float* theta_next, float* surprisal,
-                                   const eti_surp_store* store, uint32_t* err, void* part,
+                                   uint64_t seed, uint64_t offset, uint64_t* offset_dev,
+                                   int32_t* tok, float* H, float* T_out, float* dH,
+                                   float* theta_next, float* surprisal,
+                                   const eti_surp_store* store, uint32_t* err, void* scratch,
                                    cudaStream_t stream);
 size_t eti_entropy_partial_bytes(int B);
 int eti_launch_schedule(const float* dH, float* ema, const int32_t* kept_cnt, int Hkv, int P,
@@ -69,6 +71,9 @@ int eti_make_kv_tensor_map(CUtensorMap* map, const void* base, long long rows, i
 }
 
 namespace {
+
+// polls before a tile wait gives up (eti_set_wait_limit)
+std::atomic<int> g_wait_limit{eti::kMaxWaitIters};
 
 constexpr int kMaxB = 8192;
 constexpr int kMaxBlocks = 32768;
@@ -150,7 +155,12 @@ void eti_ctrl_defaults(eti_ctrl_params* p) {
     p->dtheta = 0.0f;
 }
 
-const char* eti_version(void) { return "libeti 0.1.0 (sm_103a)"; }
+const char* eti_version(void) { return "libeti 0.2.0 (sm_103a)"; }
+
+int64_t eti_set_wait_limit(int64_t polls) {
+    const int v = polls < 0 ? eti::kMaxWaitIters : (int)std::min<int64_t>(polls, 0x7fffffff);
+    return g_wait_limit.exchange(v);
+}
 
 const char* eti_status_string(int s) {
     switch (s) {
@@ -160,8 +170,9 @@ const char* eti_status_string(int s) {
         case ETI_ERR_UNSUPPORTED: return "shape not supported by this library";
         case ETI_ERR_WORKSPACE: return "workspace missing or too small";
         case ETI_ERR_CUDA: return "CUDA launch failed";
-        case ETI_ERR_ALIGN: return "a bf16 tensor is not 16-byte aligned";
+        case ETI_ERR_TIMEOUT: return "a device-side wait gave up (reserved: reported per sequence in err_flags)";
         case ETI_ERR_TOO_LARGE: return "problem exceeds the fixed scratch of the no-allocation entry point";
+        case ETI_ERR_ALIGN: return "a bf16 tensor is not 16-byte aligned";
         default: return "unknown status";
     }
 }
@@ -174,7 +185,7 @@ size_t eti_entropy_temp_sample_workspace_size(int B, int V) {
 int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
                             const float* T_in, const float* H_prev, float* tau,
                             const float* H_target, const eti_ctrl_params* params,
-                            uint64_t seed, uint64_t offset,
+                            uint64_t seed, uint64_t offset, uint64_t* offset_dev,
                             int32_t* tok, float* H, float* T_out,
                             float* dH, float* theta_next, float* tok_surprisal,
                             const eti_surp_store* surp_store,
@@ -186,9 +197,11 @@ int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
         return ETI_ERR_NULL;
     if (surp_store && (!surp_store->store || !surp_store->slot_mapping)) return ETI_ERR_NULL;
     if (!ws || ws_bytes < eti_entropy_temp_sample_workspace_size(B, V)) return ETI_ERR_WORKSPACE;
+    if ((reinterpret_cast<uintptr_t>(ws) & 3) != 0) return ETI_ERR_WORKSPACE;
     return eti_launch_entropy_temp_sample(logits, B, V, (long long)ld, T_in, H_prev, tau, H_target,
-                                          params, seed, offset, tok, H, T_out, dH, theta_next,
-                                          tok_surprisal, surp_store, err_flags, ws, (cudaStream_t)stream);
+                                          params, seed, offset, offset_dev, tok, H, T_out, dH,
+                                          theta_next, tok_surprisal, surp_store, err_flags, ws,
+                                          (cudaStream_t)stream);
 }
 
 int eti_topk_entropy(const float* logits, int B, int V, int64_t ld, const float* T_in, int k,
@@ -347,3 +360,5 @@ int eti_paged_decode(const eti_bf16* q, const eti_bf16* k_cache, const eti_bf16*
 }
 
 }  // extern "C"
+
+int eti_wait_limit() { return g_wait_limit.load(std::memory_order_relaxed); }

@@ -298,6 +298,9 @@ __device__ __forceinline__ int seq_blocks(int L, int P, int max_blocks) {
     return (L + P - 1) / P;
 }
 
+// Default number of polls before a wait for a tile copy gives up; the
+// kernels take their limit as an argument (eti_set_wait_limit), and the
+// drain after a timeout always uses this default.
 constexpr int kMaxWaitIters = 1 << 20;
 
 // Programmatic dependent launch: let the next kernel in the stream be
@@ -326,6 +329,9 @@ inline cudaError_t eti_launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 bloc
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
+
+// Host: the current wait limit for the tile waits (eti_set_wait_limit).
+int eti_wait_limit();
 
 // Host: a 2-D bf16 tensor map over a [rows][D] array with boxes of
 // 16 rows x 64 elements (128 bytes) and the 128-byte swizzle.

@@ -138,6 +138,7 @@ struct DecArgs {
     float* partial;                // [(nwarps + nseg)][g][D]
     int* ticket;                   // [nseg], zeroed by the plan kernel
     uint32_t* err;                 // [B], written by the plan kernel
+    int wait_iters;                // polls before a tile wait gives up (eti_set_wait_limit)
 };
 
 template <int D>
@@ -359,7 +360,7 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
         const int tile = i - (i / kTiles) * kTiles;
         if (tile == 0 && ((item - u0) & 31) == 0 && item > u0 && item - u0 + 32 < u1 - u0)
             resolve(((item - u0) >> 5) + 1);
-        if (!mbar_wait(bars + 8 * st, (uint32_t)((i / S) & 1), kMaxWaitIters)) {
+        if (!mbar_wait(bars + 8 * st, (uint32_t)((i / S) & 1), a.wait_iters)) {
             timed_out = true;
             break;
         }
@@ -415,10 +416,15 @@ paged_decode_kernel(const __grid_constant__ CUtensorMap vmap, const DecArgs a) {
         // a copy never arrived: let the ones in flight land (bounded), flag
         // every sequence of the rest of this range, and still close their
         // segments (tickets included) so no output is left unwritten
-        for (int k = i; k < ntiles && k < i + S; ++k) mbar_wait(bars + 8 * (k % S), (uint32_t)((k / S) & 1), 1024);
+        // (the drain waits with the default limit; a copy still in flight
+        // after it is reported as ETI_ERRF_DRAIN)
+        bool drained = true;
+        for (int k = i; k < ntiles && k < i + S; ++k)
+            drained &= mbar_wait(bars + 8 * (k % S), (uint32_t)((k / S) & 1), kMaxWaitIters);
+        const uint32_t bits = ETI_ERRF_TIMEOUT | (drained ? 0u : ETI_ERRF_DRAIN);
         for (int sg = cur_seg >= 0 ? cur_seg : a.warp_seg[warp]; sg < nseg && __ldg(a.cum + sg) < u1; ++sg) {
             if (__ldg(a.cum + sg + 1) <= __ldg(a.cum + sg)) continue;
-            if (lane == 0) atomicOr(a.err + sg / a.Hkv, ETI_ERRF_TIMEOUT);
+            if (lane == 0) atomicOr(a.err + sg / a.Hkv, bits);
             flush(sg);
         }
         zero_empty();
@@ -471,6 +477,7 @@ int eti_launch_decode(const uint16_t* v_cache, const int32_t* block_table, const
     da.B = B; da.Hq = Hq; da.Hkv = Hkv; da.g = Hq / Hkv; da.max_blocks = max_blocks;
     da.num_pages = num_pages; da.out = out; da.partial = partial;
     da.ticket = plan_ticket; da.err = err;
+    da.wait_iters = eti_wait_limit();
     const int grid = nwarps / kDecWarps;
     if (num_pages <= 0 || num_pages * Hkv * P >= (1LL << 31)) {
         if (num_pages > 0) return ETI_ERR_UNSUPPORTED;   // tile rows are int32 on the device

@@ -130,10 +130,25 @@ prune_finalize_wide_kernel(const FinArgs a) {
     int dummy;
     const bool bad_page = cl_count(__syncthreads_or(bad) != 0, &dummy) != 0;
     const bool timed_out = cl_count(__syncthreads_or(stale) != 0, &dummy) != 0 && !bad_page;
+    bool drain = false;
+    if (timed_out) {
+        // rare: a block marked l - 1 = +inf had a copy in flight when the drain gave up
+        int d = 0;
+        for (int r = r_lo; r < r_hi; ++r)
+#pragma unroll
+            for (int k = 0; k < kFlatPer; ++k) {
+                const int j = r * RB + jt + k * JS;
+                if (h < G && j < nb) {
+                    const float4 s4 = st[(long long)j * G + h];
+                    d |= (s4.x != s4.x) && s4.y == kInf;
+                }
+            }
+        drain = cl_count(__syncthreads_or(d) != 0, &dummy) != 0;
+    }
     if (a.err && tid == 0 && cr == 0) {
         // err was cleared before this kernel; every kv head ORs in its bits
         const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page ? ETI_ERRF_BAD_PAGE : 0u) |
-                           (timed_out ? ETI_ERRF_TIMEOUT : 0u);
+                           (timed_out ? ETI_ERRF_TIMEOUT : 0u) | (drain ? ETI_ERRF_DRAIN : 0u);
         if (e) atomicOr(a.err + b, e);
     }
     const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;

@@ -45,6 +45,7 @@ struct ScoreArgs {
     float4* stats;         // [B][Hkv][max_blocks][g]: (m, l - 1, u, e) with
                            // e = sum e^{x-m} s_i when tok_surp is given, else 0
     const float* tok_surp; // [num_pages][P] stored token surprisal s_i, or null
+    int wait_iters;        // polls before a tile wait gives up (eti_set_wait_limit)
 };
 
 // Exclusive prefix over sequences of (blocks * Hkv) into shared memory;
@@ -190,7 +191,7 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
         const int tile = i - (i / kTiles) * kTiles;
         if (tile == 0 && ((item - u0) & 31) == 0 && item > u0 && item - u0 + 32 < u1 - u0)
             resolve(((item - u0) >> 5) + 1);
-        if (!mbar_wait(bars + 8 * st, (uint32_t)((i / S) & 1), kMaxWaitIters)) {
+        if (!mbar_wait(bars + 8 * st, (uint32_t)((i / S) & 1), a.wait_iters)) {
             timed_out = true;
             break;
         }
@@ -313,16 +314,22 @@ score_blocks_kernel(const __grid_constant__ CUtensorMap kmap, const ScoreArgs a)
         }
     }
     if (timed_out) {
-        // a copy never arrived: let the copies still in flight land (bounded),
-        // then mark every block this warp did not finish with NaN stats, which
-        // the keep-set pass reports as ETI_ERRF_TIMEOUT for its sequence
-        for (int k = i; k < ntiles && k < i + S; ++k) mbar_wait(bars + 8 * (k % S), (uint32_t)((k / S) & 1), 1024);
+        // a copy never arrived: let the copies still in flight land (bounded
+        // by the default limit), then mark every block this warp did not
+        // finish with NaN stats, which the keep-set pass reports as
+        // ETI_ERRF_TIMEOUT for its sequence; l - 1 = +inf instead of NaN also
+        // says that a copy was still in flight when the drain gave up
+        // (ETI_ERRF_DRAIN)
+        bool drained = true;
+        for (int k = i; k < ntiles && k < i + S; ++k)
+            drained &= mbar_wait(bars + 8 * (k % S), (uint32_t)((k / S) & 1), kMaxWaitIters);
         const float nan = __int_as_float(0x7fc00000);
+        const float l1_mark = drained ? nan : kInf;
         for (int item = u0 + i / kTiles; item < u1; ++item) {
             if (((item - u0) & 31) == 0 && item > u0) resolve((item - u0) >> 5);
             const int4 e = entry(item);
             const long long unit = ((long long)e.x * a.Hkv + e.y) * a.max_blocks + e.z;
-            if (lane < a.g) a.stats[unit * a.g + lane] = make_float4(nan, nan, nan, 0.f);
+            if (lane < a.g) a.stats[unit * a.g + lane] = make_float4(nan, l1_mark, nan, 0.f);
         }
     }
 }
@@ -392,10 +399,21 @@ prune_finalize_flat_kernel(const FinArgs a) {
     }
     const bool bad_page = __syncthreads_or(bad) != 0;
     const bool timed_out = __syncthreads_or(stale) != 0 && !bad_page;
+    bool drain = false;
+    if (timed_out) {
+        // rare: a block marked l - 1 = +inf had a copy in flight when the drain gave up
+        int d = 0;
+#pragma unroll
+        for (int k = 0; k < kFlatPer; ++k) {
+            const int j = jt + k * JS;
+            if (h < G && j < nb) d |= (m[k] != m[k]) && l1[k] == kInf;
+        }
+        drain = __syncthreads_or(d) != 0;
+    }
     if (a.err && tid == 0) {
         // err was cleared before this kernel; every kv head ORs in its bits
         const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page ? ETI_ERRF_BAD_PAGE : 0u) |
-                           (timed_out ? ETI_ERRF_TIMEOUT : 0u);
+                           (timed_out ? ETI_ERRF_TIMEOUT : 0u) | (drain ? ETI_ERRF_DRAIN : 0u);
         if (e) atomicOr(a.err + b, e);
     }
     const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
@@ -612,6 +630,7 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
     a.B = B; a.Hq = Hq; a.Hkv = Hkv; a.g = Hq / Hkv; a.max_blocks = max_blocks;
     a.num_pages = num_pages; a.scale = scale; a.token_scores = token_scores; a.stats = stats;
     a.tok_surp = tok_surp;
+    a.wait_iters = eti_wait_limit();
     // tile row coordinates are int32 on the device
     if (num_pages * Hkv * P >= (1LL << 31)) return ETI_ERR_UNSUPPORTED;
     CUtensorMap kmap;

@@ -18,3 +18,11 @@ def oracle_lib():
     import oracle
     oracle.build()
     return oracle
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """One line with the parity counts of the session (near-ties accepted by
+    the stated rules, worst errors), so that a run's log keeps them."""
+    parity = sys.modules.get("parity")
+    if parity is not None and any(parity.TALLY.values()):
+        terminalreporter.write_line(parity.tally_line())

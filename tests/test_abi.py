@@ -46,7 +46,7 @@ def test_library_is_built_for_sm103a_only():
 
 def test_version_and_status_strings(lib):
     assert "libeti" in eti.version()
-    for s in (0, -1, -2, -3, -4, -5, -6):
+    for s in (0, -1, -2, -3, -4, -5, -6, -7, -8):
         assert lib.eti_status_string(s).decode()
 
 
@@ -71,21 +71,21 @@ def test_entropy_call_validation(lib):
     # tok, H, T_out, dH, theta_next, tok_surprisal, surp_store (a host struct), err_flags
     OUTS = [fake] * 6 + [NULL, fake]
     # bad shapes
-    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -2
-    assert f(fake, 4, 0, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -2
-    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -2
+    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, fake, ws, NULL) == -2
+    assert f(fake, 4, 0, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, fake, ws, NULL) == -2
+    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, fake, ws, NULL) == -2
     # B == 0 is a no-op
-    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, *[NULL] * 8, NULL, 0, NULL) == 0
+    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, NULL, *[NULL] * 8, NULL, 0, NULL) == 0
     # required pointers
-    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws, NULL) == -1
-    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, *OUTS, fake, ws, NULL) == -1
+    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, fake, ws, NULL) == -1
+    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, NULL, *OUTS, fake, ws, NULL) == -1
     # a surprisal store needs both of its arrays
     half = eti.SurpStore(fake, None, 16)
-    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *[fake] * 6, ctypes.byref(half),
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *[fake] * 6, ctypes.byref(half),
              fake, fake, ws, NULL) == -1
     # workspace
-    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL, ws, NULL) == -4
-    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, fake, ws - 1, NULL) == -4
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, NULL, ws, NULL) == -4
+    assert f(fake, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, fake, ws - 1, NULL) == -4
 
 
 def test_attention_call_validation(lib):
@@ -113,7 +113,7 @@ def test_attention_call_validation(lib):
     assert call(mb=40000) == -3
     assert call(B=9000) == -2
     assert call(q=NULL) == -1
-    assert call(q=bad) == -6
+    assert call(q=bad) == -8
     assert call(ws=NULL) == -4
     assert call(wsb=need - 1) == -4
     assert call(B=0, ws=NULL) == 0
@@ -134,7 +134,7 @@ def test_attention_call_validation(lib):
     assert g(a16, a16, a16, a16, a16, 4, 32, 8, 128, 16, 512, 1000, 0.1,
              NULL, NULL, NULL, NULL, NULL, a16, a16, a16, without - 1, NULL) == -4
     assert g(a16, a16, bad, a16, a16, 4, 32, 8, 128, 16, 512, 1000, 0.1,
-             NULL, NULL, NULL, NULL, NULL, a16, a16, a16, without, NULL) == -6
+             NULL, NULL, NULL, NULL, NULL, a16, a16, a16, without, NULL) == -8
 
 
 def test_binding_refuses_cpu_tensors(lib):
@@ -149,6 +149,17 @@ def test_binding_refuses_cpu_tensors(lib):
 def test_status_strings_cover_every_code(lib):
     for s in (-7,):
         assert "scratch" in lib.eti_status_string(s).decode()
+    assert "aligned" in lib.eti_status_string(-8).decode()
+    assert "wait" in lib.eti_status_string(-6).decode()
+
+
+def test_wait_limit_setting(lib):
+    # the diagnostic wait limit: set, read back through the previous value, restore
+    prev = eti.set_wait_limit(0)
+    assert prev == 1 << 20
+    assert eti.set_wait_limit(5) == 0
+    assert eti.set_wait_limit(-1) == 5
+    assert eti.set_wait_limit(-1) == 1 << 20
     assert lib.eti_status_string(-99).decode() == "unknown status"
 
 
@@ -203,7 +214,7 @@ def test_score_and_prune_call_validation(lib):
     for name in ("q", "k", "bt", "L", "stats"):
         assert score(**{name: NULL}) == -1, name
     for name in ("q", "k", "stats"):
-        assert score(**{name: bad}) == -6, name
+        assert score(**{name: bad}) == -8, name
 
     def prune(stats=a16, bt=a16, L=a16, B=4, Hq=32, Hkv=8, D=128, Pg=16, mb=512, pages=1000,
               theta=a16, mode=0, mask=a16, kidx=a16, kcnt=a16, err=a16):
@@ -217,7 +228,7 @@ def test_score_and_prune_call_validation(lib):
                  err=NULL) == 0
     for name in ("stats", "bt", "L", "theta", "mask", "kidx", "kcnt", "err"):
         assert prune(**{name: NULL}) == -1, name
-    assert prune(stats=bad) == -6
+    assert prune(stats=bad) == -8
 
 
 def test_noalloc_call_validation(lib):
@@ -228,11 +239,11 @@ def test_noalloc_call_validation(lib):
     prm = eti.ctrl_params()
     f = lib.eti_entropy_temp_sample_noalloc
     OUTS = [fake] * 6 + [NULL, fake]
-    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -2
-    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -2
-    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, *[NULL] * 8, NULL) == 0
-    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -1
-    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, *OUTS, NULL) == -1
+    assert f(fake, -1, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, NULL) == -2
+    assert f(fake, 4, 10, 9, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, NULL) == -2
+    assert f(NULL, 0, 10, 10, *[NULL] * 4, NULL, 0, 0, NULL, *[NULL] * 8, NULL) == 0
+    assert f(NULL, 4, 10, 10, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, NULL) == -1
+    assert f(fake, 4, 10, 10, *[fake] * 4, NULL, 0, 0, NULL, *OUTS, NULL) == -1
     # the largest batch whose scratch fits is accepted by the size check; one
     # more row than the array holds is refused with ETI_ERR_TOO_LARGE
     cap = lib.eti_entropy_temp_sample_noalloc_max_bytes()
@@ -245,7 +256,7 @@ def test_noalloc_call_validation(lib):
             lo = mid
         else:
             hi = mid
-    assert f(fake, hi, 4, 4, *[fake] * 4, ctypes.byref(prm), 0, 0, *OUTS, NULL) == -7
+    assert f(fake, hi, 4, 4, *[fake] * 4, ctypes.byref(prm), 0, 0, NULL, *OUTS, NULL) == -7
 
 
 def test_binding_constants_match_the_header():
@@ -274,7 +285,9 @@ int main(void) {
     if (eti_score_prune_workspace_size(4, 30, 8, 128, 16, 512) != 0) return 6;
     /* an argument error is reported before anything is enqueued */
     if (eti_entropy_temp_sample(NULL, 4, 10, 10, NULL, NULL, NULL, NULL, &p, 0, 0, NULL, NULL,
-                                NULL, NULL, NULL, NULL, NULL, NULL, NULL, 0, NULL) != ETI_ERR_NULL)
+                                NULL, NULL, NULL, NULL, NULL, NULL, NULL, NULL, 0, NULL) != ETI_ERR_NULL)
+        return 7;
+    if (eti_set_wait_limit(-1) != eti_set_wait_limit(-1))
         return 7;
     printf("ok %s\n", eti_version());
     return 0;

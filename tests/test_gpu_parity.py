@@ -175,6 +175,48 @@ def test_entropy_sample_reproducible(eti):
         assert np.array_equal(a[k], b[k]), k
 
 
+def _step_ets(st, tau):
+    """DecodeStep sampling outputs in the layout parity.compare_ets reads."""
+    res = dict(tok=st.tok, H=st.H, T_out=st.T_out, dH=st.dH, theta_next=st.theta_next,
+               surprisal=st.surprisal, err=st.err_ets, tau=tau)
+    res = {k: v.cpu().numpy() for k, v in res.items()}
+    res["err"] = res["err"].view(np.uint32)
+    return res
+
+
+def test_entropy_sample_device_offset(eti):
+    """offset_dev: the call reads the Philox offset from a device word and
+    leaves it advanced by one, so a captured graph replayed twice draws the
+    tokens of two consecutive offsets (each against the oracle)."""
+    w = workloads.WORKLOADS["llama3_8b"].scaled(B=16)
+    lg = workloads.make_logits(w, DEV)
+    st = eti.DecodeStep(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, w.V, device=DEV)
+    off = torch.tensor([41], dtype=torch.int64, device=DEV)
+    tau = lg["tau"].clone()
+    st.sample(lg["logits"], lg["T_in"], lg["H_prev"], tau, lg["H_target"], seed=2, offset=999,
+              offset_dev=off)
+    torch.cuda.synchronize()
+    assert off.item() == 42
+    parity.compare_ets(_step_ets(st, tau), parity.oracle_ets(lg, seed=2, offset=41), lg, seed=2, offset=41)
+    cs = torch.cuda.Stream(device=DEV)
+    cs.wait_stream(torch.cuda.current_stream())
+    graph = torch.cuda.CUDAGraph()
+    tau_g = lg["tau"].clone()
+    with torch.cuda.graph(graph, stream=cs):
+        st.sample(lg["logits"], lg["T_in"], lg["H_prev"], tau_g, lg["H_target"], seed=2, offset_dev=off)
+    torch.cuda.synchronize()
+    toks = []
+    for o in (42, 43):
+        tau_g.copy_(lg["tau"])
+        graph.replay()
+        torch.cuda.synchronize()
+        assert off.item() == o + 1
+        parity.compare_ets(_step_ets(st, tau_g), parity.oracle_ets(lg, seed=2, offset=o), lg, seed=2,
+                           offset=o)
+        toks.append(st.tok.clone())
+    assert not torch.equal(toks[0], toks[1])
+
+
 # ---------------------------------------------------------------------------
 # half (b): block scores, keep set, pruned paged decode
 
@@ -377,9 +419,13 @@ def _pool_for(w):
     return min(w.pool, 1 << max(10, cap.bit_length() - 1))
 
 
-@pytest.mark.parametrize("name,nsample", [("tiny", 4), ("llama3_8b", 4), ("long_ctx", 2),
-                                          ("mixed_batch", 6), ("llama3_70b", 2)])
+@pytest.mark.parametrize("name,nsample", [("tiny", 4), ("llama3_8b", 64), ("long_ctx", 8),
+                                          ("mixed_batch", 256), ("llama3_70b", 16)])
 def test_attention_full_workloads(eti, name, nsample):
+    """The step at full size in the benchmark's launch configuration: every
+    sequence of tiny, llama3_8b, long_ctx and mixed_batch and 16 of the 128
+    llama3_70b sequences (scores, keep set, kept lists, output, error words)
+    against the oracle on their gathered pages."""
     w = workloads.WORKLOADS[name]
     kv = workloads.make_kv(w, DEV, pool=_pool_for(w))
     lg = workloads.make_logits(w, DEV)
@@ -391,6 +437,7 @@ def test_attention_full_workloads(eti, name, nsample):
     seqs = sorted(rng.choice(w.B, size=min(nsample, w.B), replace=False).tolist())
     sub = parity.host_from_gather(workloads.gather_sequences(kv, seqs))
     s = _check_step(st, sub, theta.cpu().numpy()[seqs], B_min, w.P, seqs=seqs)
+    assert len(seqs) == min(nsample, w.B)
     kept = st.kept_cnt.sum().item()
     total = sum(-(-int(L) // w.P) for L in kv["ctx_lens"].cpu().numpy()) * w.Hkv
     print(name, s, f"kept fraction {kept / total:.3f}")

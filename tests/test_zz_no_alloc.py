@@ -112,6 +112,7 @@ def test_noalloc_rejects_problems_beyond_its_scratch(eti):
     import ctypes
     ptr = ctypes.c_void_p(x.data_ptr())
     st = lib.eti_entropy_temp_sample_noalloc(ptr, B, 4, 4, ptr, ptr, ptr, ptr, ctypes.byref(p),
-                                             0, 0, ptr, ptr, ptr, None, None, None, None, ptr, None)
+                                             0, 0, None, ptr, ptr, ptr, None, None, None, None, ptr,
+                                             None)
     assert st == -7
     assert "fixed scratch" in lib.eti_status_string(st).decode()
