@@ -17,7 +17,16 @@ event between its calls, so each kernel keeps its programmatic launch overlap
 with the one before), and a separate pass with an event between calls gives
 the per-kernel times behind `roofline`.  `value` = sequences decoded per
 second per layer step over all ranks (each rank decodes its own batch: weak
-scaling).
+scaling).  The clock sampler runs over the timed steps and a further
+--clock-seconds of the same step back to back (`clocks`, `clock_pass`).
+
+Beside the headline step the line carries: `dense_baseline` (the same batch
+decoded densely by the same library call), `sampling` (the entropy / sample
+pass against the HBM peak and against a read-only pass over the same logits),
+`e2e` (host buffers, copies inside the timed region, with a stage breakdown),
+`workloads` (tiny, long_ctx, mixed_batch and llama3_70b at H_target 0.1, 0.3
+and 0.5 log V: step time, tokens/s, kept fraction, per-kernel times and
+fractions of the peak), `keep_sweep`, `estimators` and `cpu_baseline`.
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload (the paper has no reference implementation).
@@ -211,12 +220,8 @@ def source_digest(paths) -> str:
 def ncu_traffic(kernel):
     """DRAM bytes per launch from the committed ncu record, if the kernel's
     code is unchanged since that capture (else None)."""
-    try:
-        rec = json.load(open(os.path.join(ROOT, "profiles", "ncu_traffic.json")))[kernel]
-        digest = source_digest(rec["sources"])
-    except (OSError, KeyError, TypeError, ValueError):
-        return None
-    return rec["bytes"] if digest == rec["sha256"] else None
+    rec = ncu_record(kernel)
+    return rec["bytes"] if rec else None
 
 
 def run_estimators(eti, lg, step, prm, w, flush_l2, stream, k=64, reps=50):
@@ -369,6 +374,168 @@ def run_keep_sweep(eti, device, flush_l2, stream, peak, fracs=(0.1, 0.25, 0.5, 1
                     "a dense decode that reads K and V of every block"}
 
 
+def pool_for(w, device) -> int | None:
+    """The workload's page pool, capped to the largest power of two of pages
+    (K + V) within a quarter of the free HBM: the mixed-batch recipe's 2^21
+    pages would need 256 GB.  None: exactly the pages the sequences use."""
+    if w.pool is None:
+        return None
+    free, _ = torch.cuda.mem_get_info(device)
+    page_bytes = 2 * w.Hkv * w.P * w.D * 2
+    cap = int(0.25 * free // page_bytes)
+    return min(w.pool, 1 << max(10, cap.bit_length() - 1))
+
+
+class StepRunner:
+    """One workload's inputs, buffers and the four calls of the step (score
+    -> keep set -> decode over the kept blocks -> entropy / sample)."""
+
+    def __init__(self, eti, w, device, prm, stream, H_target_frac=None):
+        self.eti, self.w, self.prm, self.stream = eti, w, prm, stream
+        self.pool = pool_for(w, device)
+        self.kv = workloads.make_kv(w, device, pool=self.pool)
+        self.lg = workloads.make_logits(w, device)
+        if H_target_frac is not None:
+            self.lg["H_target"].fill_(H_target_frac * math.log(w.V))
+        g = w.Hq // w.Hkv
+        self.step = eti.DecodeStep(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, w.V, device=device)
+        self.stats = torch.empty((w.B, w.Hkv, w.max_blocks, g, 4), dtype=torch.float32, device=device)
+        self.shape = (w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks)
+        self.B_min = 1
+        # threshold of this step: theta_next of the previous step's entropy (same logits)
+        tau0 = self.lg["tau"].clone()
+        self.step.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], tau0, self.lg["H_target"],
+                         params=prm, seed=w.seed)
+        self.theta = self.step.theta_next.clone()
+        self.L = self.kv["ctx_lens"].cpu().numpy()
+        self.total_blocks = int((-(-self.L // w.P)).sum()) * w.Hkv
+
+    def run(self, ev=None, offset=0):
+        """One step; with `ev` (5 events) an event between the calls."""
+        eti, kv, st, w = self.eti, self.kv, self.step, self.w
+        s = self.stream
+        if ev is not None:
+            ev[0].record(s)
+        eti.eti_score_blocks(kv["q"], kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
+                             self.stats, token_scores=st.token_scores, num_pages=kv["num_pages"])
+        if ev is not None:
+            ev[1].record(s)
+        eti.eti_prune_blocks(self.stats, kv["block_table"], kv["ctx_lens"], self.shape, self.theta, self.B_min,
+                             st.keep_mask, st.kept_idx, st.kept_cnt, st.err_attn, kept_norm=st.kept_norm,
+                             num_pages=kv["num_pages"])
+        if ev is not None:
+            ev[2].record(s)
+        eti.eti_paged_decode(kv["q"], kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
+                             kv["scale"], st.out, st.err_dec, st.ws_dec, kept_idx=st.kept_idx,
+                             kept_cnt=st.kept_cnt, token_scores=st.token_scores, kept_norm=st.kept_norm,
+                             num_pages=kv["num_pages"])
+        if ev is not None:
+            ev[3].record(s)
+        st.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], self.lg["tau"], self.lg["H_target"],
+                  params=self.prm, seed=w.seed, offset=offset)
+        if ev is not None:
+            ev[4].record(s)
+
+    def kept(self) -> int:
+        return int(self.step.kept_cnt.sum().item())
+
+
+def timed_median(fn, flush_l2, stream, reps):
+    """Median CUDA-event time (ms) of fn over reps calls, L2 flushed before each."""
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(reps)]
+    for i in range(reps + 2):
+        flush_l2()
+        if i >= 2:
+            ev[i - 2][0].record(stream)
+        fn()
+        if i >= 2:
+            ev[i - 2][1].record(stream)
+    torch.cuda.synchronize()
+    return statistics.median(e[0].elapsed_time(e[1]) for e in ev)
+
+
+NAMES = ("score", "prune", "decode", "sample")
+
+
+def kernel_pass(r, flush_l2, n, offset0):
+    """Per-call times (ms, mean over n steps) from a pass with an event between calls."""
+    evb = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(n)]
+    for i in range(n):
+        flush_l2()
+        r.run(evb[i], offset=offset0 + i)
+    torch.cuda.synchronize()
+    return {nm: statistics.mean(evb[i][j].elapsed_time(evb[i][j + 1]) for i in range(n))
+            for j, nm in enumerate(NAMES)}
+
+
+def dense_decode_ms(r, flush_l2, reps=20):
+    """The baseline the keep set is measured against: eti_paged_decode without
+    kept lists (every block: q.K scored and p.V accumulated over K and V of
+    every block, in the same library call)."""
+    eti, kv, w = r.eti, r.kv, r.w
+    ws = torch.empty(eti.paged_decode_workspace_size(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, False),
+                     dtype=torch.uint8, device=kv["q"].device)
+    out = torch.empty_like(r.step.out)
+    err = torch.empty_like(r.step.err_dec)
+
+    def dense():
+        eti.eti_paged_decode(kv["q"], kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
+                             kv["scale"], out, err, ws, num_pages=kv["num_pages"])
+    ms = timed_median(dense, flush_l2, r.stream, reps)
+    del ws, out, err
+    return ms
+
+
+def workload_summary(r, flush_l2, peak, steps, warmup, offset0=0):
+    """Step time, throughput, kept fraction and per-kernel times / fractions of
+    the HBM peak for one workload (same timing rules as the main line)."""
+    w = r.w
+    for i in range(warmup):
+        flush_l2()
+        r.run(offset=offset0 + i)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+    for i in range(steps):
+        flush_l2()
+        evs[i][0].record(r.stream)
+        r.run(offset=offset0 + warmup + i)
+        evs[i][1].record(r.stream)
+    torch.cuda.synchronize()
+    ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+    per = kernel_pass(r, flush_l2, min(steps, 50), offset0 + warmup + steps)
+    kept = r.kept()
+    ab = algorithmic_bytes(w, r.L, kept)
+    gbs = {n: ab[n] / (per[n] / 1e3) / 1e9 for n in NAMES}
+    out = {"workload": workload_desc(w), "steps": steps, "ms_per_step": round(ms, 5),
+           "tokens_per_s": round(w.B / (ms / 1e3), 1),
+           "kept_fraction": round(kept / max(1, r.total_blocks), 4),
+           "kernels_ms": {n: round(v, 5) for n, v in per.items()},
+           "kernels_gbs": {n: round(v, 1) for n, v in gbs.items()},
+           "kernels_frac_of_peak": {n: round(v / peak, 4) for n, v in gbs.items()}}
+    if r.pool is not None:
+        out["page_pool"] = r.pool
+    return out
+
+
+def read_floor(lg, flush_l2, stream, reps=50):
+    """A size-matched read-only floor for the sampling pass: torch.sum over the
+    same logits, L2 flushed before each call (median ms, GB/s)."""
+    ms = timed_median(lambda: lg["logits"].sum(), flush_l2, stream, reps)
+    byt = lg["logits"].numel() * 4
+    return {"kernel": "torch.sum over the same logits", "ms": round(ms, 5),
+            "gbs": round(byt / (ms / 1e3) / 1e9, 1)}
+
+
+def ncu_record(kernel):
+    """The committed ncu record of a kernel (bytes, instructions, ...), if its
+    code is unchanged since that capture (else None)."""
+    try:
+        rec = json.load(open(os.path.join(ROOT, "profiles", "ncu_traffic.json")))[kernel]
+        digest = source_digest(rec["sources"])
+    except (OSError, KeyError, TypeError, ValueError):
+        return None
+    return rec if digest == rec["sha256"] else None
+
+
 def run_gpu(args):
     import paper_2603_03310_gb300 as eti
 
@@ -380,20 +547,9 @@ def run_gpu(args):
         dist.init_process_group("nccl", device_id=device)
     eti.load()
     w = shard_workload(workloads.WORKLOADS[args.workload], rank)
-    kv = workloads.make_kv(w, device)
-    lg = workloads.make_logits(w, device)
-    g = w.Hq // w.Hkv
-    step = eti.DecodeStep(w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, w.V, device=device)
-    stats = torch.empty((w.B, w.Hkv, w.max_blocks, g, 4), dtype=torch.float32, device=device)
-    shape = (w.B, w.Hq, w.Hkv, w.D, w.P, w.max_blocks)
     prm = eti.ctrl_params()
-    # threshold of this step: theta_next of the previous step's entropy (same logits)
-    tau0 = lg["tau"].clone()
-    step.sample(lg["logits"], lg["T_in"], lg["H_prev"], tau0, lg["H_target"], params=prm,
-                seed=w.seed)
-    theta = step.theta_next.clone()
-    B_min = 1
     stream = torch.cuda.current_stream()
+    r = StepRunner(eti, w, device, prm, stream)
     L2 = torch.cuda.get_device_properties(device).L2_cache_size
     flush_w = torch.empty(max(2 * L2, 256 << 20), dtype=torch.uint8, device=device)
     flush_r = torch.ones(max(2 * L2, 256 << 20) // 4, dtype=torch.int32, device=device)
@@ -405,37 +561,17 @@ def run_gpu(args):
         flush_w.zero_()
         flush_r.sum()
 
-    def one_step(ev=None, offset=0):
-        if ev is not None:
-            ev[0].record(stream)
-        eti.eti_score_blocks(kv["q"], kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
-                             stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
-        if ev is not None:
-            ev[1].record(stream)
-        eti.eti_prune_blocks(stats, kv["block_table"], kv["ctx_lens"], shape, theta, B_min,
-                             step.keep_mask, step.kept_idx, step.kept_cnt, step.err_attn,
-                             kept_norm=step.kept_norm, num_pages=kv["num_pages"])
-        if ev is not None:
-            ev[2].record(stream)
-        eti.eti_paged_decode(kv["q"], kv["k_cache"], kv["v_cache"], kv["block_table"],
-                             kv["ctx_lens"], kv["scale"], step.out, step.err_dec, step.ws_dec,
-                             kept_idx=step.kept_idx, kept_cnt=step.kept_cnt,
-                             token_scores=step.token_scores, kept_norm=step.kept_norm,
-                             num_pages=kv["num_pages"])
-        if ev is not None:
-            ev[3].record(stream)
-        step.sample(lg["logits"], lg["T_in"], lg["H_prev"], lg["tau"], lg["H_target"], params=prm,
-                    seed=w.seed, offset=offset)
-        if ev is not None:
-            ev[4].record(stream)
+    try:
+        peak, peak_src = float(json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        peak, peak_src = 6800.0, "fallback"
 
     for i in range(args.warmup):
         flush_l2()
-        one_step(offset=i)
+        r.run(offset=i)
     torch.cuda.synchronize()
-    kept = int(step.kept_cnt.sum().item())
-    L = kv["ctx_lens"].cpu().numpy()
-    total_blocks = int((-(-L // w.P)).sum()) * w.Hkv
+    kept = r.kept()
+    total_blocks = r.total_blocks
     # the timed steps carry one event pair each (no event between the calls, so
     # every kernel keeps its programmatic launch overlap with the one before);
     # the per-kernel breakdown comes from a separate pass with an event per call
@@ -448,51 +584,67 @@ def run_gpu(args):
     if args.clock_log:
         clock_log = args.clock_log.replace("{rank}", str(rank))
         os.makedirs(os.path.dirname(os.path.abspath(clock_log)), exist_ok=True)
+    off = args.warmup
     with ClockSampler(local, clock_log) as clk:
         t0 = time.perf_counter()
         for i in range(args.steps):
             flush_l2()
             evs[i][0].record(stream)
-            one_step(offset=args.warmup + i)
+            r.run(offset=off + i)
             evs[i][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
+        timed_samples = len(clk.lines)
+        off += args.steps
+        # the same step back to back for args.clock_seconds more, so that the
+        # clock record holds enough samples whatever K is
+        cp = None
+        if args.clock_seconds > 0:
+            ncp, t1 = 0, time.perf_counter()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            while time.perf_counter() - t1 < args.clock_seconds:
+                for _ in range(50):
+                    flush_l2()
+                    r.run(offset=off + ncp)
+                    ncp += 1
+                torch.cuda.synchronize()
+            e1.record(stream)
+            torch.cuda.synchronize()
+            off += ncp
+            cp = {"steps": ncp, "seconds": round(time.perf_counter() - t1, 3),
+                  "ms_per_step_with_flush": round(e0.elapsed_time(e1) / ncp, 5)}
     if world > 1:
         dist.barrier()
     step_ms = [evs[i][0].elapsed_time(evs[i][1]) for i in range(args.steps)]
-    names = ["score", "prune", "decode", "sample"]
-    nb = min(args.steps, 300)
-    evb = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(nb)]
-    for i in range(nb):
-        flush_l2()
-        one_step(evb[i], offset=args.warmup + args.steps + i)
-    torch.cuda.synchronize()
-    per = {n: [evb[i][j].elapsed_time(evb[i][j + 1]) for i in range(nb)] for j, n in enumerate(names)}
+    clocks = clk.summary()
+    if clocks is not None:
+        clocks["timed_region_samples"] = timed_samples
+    if cp is not None and clocks is not None:
+        cp["sm_mhz_median"] = clocks["sm_mhz"]
+    mean_ms = kernel_pass(r, flush_l2, min(args.steps, 300), off)
+    off += min(args.steps, 300)
     # share of the attention the keep set retains (outside the timed region;
     # a diagnostic never fails the run)
     try:
-        kept_mass = kept_attention_mass(stats, step.keep_mask, kv["ctx_lens"], w.P)
+        kept_mass = kept_attention_mass(r.stats, r.step.keep_mask, r.kv["ctx_lens"], w.P)
     except Exception as ex:
         kept_mass = {"error": f"{type(ex).__name__}: {ex}"}
     ms_local = statistics.mean(step_ms)
     ms = max_over_ranks(ms_local, world, device)
     value, _ = aggregate([ms / 1e3] * world, w.B)
-    mean_ms = {n: statistics.mean(v) for n, v in per.items()}
-    abytes = algorithmic_bytes(w, L, kept)
+    if cp is not None:
+        cp["kcycles_per_step"] = round(ms * (clocks or {}).get("sm_mhz", 0.0), 1)
+    abytes = algorithmic_bytes(w, r.L, kept)
     dom = max(mean_ms, key=mean_ms.get)
-    peaks = {}
-    try:
-        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
-        peak, peak_src = float(peaks["hbm_gbs"]), "measured"
-    except (OSError, KeyError, ValueError):
-        peak, peak_src = 6800.0, "fallback"
-    achieved = {n: abytes[n] / (mean_ms[n] / 1e3) / 1e9 for n in names}
-    traffic = args.traffic if args.traffic is not None else ncu_traffic(
-        {"score": "score_blocks", "prune": "prune_finalize", "decode": "paged_decode",
-         "sample": "entropy_sample_partial"}.get(dom))
+    achieved = {n: abytes[n] / (mean_ms[n] / 1e3) / 1e9 for n in NAMES}
+    rec_name = {"score": "score_blocks", "prune": "prune_finalize", "decode": "paged_decode",
+                "sample": "entropy_sample"}
+    rec = ncu_record(rec_name[dom])
+    traffic = args.traffic if args.traffic is not None else (rec["bytes"] if rec else None)
     roof = {"kernel": {"score": "score_blocks", "prune": "prune_finalize",
                        "decode": "paged_decode (plan + decode; split segments merged in-kernel)",
-                       "sample": "entropy_temp_sample"}[dom],
+                       "sample": "entropy_temp_sample (ticket clear + pass)"}[dom],
             "bound": "hbm", "achieved": round(achieved[dom], 1), "peak": peak, "unit": "GB/s",
             "frac": round(achieved[dom] / peak, 4), "peak_source": peak_src,
             "bytes_per_launch": abytes[dom], "ms_per_launch": round(mean_ms[dom], 5),
@@ -500,66 +652,117 @@ def run_gpu(args):
             "traffic_note": "ncu dram read+write per launch of the main kernel (profiles/), "
                             "null if its source changed since the capture"}
 
+    # the keep set against dense attention on the same batch (paper Section 6.7)
+    attn_ms = mean_ms["score"] + mean_ms["prune"] + mean_ms["decode"]
+    dms = dense_decode_ms(r, flush_l2)
+    dense = {"dense_decode_ms": round(dms, 5), "attention_ms": round(attn_ms, 5),
+             "speedup_vs_dense": round(dms / attn_ms, 3),
+             "note": "attention_ms = score + keep set + decode over the kept blocks (kernels_ms); "
+                     "dense = eti_paged_decode without kept lists on the same batch (every block "
+                     "scored, then K and V of every block)"}
+    # the sampling pass against a read-only pass over the same bytes
+    floor = read_floor(r.lg, flush_l2, stream)
+    srec = ncu_record("entropy_sample")
+    sampling = {"ms": round(mean_ms["sample"], 5), "gbs": round(achieved["sample"], 1),
+                "frac_of_peak": round(achieved["sample"] / peak, 4), "read_floor": floor,
+                "frac_of_read_floor": round(floor["ms"] / mean_ms["sample"], 4),
+                "inst_per_logit": (round(srec["inst_executed"] * 32 / (w.B * w.V), 2)
+                                   if srec and srec.get("inst_executed") else None),
+                "inst_note": "smsp__inst_executed x 32 lanes / logits of the pass kernel, from the "
+                             "committed ncu record (null if the kernel changed since)"}
+
     # top-k entropy estimators (Section 2.1) on the same logits: cost next to the
     # exact pass, and how they track the exact entropy of the step
     est = None
     if not args.no_estimators:
-        est = run_estimators(eti, lg, step, prm, w, flush_l2, stream)
-        est["schedule_ms"] = run_schedule(eti, step, kv, w, stream)
+        est = run_estimators(eti, r.lg, r.step, prm, w, flush_l2, stream)
+        est["schedule_ms"] = run_schedule(eti, r.step, r.kv, w, stream)
+
+    # end to end through the public API: host (pinned) inputs -> device -> step -> host results
+    e2e = None if args.no_e2e else run_e2e(eti, r, args, device)
+    if e2e is not None:
+        e2e = aggregate_e2e(e2e, w.B, world, device)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, r.kv, r.lg, r.theta, r.B_min, budget_s=args.cpu_budget)
+    main_desc = workload_desc(w)
+    del r
+    torch.cuda.empty_cache()
 
     sweep = None if args.no_sweep else run_keep_sweep(eti, device, flush_l2, stream, peak)
 
-    # end to end through the public API: host (pinned) inputs -> device -> step -> host results
-    e2e = None if args.no_e2e else run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm,
-                                           args, device)
-    if e2e is not None:
-        e2e = aggregate_e2e(e2e, w.B, world, device)
+    # the other workloads (the same step and timing rules, fewer steps)
+    others = None
+    if not args.no_workloads:
+        others = {}
+        ksteps = max(20, min(args.steps, 200))
+        for name in ("tiny", "long_ctx", "mixed_batch", "llama3_70b"):
+            if name == args.workload:
+                continue
+            ow = shard_workload(workloads.WORKLOADS[name], rank)
+            fracs = (0.1, 0.3, 0.5) if name == "llama3_70b" else (None,)
+            res = []
+            for f in fracs:
+                ro = StepRunner(eti, ow, device, prm, stream, H_target_frac=f)
+                s = workload_summary(ro, flush_l2, peak, ksteps, 5)
+                if f is not None:
+                    s["H_target"] = f"{f} log V"
+                res.append(s)
+                del ro
+                torch.cuda.empty_cache()
+            others[name] = res[0] if len(res) == 1 else {"H_target_sweep": res}
 
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16/fp32",
         "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
-        "config": {"workload": workload_desc(w),
+        "config": {"workload": main_desc,
                    "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write, then 2x L2 read)",
-                   "parallelism": f"replicas x{world} (independent batches)", "B_min": B_min,
+                   "parallelism": f"replicas x{world} (independent batches)", "B_min": 1,
                    "theta": "theta_next of the step's own entropy (defaults)",
-                   "kept_fraction": round(kept / total_blocks, 4)},
+                   "kept_fraction": round(kept / max(1, total_blocks), 4)},
         "roofline": roof,
         "kernels_ms": {n: round(v, 5) for n, v in mean_ms.items()},
         "kernels_ms_note": "per call, from a separate pass with an event between calls (the timed "
                            "steps have none, so their sum can exceed ms_per_step)",
         "kernels_gbs": {n: round(v, 1) for n, v in achieved.items()},
         "entropy_sample_gbs": round(achieved["sample"], 1),
-        "attention_tbs": round((abytes["score"] + abytes["decode"]) /
-                               ((mean_ms["score"] + mean_ms["prune"] + mean_ms["decode"]) / 1e3) / 1e12, 3),
+        "sampling": sampling,
+        "attention_tbs": round((abytes["score"] + abytes["decode"]) / (attn_ms / 1e3) / 1e12, 3),
+        "dense_baseline": dense,
         "gpu_launches": 7 * args.steps,
         "launches_per_step": {"score_blocks": 1, "clear_words (keep-set error words)": 1,
                               "prune_finalize": 1, "decode_plan": 1, "paged_decode": 1,
-                              "entropy_sample_partial": 1, "entropy_sample_finalize": 1},
+                              "ets_clear (sampling tickets)": 1, "entropy_sample": 1},
         "e2e": e2e,
         "estimators": est,
         "keep_sweep": sweep,
+        "workloads": others,
         "kept_attention_mass": kept_mass,
         "wall_s_timed_region": round(wall, 4),
-        "clocks": clk.summary(),
+        "clocks": clocks,
+        "clock_pass": cp,
     }
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(w, kv, lg, theta, B_min, budget_s=args.cpu_budget)
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
 
 
-def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device):
+def run_e2e(eti, r, args, device):
     """Same metric through the public API from pinned host buffers: per step the
     step's inputs (q, logits, per-sequence state, threshold) go host -> device and
-    its results (attention output, token, entropy, temperature, threshold) come back."""
+    its results (attention output, token, entropy, temperature, threshold) come
+    back.  Returns the figure and the time of each stage (an eager pass with
+    events at the stage boundaries)."""
     # One byte buffer per direction for the small per-step data, so each
     # direction costs one copy (a small copy costs ~12 us whatever its size):
     #   [q | T_in H_prev H_target theta | tau theta_next tok H T_out surprisal err]
     # goes up as far as tau (q, the state, tau) and comes back from tau on.
+    w, kv, lg, step, prm = r.w, r.kv, r.lg, r.step, r.prm
     B = w.B
     qb = kv["q"].numel() * 2
     row = B * 4
@@ -571,33 +774,45 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
     th_next, H_out, T_out, surp = rows[5], rows[7], rows[8], rows[9]
     tok, err = rows[6].view(torch.int32), rows[10].view(torch.int32)
     d_io[:qb].view(torch.bfloat16).copy_(kv["q"].reshape(-1))
-    rows[:5].copy_(torch.stack([lg["T_in"], lg["H_prev"], lg["H_target"], theta, lg["tau"]]))
+    rows[:5].copy_(torch.stack([lg["T_in"], lg["H_prev"], lg["H_target"], r.theta, lg["tau"]]))
     h_in = d_io[:n_in].cpu().pin_memory()
     h_res = torch.empty(n_all - (qb + 4 * row), dtype=torch.uint8).pin_memory()
     h_logits = lg["logits"].cpu().pin_memory()
     d_logits = torch.empty_like(lg["logits"])
     h_out = torch.empty(step.out.shape, dtype=step.out.dtype).pin_memory()
+    off_dev = torch.zeros(1, dtype=torch.int64, device=device)   # Philox offset, advanced by each call
 
-    # The logits (the bulk of the bytes) go up on a copy stream while the
-    # attention half runs; the sampling call waits for them.  The attention
+    # The small inputs go up first; the logits (the bulk of the bytes) then go
+    # up on a copy stream while the attention half runs; the sampling call
+    # waits for them.  The attention
     # output comes down on the copy stream while the sampling call runs.  The
     # whole step (copies and calls, both streams) is captured once in a CUDA
-    # graph and replayed every step, as a serving loop would; if the capture
-    # is refused the same body runs eagerly.
+    # graph and replayed every step, as a serving loop would; the sampling
+    # offset lives in device memory (the call advances it), so every replay
+    # draws fresh numbers.  If the capture is refused the same body runs eagerly.
     main = torch.cuda.current_stream()
     copy = torch.cuda.Stream(device=device)
     ev_logits = torch.cuda.Event()
     ev_out = torch.cuda.Event()
+    stages = ("start", "logits_up_start", "logits_up_end", "small_up_end", "attention_end", "out_down_end",
+              "sample_end", "results_down_end", "end")
 
-    def body(i, cur):
+    def body(cur, mk=None):
+        rec = (lambda name, s: mk[name].record(s)) if mk is not None else (lambda name, s: None)
+        rec("start", cur)
+        # the small inputs go first: both uploads use the same copy engine, in
+        # the order they are issued, and the attention half waits only for these
+        d_io[:n_in].copy_(h_in, non_blocking=True)
+        rec("small_up_end", cur)
         copy.wait_stream(cur)                                  # fork
         with torch.cuda.stream(copy):
+            rec("logits_up_start", copy)
             d_logits.copy_(h_logits, non_blocking=True)
             ev_logits.record(copy)
-        d_io[:n_in].copy_(h_in, non_blocking=True)
+            rec("logits_up_end", copy)
         eti.eti_score_blocks(d_q, kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
-                             stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
-        eti.eti_prune_blocks(stats, kv["block_table"], kv["ctx_lens"], shape, th, B_min,
+                             r.stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
+        eti.eti_prune_blocks(r.stats, kv["block_table"], kv["ctx_lens"], r.shape, th, r.B_min,
                              step.keep_mask, step.kept_idx, step.kept_cnt, step.err_attn,
                              kept_norm=step.kept_norm, num_pages=kv["num_pages"])
         eti.eti_paged_decode(d_q, kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
@@ -606,32 +821,62 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
                              token_scores=step.token_scores, kept_norm=step.kept_norm,
                              num_pages=kv["num_pages"])
         ev_out.record(cur)
+        rec("attention_end", cur)
         with torch.cuda.stream(copy):
             copy.wait_event(ev_out)
             h_out.copy_(step.out, non_blocking=True)
+            rec("out_down_end", copy)
         cur.wait_event(ev_logits)
         eti.eti_entropy_temp_sample(d_logits, T_in, H_prev, tau, H_tgt, tok, H_out, T_out, err,
-                                    step.ws_ets, params=prm, seed=w.seed, offset=i,
+                                    step.ws_ets, params=prm, seed=w.seed, offset_dev=off_dev,
                                     theta_next=th_next, tok_surprisal=surp)
+        rec("sample_end", cur)
         h_res.copy_(d_io[qb + 4 * row:], non_blocking=True)
+        rec("results_down_end", cur)
         cur.wait_stream(copy)                                  # join
+        rec("end", cur)
 
-    for i in range(args.warmup):
-        body(i, main)
+    for _ in range(args.warmup):
+        body(main)
         main.synchronize()
-    mode = "cuda graph replay (copies and calls of one step; fixed sampling offset)"
+    # where the time of one step goes (eager, events at the stage boundaries)
+    n_bd = 20
+    marks = [{s: torch.cuda.Event(enable_timing=True) for s in stages} for _ in range(n_bd)]
+    for i in range(n_bd):
+        body(main, marks[i])
+        main.synchronize()
+
+    def span(a, b):
+        return statistics.median(m[a].elapsed_time(m[b]) for m in marks)
+    breakdown = {
+        "logits_upload_ms": span("logits_up_start", "logits_up_end"),
+        "small_upload_ms": span("start", "small_up_end"),
+        "attention_ms": span("small_up_end", "attention_end"),
+        "out_download_ms": span("attention_end", "out_down_end"),
+        "logits_ready_after_attention_ms": span("attention_end", "logits_up_end"),
+        "sample_ms": span("attention_end", "sample_end"),
+        "results_download_ms": span("sample_end", "results_down_end"),
+        "device_span_ms": span("start", "end"),
+    }
+    breakdown = {k: round(v, 4) for k, v in breakdown.items()}
+    breakdown["note"] = ("eager pass with events at the stage boundaries (median of 20); sample_ms "
+                         "includes any wait for the logits upload; logits_ready_after_attention_ms < 0 "
+                         "means the upload finished before the attention half")
+    mode = "cuda graph replay (copies and calls of one step; sampling offset in device memory)"
     graph, gs = None, torch.cuda.Stream(device=device)
     try:
         gs.wait_stream(main)
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=gs):
-            body(args.warmup, gs)
+            body(gs)
         graph.replay()                 # on the current stream, like every replay below
         torch.cuda.synchronize()
     except Exception as ex:                                    # capture refused: eager steps
         graph = None
         mode = f"eager (graph capture refused: {type(ex).__name__})"
         torch.cuda.synchronize()
+    o0 = int(off_dev.item())
+    toks = []
     times = []
     for i in range(args.steps):
         t0 = time.perf_counter()
@@ -641,14 +886,20 @@ def run_e2e(eti, w, kv, lg, step, stats, theta, B_min, shape, prm, args, device)
             graph.replay()
             torch.cuda.synchronize()
         else:
-            body(args.warmup + i, main)
+            body(main)
             main.synchronize()
         times.append(time.perf_counter() - t0)
+        if i < 2:
+            toks.append(h_res[2 * row:3 * row].view(torch.int32).clone())
     s = statistics.mean(times)
     bi = h_in.numel() + h_logits.numel() * 4
     bo = h_out.numel() * 2 + h_res.numel()
+    breakdown["host_and_launch_ms"] = round(s * 1e3 - breakdown["device_span_ms"], 4)
     return {"value": round(w.B / s, 1), "unit": UNIT, "ms_per_step": round(s * 1e3, 4),
             "h2d_bytes_per_step": int(bi), "d2h_bytes_per_step": int(bo), "mode": mode,
+            "offset_advanced": int(off_dev.item()) - o0,
+            "fresh_tokens_per_replay": bool(len(toks) == 2 and not torch.equal(toks[0], toks[1])),
+            "breakdown": breakdown,
             "l2": "not flushed: every step uploads its logits and reads "
                   f"{(key_bytes(w, kv) / 1e9):.2f} GB of keys plus the kept values, more than the L2"}
 
@@ -761,6 +1012,10 @@ def main(argv=None):
                     help="skip the long-context keep-fraction sweep (decode time against kept blocks)")
     ap.add_argument("--no-estimators", action="store_true",
                     help="skip the top-k entropy estimator line")
+    ap.add_argument("--no-workloads", action="store_true",
+                    help="skip the other four workloads (tiny, long_ctx, mixed_batch, llama3_70b)")
+    ap.add_argument("--clock-seconds", type=float, default=2.0,
+                    help="seconds of back-to-back steps after the timed ones, under the clock sampler")
     ap.add_argument("--clock-log", default=None,
                     help="also write the raw nvidia-smi clock samples of the timed region to this "
                          "CSV file ({rank} is replaced by the rank)")
