@@ -31,7 +31,14 @@ struct FinArgs {
     float* block_score;     // nullable
     float* kept_norm;       // nullable: [B][Hq][2]
     uint32_t* err;          // nullable
+    int share_cache;        // wide kernel with the term cache: also cache each
+                            // block-head's share (1 + l1) e^{m - M} of Z
 };
+
+// e^d for d <= 0 (a block's weight against the head's max) with the MUFU
+// exp2: relative error about 2^-22 plus |d| 2^-24 from the scaling, far below
+// the 1e-5 keep-decision ties; weights below 2^-126 flush to zero.
+__device__ __forceinline__ float exp_le0(float d) { return fast_ex2(d * kLog2e); }
 
 __device__ __forceinline__ uint32_t order_key(float f) {
     if (f != f) return 0u;
@@ -72,6 +79,43 @@ __device__ __forceinline__ void head_reduce(float (&v)[N], float* red) {
         }
         v[i] = r;
     }
+}
+
+// The same reduction in two stages, for CTAs of many warps: after the warps'
+// partials are in `red`, warp u < GP reduces head u's partials over the warps
+// (one load per lane, a shuffle butterfly) and publishes it in `fin`
+// (N * GP floats), so that each thread reads one value per reduction instead of
+// one per warp.  Two barriers.
+template <int GP, int N, bool kMax>
+__device__ __forceinline__ void head_reduce2(float (&v)[N], float* red, float* fin) {
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int o = 16; o >= GP; o >>= 1)
+#pragma unroll
+        for (int i = 0; i < N; ++i) {
+            const float y = __shfl_xor_sync(0xffffffffu, v[i], o);
+            v[i] = kMax ? fmaxf(v[i], y) : v[i] + y;
+        }
+    if (lane < GP)
+#pragma unroll
+        for (int i = 0; i < N; ++i) red[(i * 32 + w) * GP + lane] = v[i];
+    __syncthreads();
+    if (w < GP) {
+#pragma unroll
+        for (int i = 0; i < N; ++i) {
+            float r = lane < nw ? red[(i * 32 + lane) * GP + w] : (kMax ? -kInf : 0.f);
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                const float y = __shfl_xor_sync(0xffffffffu, r, o);
+                r = kMax ? fmaxf(r, y) : r + y;
+            }
+            if (lane == 0) fin[i * GP + w] = r;
+        }
+    }
+    __syncthreads();
+    const int h = lane & (GP - 1);
+#pragma unroll
+    for (int i = 0; i < N; ++i) v[i] = fin[i * GP + h];
 }
 
 // Exclusive ranks in ascending block order of the flagged blocks (flags

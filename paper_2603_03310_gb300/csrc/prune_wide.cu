@@ -26,7 +26,7 @@ namespace eti {
 constexpr int kWideX = 16;    // exchange slots (one per exchange, never reused)
 
 template <int G, int NT, bool kTerm, int kCl>
-__global__ void __launch_bounds__(NT, 1024 / NT)
+__global__ void __launch_bounds__(NT, NT >= 1024 ? 1 : 2)
 prune_finalize_wide_kernel(const FinArgs a) {
     constexpr int GP = FlatGP<G>::v;
     constexpr int JS = NT / GP;                  // block stride between a thread's chunks
@@ -36,9 +36,14 @@ prune_finalize_wide_kernel(const FinArgs a) {
     extern __shared__ __align__(16) float wf_smem[];
     float* sh = wf_smem;                         // [max_blocks]: group scores, then keep flags
     // kTerm: [max_blocks * GP] per block-head e^{m_b - M}, then the term I_b
-    // (index j * GP + h: a warp's accesses are consecutive)
+    // (index j * GP + h: a warp's accesses are consecutive); with
+    // a.share_cache also [max_blocks * GP] shares (1 + l1_b) e^{m_b - M} of Z,
+    // which give the kept-token normaliser when the head's top block is kept
     float* sh_t = wf_smem + a.max_blocks;
+    float* sh_s = sh_t + (size_t)a.max_blocks * GP;
+    const bool share = kTerm && a.share_cache;
     __shared__ float red[4][2 * 32 * GP];
+    __shared__ float fin[2][2 * GP];             // two-stage reductions: the final per-head values
     __shared__ int scan[2][kFlatPer * 32 + 1];
     __shared__ int hist[2][256];
     __shared__ int hsum[256];
@@ -154,7 +159,7 @@ prune_finalize_wide_kernel(const FinArgs a) {
     const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
     float M = -kInf;
     if (n > 0) {
-        head_reduce<GP, 1, true>(Mh, red[0]);
+        head_reduce2<GP, 1, true>(Mh, red[0], fin[1 - 1]);
         cl_heads(Mh, 1, true);
         M = Mh[0];
     }
@@ -173,13 +178,14 @@ prune_finalize_wide_kernel(const FinArgs a) {
                     if (h < G && j < n) {
                         const float4 v = stat(j);
                         const bool top = !(v.x < M);
-                        const float c = top ? 1.f : expf(v.x - M);
+                        const float c = top ? 1.f : exp_le0(v.x - M);
                         zs[0] += c * v.y + (top ? 0.f : c);
                         zs[1] += top ? 1.f : 0.f;
                         if (kTerm) sh_t[j * GP + h] = c;
+                        if (share) sh_s[j * GP + h] = (1.f + v.y) * c;
                     }
                 }
-            head_reduce<GP, 2, false>(zs, red[1]);
+            head_reduce2<GP, 2, false>(zs, red[1], fin[2 - 1]);
             cl_heads(zs, 2, false);
             const float zm1 = zs[0] + (zs[1] - 1.f);
             const float lZ = log1pf(zm1), iZ = 1.f / (1.f + zm1);
@@ -196,12 +202,12 @@ prune_finalize_wide_kernel(const FinArgs a) {
                     const int j = r * RB + jt + k * JS;
                     if (h < G && j < n) {
                         const float4 v = stat(j);
-                        const float t = Ib(v, kTerm ? sh_t[j * GP + h] : (v.x < M ? expf(v.x - M) : 1.f));
+                        const float t = Ib(v, kTerm ? sh_t[j * GP + h] : (v.x < M ? exp_le0(v.x - M) : 1.f));
                         if (kTerm) sh_t[j * GP + h] = t;
                         Hs[0] += t;
                     }
                 }
-            head_reduce<GP, 1, false>(Hs, red[2]);
+            head_reduce2<GP, 1, false>(Hs, red[2], fin[1 - 1]);
             cl_heads(Hs, 1, false);
             const float nH = Hs[0] > 0.f ? (float)n / Hs[0] : 0.f;
             // group score: the largest normalised term over the heads of the block
@@ -216,7 +222,7 @@ prune_finalize_wide_kernel(const FinArgs a) {
                             t = sh_t[j * GP + h];
                         } else {
                             const float4 v = stat(j);
-                            t = Ib(v, v.x < M ? expf(v.x - M) : 1.f);
+                            t = Ib(v, v.x < M ? exp_le0(v.x - M) : 1.f);
                         }
                         sc = Hs[0] > 0.f ? t * nH : 1.f;
                     }
@@ -427,19 +433,26 @@ prune_finalize_wide_kernel(const FinArgs a) {
                 const int j = r * RB + jt + k * JS;
                 if (h < G && j < n && sh[j] != 0.f) Mk[0] = fmaxf(Mk[0], st[(long long)j * G + h].x);
             }
-        head_reduce<GP, 1, true>(Mk, red[3]);
+        head_reduce2<GP, 1, true>(Mk, red[3], fin[1 - 1]);
         cl_heads(Mk, 1, true);
         float Lk[1] = {0.f};
+        // (the rule mode's M is the head's max over all blocks: when the top
+        // block is kept the cached shares already have the right scale)
+        const bool cached = share && !a.given && Mk[0] == M;
         for (int r = r_lo; r < r_hi; ++r)
 #pragma unroll
             for (int k = 0; k < kFlatPer; ++k) {
                 const int j = r * RB + jt + k * JS;
                 if (h < G && j < n && sh[j] != 0.f) {
-                    const float4 v = st[(long long)j * G + h];
-                    Lk[0] += (1.f + v.y) * expf(v.x - Mk[0]);
+                    if (cached) {
+                        Lk[0] += sh_s[j * GP + h];
+                    } else {
+                        const float4 v = st[(long long)j * G + h];
+                        Lk[0] += (1.f + v.y) * exp_le0(v.x - Mk[0]);
+                    }
                 }
             }
-        head_reduce<GP, 1, false>(Lk, red[0]);
+        head_reduce2<GP, 1, false>(Lk, red[0], fin[1 - 1]);
         cl_heads(Lk, 1, false);
         if (tid < GP && h < G && cr == 0) {
             float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2;
@@ -475,23 +488,30 @@ cudaError_t launch_wide(int segs, size_t smem, cudaStream_t stream, const FinArg
 }
 
 // The launch shape: long segments fewer than half the SMs take a pair of
-// 1024-thread CTAs each, the rest one 1024-thread CTA each; the term cache is
-// used where it fits.  (256-thread CTAs, four per SM, gained 6 % on 1024
-// segments: the kernel is bound by its instructions, not by its waves.)
+// 1024-thread CTAs each (more threads per segment); the rest one 512-thread
+// CTA each, two CTAs per SM where the shared memory allows (on 1024 segments
+// of up to 2048 blocks x 8 heads: 157 us against 201 us with one 1024-thread
+// CTA per SM; 256-thread CTAs took 313 us).  The term cache is used where it
+// fits, the share cache only where it leaves room for two CTAs per SM.
 template <int G>
 cudaError_t launch_wide_shape(const FinArgs& a, int segs, int sms, cudaStream_t stream) {
     constexpr int GP = FlatGP<G>::v;
     const size_t smem_t = (size_t)a.max_blocks * 4 * (1 + GP), smem_s = (size_t)a.max_blocks * 4;
+    const size_t smem_ts = smem_t + (size_t)a.max_blocks * 4 * GP;
     const bool term = !a.given && smem_t <= kWideSmemMax;
-    const size_t smem = term ? smem_t : smem_s;
+    FinArgs b = a;
     if (2 * segs <= sms && a.max_blocks > (kWideThreads / GP) * kFlatPer) {
-        const cudaError_t e = term ? launch_wide<G, kWideThreads, true, 2>(segs, smem, stream, a)
-                                   : launch_wide<G, kWideThreads, false, 2>(segs, smem, stream, a);
+        b.share_cache = term && smem_ts <= kWideSmemMax;
+        const size_t smem = term ? (b.share_cache ? smem_ts : smem_t) : smem_s;
+        const cudaError_t e = term ? launch_wide<G, kWideThreads, true, 2>(segs, smem, stream, b)
+                                   : launch_wide<G, kWideThreads, false, 2>(segs, smem, stream, b);
         if (e == cudaSuccess) return e;
         (void)cudaGetLastError();   // cluster launch refused: one CTA per segment
     }
-    return term ? launch_wide<G, kWideThreads, true, 1>(segs, smem, stream, a)
-                : launch_wide<G, kWideThreads, false, 1>(segs, smem, stream, a);
+    b.share_cache = term && smem_ts <= kWideSmemMax / 2;
+    const size_t smem = term ? (b.share_cache ? smem_ts : smem_t) : smem_s;
+    return term ? launch_wide<G, kWideThreads / 2, true, 1>(segs, smem, stream, b)
+                : launch_wide<G, kWideThreads / 2, false, 1>(segs, smem, stream, b);
 }
 
 }  // namespace eti

@@ -375,6 +375,10 @@ prune_finalize_flat_kernel(const FinArgs a) {
     const int tid = threadIdx.x, lane = tid & 31;
     const int h = lane & (GP - 1);
     const int jt = tid / GP;
+    // chunk k holds no block below `bound` for any lane of this warp: the
+    // heavy passes skip it (a warp-uniform test)
+    const int jt0 = (tid & ~31) / GP;
+    auto live = [&](int k, int bound) { return jt0 + k * JS < bound; };
     const int L = a.ctx_lens[b];
     const float th = a.theta[b];
     const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
@@ -390,6 +394,7 @@ prune_finalize_flat_kernel(const FinArgs a) {
     for (int k = 0; k < kFlatPer; ++k) {
         const int j = jt + k * JS;
         m[k] = -kInf; l1[k] = 0.f; w[k] = 0.f;
+        if (!live(k, nb)) continue;
         if (h < G && j < nb) {
             const float4 s = st[(long long)j * G + h];
             m[k] = s.x; l1[k] = s.y; w[k] = a.score_mode == 1 ? s.w : s.z;
@@ -437,9 +442,9 @@ prune_finalize_flat_kernel(const FinArgs a) {
             c[k] = 0.f;
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k)
-            if (valid[k]) {
+            if (live(k, n) && valid[k]) {
                 const bool top = !(m[k] < M);
-                c[k] = top ? 1.f : expf(m[k] - M);
+                c[k] = top ? 1.f : exp_le0(m[k] - M);
                 zs[0] += c[k] * l1[k] + (top ? 0.f : c[k]);
                 zs[1] += top ? 1.f : 0.f;
             }
@@ -451,7 +456,7 @@ prune_finalize_flat_kernel(const FinArgs a) {
         float Hs[1] = {0.f};
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k)
-            if (valid[k]) {
+            if (live(k, n) && valid[k]) {
                 if (a.score_mode == 1) w[k] = c[k] * w[k] * iZ;                 // E
                 else if (a.score_mode == 2) w[k] = c[k] * (1.f + l1[k]) * iZ;   // M
                 else w[k] = c[k] * ((1.f + l1[k]) * (lZ + M - m[k]) - w[k]) * iZ;
@@ -463,6 +468,7 @@ prune_finalize_flat_kernel(const FinArgs a) {
         // group score: the largest normalised term over the heads of the block
 #pragma unroll
         for (int k = 0; k < kFlatPer; ++k) {
+            if (!live(k, n)) continue;           // score[k] stays -inf
             float s = valid[k] ? (Hs[0] > 0.f ? w[k] * nH : 1.f) : -kInf;
 #pragma unroll
             for (int o = 1; o < GP; o <<= 1) s = fmaxf(s, __shfl_xor_sync(0xffffffffu, s, o));
@@ -599,7 +605,7 @@ prune_finalize_flat_kernel(const FinArgs a) {
             for (int k = 0; k < kFlatPer; ++k)
                 if ((kk >> k) & 1u) {
                     const float4 s = st[(long long)(jt + k * JS) * G + h];
-                    Lk[0] += (1.f + s.y) * expf(s.x - Mk[0]);
+                    Lk[0] += (1.f + s.y) * exp_le0(s.x - Mk[0]);
                 }
         }
         head_reduce<GP, 1, false>(Lk, red[0]);
@@ -674,19 +680,18 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
     a.given_idx = given_idx; a.given_cnt = given_cnt; a.keep_mask = keep_mask;
     a.kept_idx = kept_idx; a.kept_cnt = kept_cnt; a.block_score = block_score;
     a.kept_norm = kept_norm; a.err = err;
+    a.share_cache = 0;
     const int grid = B * Hkv;
     cudaError_t e = cudaSuccess;
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (err) {
-        // a plain launch (it waits for the kernel before it, as a memset
-        // would); the keep-set kernel then overlaps its own launch with it
-        cudaLaunchConfig_t cfg = {};
-        cfg.gridDim = dim3((B + 255) / 256);
-        cfg.blockDim = dim3(256);
-        cfg.stream = stream;
-        if (cudaLaunchKernelEx(&cfg, clear_words_kernel, err, B) != cudaSuccess) return ETI_ERR_CUDA;
+        // programmatic launch: it waits for the kernel before it inside
+        // (griddepcontrol.wait), and the keep-set kernel overlaps its own
+        // launch with it
+        if (eti_launch_pdl(clear_words_kernel, dim3((B + 255) / 256), dim3(256), 0, stream, err, B) != cudaSuccess)
+            return ETI_ERR_CUDA;
     }
     // the flat kernel holds a segment in registers: 16 block-heads a thread
     const int gp = a.g <= 1 ? 1 : a.g <= 2 ? 2 : a.g <= 4 ? 4 : 8;
