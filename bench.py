@@ -547,6 +547,8 @@ def run_gpu(args):
         dist.init_process_group("nccl", device_id=device)
     eti.load()
     w = shard_workload(workloads.WORKLOADS[args.workload], rank)
+    if args.batch:
+        w = w.scaled(B=args.batch)   # a reduced case of the same shape (for profiling)
     prm = eti.ctrl_params()
     stream = torch.cuda.current_stream()
     r = StepRunner(eti, w, device, prm, stream)
@@ -1012,6 +1014,9 @@ def main(argv=None):
                     help="skip the long-context keep-fraction sweep (decode time against kept blocks)")
     ap.add_argument("--no-estimators", action="store_true",
                     help="skip the top-k entropy estimator line")
+    ap.add_argument("--batch", type=int, default=None,
+                    help="run the workload with this many sequences instead (a reduced case of the "
+                         "same shape, e.g. for an ncu capture that must stay small)")
     ap.add_argument("--no-workloads", action="store_true",
                     help="skip the other four workloads (tiny, long_ctx, mixed_batch, llama3_70b)")
     ap.add_argument("--clock-seconds", type=float, default=2.0,

@@ -56,7 +56,7 @@ def test_source_digest_ignores_comments_not_code(tmp_path):
 def test_ncu_traffic_record_matches_the_committed_kernels():
     rec = json.load(open(os.path.join(bench.ROOT, "profiles", "ncu_traffic.json")))
     kernels = [k for k in rec if not k.startswith("_")]
-    assert {"score_blocks", "paged_decode", "entropy_sample_partial"} <= set(kernels)
+    assert {"score_blocks", "paged_decode", "entropy_sample", "prune_finalize"} <= set(kernels)
     for k in kernels:
         for p in rec[k]["sources"]:
             assert os.path.exists(os.path.join(bench.ROOT, p)), p
