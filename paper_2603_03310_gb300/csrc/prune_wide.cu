@@ -464,6 +464,309 @@ prune_finalize_wide_kernel(const FinArgs a) {
     if (kCl > 1) cluster_sync();
 }
 
+// ---------------------------------------------------------------------------
+// prune_finalize_seg_kernel: the rule mode for a segment whose per-block-head
+// terms fit in shared memory (max_blocks * (GP + 1) floats), one CTA of NT
+// threads per (sequence, kv head) segment, two CTAs per SM.
+//  - three passes over the block stats in the head-lane layout (thread t:
+//    head t % GP of blocks t / GP, t / GP + NT / GP, ... up to the segment's
+//    end, not to max_blocks): the per-head max, then e^{m_b - M} and Z, then
+//    the terms I_b and H, the terms kept in shared memory; the first pass
+//    reads the stats from HBM, the next two from L2.  (Folding the terms into
+//    the second pass as pairs (A_b, B_b) with I_b = (A_b log Z + B_b) / Z
+//    needs twice the shared memory, one CTA per SM, and was slower: 168
+//    against 117 us on the 70B-shaped step);
+//  - per block, over shared memory (thread t: the contiguous run of blocks
+//    [t q, (t + 1) q)): the group score max_h n I_b^(h) / H^(h), the budget
+//    (argmax, or a radix select with ties to the lower index), the keep
+//    flag, and the compaction from an exclusive scan of the runs' counts;
+//  - one pass over the kept blocks' stats for the kept-token normaliser
+//    (an online max and sum per head).
+template <int G, int NT>
+__global__ void __launch_bounds__(NT, 2)
+prune_finalize_seg_kernel(const FinArgs a) {
+    constexpr int GP = FlatGP<G>::v;
+    constexpr int JS = NT / GP;                  // block stride of a head lane
+    constexpr int NW = NT / 32;
+    pdl_trigger();
+    pdl_wait();
+    extern __shared__ __align__(16) float sg_smem[];
+    float* term = sg_smem;                                  // [max_blocks * GP]
+    float* sc = sg_smem + (size_t)a.max_blocks * GP;        // [max_blocks]: scores, then keep flags
+    __shared__ float red[4][2 * 32 * GP];
+    __shared__ float fin[2][2 * GP];
+    __shared__ float nHs[GP];                    // n / H per head (< 0: H = 0, every block scores 1)
+    __shared__ int wsum[NW];
+    __shared__ int hist[256];
+    __shared__ int sel_digit, sel_rem;
+    __shared__ float arg_v[NW];
+    __shared__ int arg_j[NW];
+    __shared__ float nm[NW][GP], nl[NW][GP];     // kept-norm partials per warp and head
+    const int seg = blockIdx.x;
+    const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int h = lane & (GP - 1);
+    const int jt = tid / GP;
+    const int L = a.ctx_lens[b];
+    const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
+    const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
+    const long long segbase = (long long)seg * a.max_blocks;
+    const float4* st = a.stats + segbase * G;
+
+    // exclusive prefix of one int per thread over the CTA (in thread order);
+    // returns it and the total in *tot
+    auto scan_excl = [&](int v, int* tot) {
+        int x = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(0xffffffffu, x, o);
+            if (lane >= o) x += y;
+        }
+        if (lane == 31) wsum[wid] = x;
+        __syncthreads();
+        int before = 0, all = 0;
+        for (int u = 0; u < NW; ++u) {
+            const int y = wsum[u];
+            before += u < wid ? y : 0;
+            all += y;
+        }
+        __syncthreads();
+        *tot = all;
+        return before + x - v;
+    };
+
+    // pass 1: page ids, stale stats, the per-head max
+    const int bad = any_bad_page(a.block_table + (long long)b * a.max_blocks, tid, NT, nb, a.num_pages);
+    int stale = 0;
+    float Mh[1] = {-kInf};
+    if (h < G)
+        for (int j = jt; j < nb; j += JS) {
+            const float x = st[(long long)j * G + h].x;
+            stale |= (x != x);                   // NaN max: the scoring pass gave up on this block
+            Mh[0] = fmaxf(Mh[0], x);
+        }
+    const bool bad_page = __syncthreads_or(bad) != 0;
+    const bool timed_out = __syncthreads_or(stale) != 0 && !bad_page;
+    bool drain = false;
+    if (timed_out) {
+        // rare: a block marked l - 1 = +inf had a copy in flight when the drain gave up
+        int d = 0;
+        if (h < G)
+            for (int j = jt; j < nb; j += JS) {
+                const float4 v = st[(long long)j * G + h];
+                d |= (v.x != v.x) && v.y == kInf;
+            }
+        drain = __syncthreads_or(d) != 0;
+    }
+    if (a.err && tid == 0) {
+        // err was cleared before this kernel; every kv head ORs in its bits
+        const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page ? ETI_ERRF_BAD_PAGE : 0u) |
+                           (timed_out ? ETI_ERRF_TIMEOUT : 0u) | (drain ? ETI_ERRF_DRAIN : 0u);
+        if (e) atomicOr(a.err + b, e);
+    }
+    const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
+    if (n > 0) {
+        head_reduce2<GP, 1, true>(Mh, red[0], fin[0]);
+        const float M = Mh[0];
+        // pass 2: Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
+        // c_b = e^{m_b - M} (the blocks at the max are counted, not summed)
+        float zs[2] = {0.f, 0.f};
+        if (h < G)
+            for (int j = jt; j < n; j += JS) {
+                const float2 v = *reinterpret_cast<const float2*>(st + (long long)j * G + h);
+                const bool top = !(v.x < M);
+                const float c = top ? 1.f : exp_le0(v.x - M);
+                zs[0] += c * v.y + (top ? 0.f : c);
+                zs[1] += top ? 1.f : 0.f;
+                term[j * GP + h] = c;
+            }
+        head_reduce2<GP, 2, false>(zs, red[1], fin[1]);
+        const float zm1 = zs[0] + (zs[1] - 1.f);
+        const float lZ = log1pf(zm1), iZ = 1.f / (1.f + zm1);
+        // pass 3: I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
+        float Hs[1] = {0.f};
+        if (h < G)
+            for (int j = jt; j < n; j += JS) {
+                const float4 v = st[(long long)j * G + h];
+                const float c = term[j * GP + h];
+                float t;
+                if (a.score_mode == 1) t = c * v.w * iZ;                       // E
+                else if (a.score_mode == 2) t = c * (1.f + v.y) * iZ;          // M
+                else t = c * ((1.f + v.y) * (lZ + M - v.x) - v.z) * iZ;        // A
+                term[j * GP + h] = t;
+                Hs[0] += t;
+            }
+        head_reduce2<GP, 1, false>(Hs, red[2], fin[0]);
+        if (tid < GP) nHs[tid] = Hs[0] > 0.f ? (float)n / Hs[0] : -1.f;
+        __syncthreads();
+    }
+
+    // per block from here: thread t takes blocks [j0, j1)
+    const int q = (n + NT - 1) / NT;
+    const int j0 = min(n, tid * q), j1 = min(n, j0 + q);
+    float bs = -kInf;                            // this run's best score and its block
+    int bj = 0x7fffffff;
+    for (int j = j0; j < j1; ++j) {
+        float s = -kInf;
+#pragma unroll
+        for (int hh = 0; hh < G; ++hh) {
+            const float f = nHs[hh];
+            s = fmaxf(s, f < 0.f ? 1.f : term[j * GP + hh] * f);
+        }
+        sc[j] = s;
+        if (a.block_score) a.block_score[segbase + j] = s;
+        if (s > bs || bj == 0x7fffffff) { bs = s; bj = j; }
+    }
+    if (a.block_score)
+        for (int j = n + tid; j < a.max_blocks; j += NT) a.block_score[segbase + j] = 0.f;
+    __syncthreads();
+
+    // B_min budget: the first kb blocks by (score desc, index asc)
+    const float th = a.theta[b];
+    const int kb = min(max(a.B_min, 0), n);
+    const bool sel = kb > 1 && kb < n;
+    int arg = -1, need = 0;
+    uint32_t kth = 0u;
+    if (kb == 1 && n > 1) {
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float ov = __shfl_xor_sync(0xffffffffu, bs, o);
+            const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+            if (oj != 0x7fffffff && (bj == 0x7fffffff || ov > bs || (ov == bs && oj < bj))) { bs = ov; bj = oj; }
+        }
+        if (lane == 0) { arg_v[wid] = bs; arg_j[wid] = bj; }
+        __syncthreads();
+        for (int u = 0; u < NW; ++u)
+            if (arg_j[u] != 0x7fffffff && (bj == 0x7fffffff || arg_v[u] > bs || (arg_v[u] == bs && arg_j[u] < bj))) {
+                bs = arg_v[u];
+                bj = arg_j[u];
+            }
+        arg = bj;
+    } else if (sel) {
+        uint32_t prefix = 0, mask = 0;
+        need = kb;
+        for (int digit = 3; digit >= 0; --digit) {
+            const int shf = digit * 8;
+            for (int i = tid; i < 256; i += NT) hist[i] = 0;
+            __syncthreads();
+            for (int jb = 0; jb < n; jb += NT) {      // the same trip count for every lane
+                const int j = jb + tid;
+                const uint32_t key = j < n ? order_key(sc[j]) : 0u;
+                warp_hist_add(hist, (key >> shf) & 255, j < n && (key & mask) == prefix);
+            }
+            __syncthreads();
+            // bucket where the count from the top reaches `need`
+            if (tid < 32) {
+                int cnt8[8], s8 = 0;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) { cnt8[e] = hist[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
+                int incl = s8;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (tid >= o) incl += y;
+                }
+                int above = incl - s8;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    if (above < need && need <= above + cnt8[e]) {
+                        sel_digit = 255 - (tid * 8 + e);
+                        sel_rem = need - above;
+                    }
+                    above += cnt8[e];
+                }
+            }
+            __syncthreads();
+            prefix |= (uint32_t)sel_digit << shf;
+            mask |= 255u << shf;
+            need = sel_rem;
+            __syncthreads();
+        }
+        kth = prefix;
+    }
+    // keep flags (ties at the k-th key to the lower block index: ranked in
+    // thread order, which is block order)
+    int neq = 0;
+    if (sel)
+        for (int j = j0; j < j1; ++j) neq += order_key(sc[j]) == kth;
+    int eq_tot;
+    int eq_rank = sel ? scan_excl(neq, &eq_tot) : 0;
+    int nkeep = 0;
+    uint32_t kbits = 0;                          // this run's keep flags (q <= 32 blocks a thread)
+    for (int j = j0; j < j1; ++j) {
+        const float s = sc[j];
+        const uint32_t key = order_key(s);
+        bool keep = s >= th || kb >= n || j == arg || (sel && key > kth);
+        if (sel && key == kth) keep |= eq_rank++ < need;
+        kbits |= keep ? 1u << (j - j0) : 0u;
+        nkeep += keep;
+    }
+    int total;
+    int pos = scan_excl(nkeep, &total);          // (its barriers order the score reads above)
+    for (int j = j0; j < j1; ++j) {
+        const bool keep = (kbits >> (j - j0)) & 1u;
+        if (keep) a.kept_idx[segbase + pos++] = j;
+        if (a.keep_mask) a.keep_mask[segbase + j] = keep ? 1 : 0;
+        sc[j] = keep ? 1.f : 0.f;
+    }
+    for (int i = total + tid; i < a.max_blocks; i += NT) a.kept_idx[segbase + i] = -1;
+    if (a.keep_mask)
+        for (int j = n + tid; j < a.max_blocks; j += NT) a.keep_mask[segbase + j] = 0;
+    if (tid == 0) a.kept_cnt[seg] = total;
+
+    // softmax normaliser over the kept tokens of each query head: an online
+    // (max, sum of (1 + l1) e^{m - max}) over the kept blocks, merged over
+    // the lanes of a head and then over the warps in warp order
+    if (a.kept_norm) {
+        __syncthreads();                         // the keep flags in sc
+        float mk = -kInf, lk = 0.f;
+        if (h < G)
+            for (int j = jt; j < n; j += JS) {
+                if (sc[j] == 0.f) continue;
+                const float2 v = *reinterpret_cast<const float2*>(st + (long long)j * G + h);
+                if (v.x > mk) {
+                    lk = (mk == -kInf ? 0.f : lk * exp_le0(mk - v.x)) + (1.f + v.y);
+                    mk = v.x;
+                } else {
+                    lk += (1.f + v.y) * exp_le0(v.x - mk);
+                }
+            }
+        auto merge = [](float& m1, float& l1, float m2, float l2) {
+            if (m2 == -kInf) return;
+            if (m1 == -kInf) { m1 = m2; l1 = l2; return; }
+            const float mm = fmaxf(m1, m2);
+            l1 = l1 * exp_le0(m1 - mm) + l2 * exp_le0(m2 - mm);
+            m1 = mm;
+        };
+#pragma unroll
+        for (int o = 16; o >= GP; o >>= 1) {
+            const float om = __shfl_xor_sync(0xffffffffu, mk, o);
+            const float ol = __shfl_xor_sync(0xffffffffu, lk, o);
+            merge(mk, lk, om, ol);               // (the two sides agree: the sum commutes)
+        }
+        if (lane < GP) { nm[wid][lane] = mk; nl[wid][lane] = lk; }
+        __syncthreads();
+        if (tid < G) {
+            float m1 = -kInf, l1 = 0.f;
+            for (int u = 0; u < NW; ++u) merge(m1, l1, nm[u][tid], nl[u][tid]);
+            float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + tid) * 2;
+            kn[0] = m1;
+            kn[1] = l1;
+        }
+    }
+}
+
+// Launch of the segment kernel (programmatic dependent launch).
+template <int G>
+cudaError_t launch_seg(int segs, cudaStream_t stream, const FinArgs& a) {
+    constexpr int GP = FlatGP<G>::v;
+    constexpr int NT = 512;
+    auto k = prune_finalize_seg_kernel<G, NT>;
+    const size_t smem = (size_t)a.max_blocks * (GP + 1) * 4;
+    if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    return eti_launch_pdl(k, dim3(segs), dim3(NT), smem, stream, a);
+}
+
 // Launch of the wide kernel for `segs` segments, kCl CTAs of NT threads per
 // segment (a cluster), with programmatic dependent launch.
 template <int G, int NT, bool kTerm, int kCl>
@@ -508,6 +811,11 @@ cudaError_t launch_wide_shape(const FinArgs& a, int segs, int sms, cudaStream_t 
         if (e == cudaSuccess) return e;
         (void)cudaGetLastError();   // cluster launch refused: one CTA per segment
     }
+    // the rule mode with the terms of a segment in shared memory (and at most
+    // 32 blocks per thread in the per-block passes): the segment kernel
+    if (!a.given && a.theta && (size_t)a.max_blocks * (GP + 1) * 4 <= kWideSmemMax / 2 &&
+        a.max_blocks <= 512 * 32)
+        return launch_seg<G>(segs, stream, a);
     b.share_cache = term && smem_ts <= kWideSmemMax / 2;
     const size_t smem = term ? (b.share_cache ? smem_ts : smem_t) : smem_s;
     return term ? launch_wide<G, kWideThreads / 2, true, 1>(segs, smem, stream, b)
