@@ -601,25 +601,38 @@ prune_finalize_seg_kernel(const FinArgs a) {
         __syncthreads();
     }
 
-    // per block from here: thread t takes blocks [j0, j1)
-    const int q = (n + NT - 1) / NT;
-    const int j0 = min(n, tid * q), j1 = min(n, j0 + q);
-    float bs = -kInf;                            // this run's best score and its block
+    // group scores: thread t takes blocks t, t + NT, ... (a warp reads
+    // consecutive blocks' terms with 16-byte loads: few bank conflicts)
+    float nh[GP];
+#pragma unroll
+    for (int hh = 0; hh < GP; ++hh) nh[hh] = hh < G ? nHs[hh] : -kInf;
+    float bs = -kInf;                            // this thread's best score and its block
     int bj = 0x7fffffff;
-    for (int j = j0; j < j1; ++j) {
+    for (int j = tid; j < n; j += NT) {
+        float t[GP];
+        if (GP >= 4) {
+#pragma unroll
+            for (int c = 0; c < GP / 4; ++c) {
+                const float4 v = reinterpret_cast<const float4*>(term + j * GP)[c];
+                t[4 * c] = v.x; t[4 * c + 1] = v.y; t[4 * c + 2] = v.z; t[4 * c + 3] = v.w;
+            }
+        } else {
+#pragma unroll
+            for (int hh = 0; hh < GP; ++hh) t[hh] = term[j * GP + hh];
+        }
         float s = -kInf;
 #pragma unroll
-        for (int hh = 0; hh < G; ++hh) {
-            const float f = nHs[hh];
-            s = fmaxf(s, f < 0.f ? 1.f : term[j * GP + hh] * f);
-        }
+        for (int hh = 0; hh < G; ++hh) s = fmaxf(s, nh[hh] < 0.f ? 1.f : t[hh] * nh[hh]);
         sc[j] = s;
         if (a.block_score) a.block_score[segbase + j] = s;
-        if (s > bs || bj == 0x7fffffff) { bs = s; bj = j; }
+        if (s > bs || bj == 0x7fffffff) { bs = s; bj = j; }   // ascending j: the first of equal scores stays
     }
     if (a.block_score)
         for (int j = n + tid; j < a.max_blocks; j += NT) a.block_score[segbase + j] = 0.f;
     __syncthreads();
+    // per block from here: thread t takes the run of blocks [j0, j1)
+    const int q = (n + NT - 1) / NT;
+    const int j0 = min(n, tid * q), j1 = min(n, j0 + q);
 
     // B_min budget: the first kb blocks by (score desc, index asc)
     const float th = a.theta[b];
