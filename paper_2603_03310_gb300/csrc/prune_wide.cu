@@ -769,15 +769,23 @@ prune_finalize_seg_kernel(const FinArgs a) {
     }
 }
 
-// Launch of the segment kernel (programmatic dependent launch).
-template <int G>
-cudaError_t launch_seg(int segs, cudaStream_t stream, const FinArgs& a) {
+// Launch of the segment kernel (programmatic dependent launch): 128, 256 or
+// 512 threads, about 16 block-heads of the longest segment a thread.
+template <int G, int NT>
+cudaError_t launch_seg_nt(int segs, cudaStream_t stream, const FinArgs& a) {
     constexpr int GP = FlatGP<G>::v;
-    constexpr int NT = 512;
     auto k = prune_finalize_seg_kernel<G, NT>;
     const size_t smem = (size_t)a.max_blocks * (GP + 1) * 4;
     if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     return eti_launch_pdl(k, dim3(segs), dim3(NT), smem, stream, a);
+}
+template <int G>
+cudaError_t launch_seg(int segs, cudaStream_t stream, const FinArgs& a) {
+    constexpr int GP = FlatGP<G>::v;
+    const long long slots = (long long)a.max_blocks * GP;
+    if (slots <= 128 * 16) return launch_seg_nt<G, 128>(segs, stream, a);
+    if (slots <= 256 * 16) return launch_seg_nt<G, 256>(segs, stream, a);
+    return launch_seg_nt<G, 512>(segs, stream, a);
 }
 
 // Launch of the wide kernel for `segs` segments, kCl CTAs of NT threads per

@@ -693,10 +693,17 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
         if (eti_launch_pdl(clear_words_kernel, dim3((B + 255) / 256), dim3(256), 0, stream, err, B) != cudaSuccess)
             return ETI_ERR_CUDA;
     }
-    // the flat kernel holds a segment in registers: 16 block-heads a thread
+    // the flat kernel holds a segment in registers: 16 block-heads a thread.
+    // Its work follows max_blocks whatever the segment's length, so it is
+    // taken when the segments run in one wave (at most four a SM, where it is
+    // latency-bound); more segments go to the segment kernel, whose work
+    // follows each segment's length (on 2048 segments of 4 to 512 blocks x 4
+    // heads: 23 against 41 us; on 512 segments of 64 to 512 blocks: 18.7
+    // against 16.6 us)
     const int gp = a.g <= 1 ? 1 : a.g <= 2 ? 2 : a.g <= 4 ? 4 : 8;
     const long long flat_need = ((long long)max_blocks * gp + kFlatPer - 1) / kFlatPer;
-    const int flat_nt = !given && theta && flat_need <= 512
+    const bool seg_fits = (size_t)max_blocks * (gp + 1) * 4 <= kWideSmemMax / 2;
+    const int flat_nt = !given && theta && flat_need <= 512 && (grid <= 4 * sms || !seg_fits)
                             ? (flat_need <= 128 ? 128 : flat_need <= 256 ? 256 : 512) : 0;
 #define ETI_FIN_FLAT(GG, NT)                                                                \
     if (flat_nt == NT) {                                                                    \
