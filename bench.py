@@ -410,10 +410,17 @@ class StepRunner:
         self.L = self.kv["ctx_lens"].cpu().numpy()
         self.total_blocks = int((-(-self.L // w.P)).sum()) * w.Hkv
 
-    def run(self, ev=None, offset=0):
-        """One step; with `ev` (5 events) an event between the calls."""
+    def run(self, ev=None, offset=0, side=None):
+        """One step; with `ev` (5 events) an event between the calls.  With a
+        `side` stream the sampling call (which reads only the logits and the
+        per-sequence state) runs there, beside the attention half, and the
+        launching stream waits for it before the step ends."""
         eti, kv, st, w = self.eti, self.kv, self.step, self.w
         s = self.stream
+        if side is not None:
+            side.wait_stream(s)                  # fork
+            st.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], self.lg["tau"],
+                      self.lg["H_target"], params=self.prm, seed=w.seed, offset=offset, stream=side)
         if ev is not None:
             ev[0].record(s)
         eti.eti_score_blocks(kv["q"], kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
@@ -431,8 +438,11 @@ class StepRunner:
                              num_pages=kv["num_pages"])
         if ev is not None:
             ev[3].record(s)
-        st.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], self.lg["tau"], self.lg["H_target"],
-                  params=self.prm, seed=w.seed, offset=offset)
+        if side is None:
+            st.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], self.lg["tau"], self.lg["H_target"],
+                      params=self.prm, seed=w.seed, offset=offset)
+        else:
+            s.wait_stream(side)                  # join
         if ev is not None:
             ev[4].record(s)
 
@@ -486,26 +496,33 @@ def dense_decode_ms(r, flush_l2, reps=20):
     return ms
 
 
-def workload_summary(r, flush_l2, peak, steps, warmup, offset0=0):
+def timed_steps(r, flush_l2, steps, offset0, side=None):
+    """Mean CUDA-event time (ms) of `steps` steps, L2 flushed before each."""
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+    for i in range(steps):
+        flush_l2()
+        evs[i][0].record(r.stream)
+        r.run(offset=offset0 + i, side=side)
+        evs[i][1].record(r.stream)
+    torch.cuda.synchronize()
+    return statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+
+
+def workload_summary(r, flush_l2, peak, steps, warmup, side, offset0=0):
     """Step time, throughput, kept fraction and per-kernel times / fractions of
     the HBM peak for one workload (same timing rules as the main line)."""
     w = r.w
     for i in range(warmup):
         flush_l2()
-        r.run(offset=offset0 + i)
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
-    for i in range(steps):
-        flush_l2()
-        evs[i][0].record(r.stream)
-        r.run(offset=offset0 + warmup + i)
-        evs[i][1].record(r.stream)
-    torch.cuda.synchronize()
-    ms = statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
+        r.run(offset=offset0 + i, side=side)
+    ms = timed_steps(r, flush_l2, steps, offset0 + warmup, side)
+    ms_seq = timed_steps(r, flush_l2, min(steps, 50), offset0 + warmup + steps)
     per = kernel_pass(r, flush_l2, min(steps, 50), offset0 + warmup + steps)
     kept = r.kept()
     ab = algorithmic_bytes(w, r.L, kept)
     gbs = {n: ab[n] / (per[n] / 1e3) / 1e9 for n in NAMES}
     out = {"workload": workload_desc(w), "steps": steps, "ms_per_step": round(ms, 5),
+           "ms_per_step_sequential": round(ms_seq, 5),
            "tokens_per_s": round(w.B / (ms / 1e3), 1),
            "kept_fraction": round(kept / max(1, r.total_blocks), 4),
            "kernels_ms": {n: round(v, 5) for n, v in per.items()},
@@ -551,6 +568,7 @@ def run_gpu(args):
         w = w.scaled(B=args.batch)   # a reduced case of the same shape (for profiling)
     prm = eti.ctrl_params()
     stream = torch.cuda.current_stream()
+    side = torch.cuda.Stream(device=device)      # the sampling call runs beside the attention half
     r = StepRunner(eti, w, device, prm, stream)
     L2 = torch.cuda.get_device_properties(device).L2_cache_size
     flush_w = torch.empty(max(2 * L2, 256 << 20), dtype=torch.uint8, device=device)
@@ -570,7 +588,7 @@ def run_gpu(args):
 
     for i in range(args.warmup):
         flush_l2()
-        r.run(offset=i)
+        r.run(offset=i, side=side)
     torch.cuda.synchronize()
     kept = r.kept()
     total_blocks = r.total_blocks
@@ -592,7 +610,7 @@ def run_gpu(args):
         for i in range(args.steps):
             flush_l2()
             evs[i][0].record(stream)
-            r.run(offset=off + i)
+            r.run(offset=off + i, side=side)
             evs[i][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
@@ -608,7 +626,7 @@ def run_gpu(args):
             while time.perf_counter() - t1 < args.clock_seconds:
                 for _ in range(50):
                     flush_l2()
-                    r.run(offset=off + ncp)
+                    r.run(offset=off + ncp, side=side)
                     ncp += 1
                 torch.cuda.synchronize()
             e1.record(stream)
@@ -625,6 +643,8 @@ def run_gpu(args):
     if cp is not None and clocks is not None:
         cp["sm_mhz_median"] = clocks["sm_mhz"]
     mean_ms = kernel_pass(r, flush_l2, min(args.steps, 300), off)
+    off += min(args.steps, 300)
+    seq_ms = timed_steps(r, flush_l2, min(args.steps, 300), off)   # the four calls on one stream
     off += min(args.steps, 300)
     # share of the attention the keep set retains (outside the timed region;
     # a diagnostic never fails the run)
@@ -706,7 +726,7 @@ def run_gpu(args):
             res = []
             for f in fracs:
                 ro = StepRunner(eti, ow, device, prm, stream, H_target_frac=f)
-                s = workload_summary(ro, flush_l2, peak, ksteps, 5)
+                s = workload_summary(ro, flush_l2, peak, ksteps, 5, side)
                 if f is not None:
                     s["H_target"] = f"{f} log V"
                 res.append(s)
@@ -719,7 +739,11 @@ def run_gpu(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms, 5),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16/fp32",
         "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
+        "ms_per_step_sequential": round(seq_ms, 5),
         "config": {"workload": main_desc,
+                   "streams": "the sampling call on a second stream beside the attention half "
+                              "(forked at the step's start, joined before its end event); "
+                              "ms_per_step_sequential: the four calls on one stream",
                    "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write, then 2x L2 read)",
                    "parallelism": f"replicas x{world} (independent batches)", "B_min": 1,
                    "theta": "theta_next of the step's own entropy (defaults)",
@@ -785,16 +809,15 @@ def run_e2e(eti, r, args, device):
     off_dev = torch.zeros(1, dtype=torch.int64, device=device)   # Philox offset, advanced by each call
 
     # The small inputs go up first; the logits (the bulk of the bytes) then go
-    # up on a copy stream while the attention half runs; the sampling call
-    # waits for them.  The attention
-    # output comes down on the copy stream while the sampling call runs.  The
-    # whole step (copies and calls, both streams) is captured once in a CUDA
+    # up on a second stream, where the sampling call follows them and its
+    # results come down, all while the attention half runs on the first; the
+    # attention output comes down on the second stream once both are done.
+    # The whole step (copies and calls, both streams) is captured once in a CUDA
     # graph and replayed every step, as a serving loop would; the sampling
     # offset lives in device memory (the call advances it), so every replay
     # draws fresh numbers.  If the capture is refused the same body runs eagerly.
     main = torch.cuda.current_stream()
     copy = torch.cuda.Stream(device=device)
-    ev_logits = torch.cuda.Event()
     ev_out = torch.cuda.Event()
     stages = ("start", "logits_up_start", "logits_up_end", "small_up_end", "attention_end", "out_down_end",
               "sample_end", "results_down_end", "end")
@@ -810,8 +833,13 @@ def run_e2e(eti, r, args, device):
         with torch.cuda.stream(copy):
             rec("logits_up_start", copy)
             d_logits.copy_(h_logits, non_blocking=True)
-            ev_logits.record(copy)
             rec("logits_up_end", copy)
+            eti.eti_entropy_temp_sample(d_logits, T_in, H_prev, tau, H_tgt, tok, H_out, T_out, err,
+                                        step.ws_ets, params=prm, seed=w.seed, offset_dev=off_dev,
+                                        theta_next=th_next, tok_surprisal=surp, stream=copy)
+            rec("sample_end", copy)
+            h_res.copy_(d_io[qb + 4 * row:], non_blocking=True)
+            rec("results_down_end", copy)
         eti.eti_score_blocks(d_q, kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
                              r.stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
         eti.eti_prune_blocks(r.stats, kv["block_table"], kv["ctx_lens"], r.shape, th, r.B_min,
@@ -828,13 +856,6 @@ def run_e2e(eti, r, args, device):
             copy.wait_event(ev_out)
             h_out.copy_(step.out, non_blocking=True)
             rec("out_down_end", copy)
-        cur.wait_event(ev_logits)
-        eti.eti_entropy_temp_sample(d_logits, T_in, H_prev, tau, H_tgt, tok, H_out, T_out, err,
-                                    step.ws_ets, params=prm, seed=w.seed, offset_dev=off_dev,
-                                    theta_next=th_next, tok_surprisal=surp)
-        rec("sample_end", cur)
-        h_res.copy_(d_io[qb + 4 * row:], non_blocking=True)
-        rec("results_down_end", cur)
         cur.wait_stream(copy)                                  # join
         rec("end", cur)
 
@@ -855,15 +876,16 @@ def run_e2e(eti, r, args, device):
         "small_upload_ms": span("start", "small_up_end"),
         "attention_ms": span("small_up_end", "attention_end"),
         "out_download_ms": span("attention_end", "out_down_end"),
-        "logits_ready_after_attention_ms": span("attention_end", "logits_up_end"),
-        "sample_ms": span("attention_end", "sample_end"),
+        "sample_ms": span("logits_up_end", "sample_end"),
         "results_download_ms": span("sample_end", "results_down_end"),
+        "sampling_side_done_after_attention_ms": span("attention_end", "results_down_end"),
         "device_span_ms": span("start", "end"),
     }
     breakdown = {k: round(v, 4) for k, v in breakdown.items()}
-    breakdown["note"] = ("eager pass with events at the stage boundaries (median of 20); sample_ms "
-                         "includes any wait for the logits upload; logits_ready_after_attention_ms < 0 "
-                         "means the upload finished before the attention half")
+    breakdown["note"] = ("eager pass with events at the stage boundaries (median of 20); the logits "
+                         "upload, the sampling call and its results download run on a second stream "
+                         "beside the attention half; sampling_side_done_after_attention_ms < 0 means "
+                         "that side finished first; out_download_ms includes any wait for it")
     mode = "cuda graph replay (copies and calls of one step; sampling offset in device memory)"
     graph, gs = None, torch.cuda.Stream(device=device)
     try:
