@@ -17,7 +17,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libeti.so")
-SOURCES = ["api.cu", "entropy_sample.cu", "score_prune.cu", "prune_wide.cu", "paged_decode.cu",
+SOURCES = ["api.cu", "entropy_sample.cu", "score_prune.cu", "keep_tile.cu", "prune_wide.cu", "paged_decode.cu",
            "topk_entropy.cu", "schedule.cu"]
 HEADERS = ["common.cuh", "keep_set.cuh"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]

@@ -120,22 +120,22 @@ __device__ __forceinline__ void head_reduce2(float (&v)[N], float* red, float* f
 
 // Exclusive ranks in ascending block order of the flagged blocks (flags
 // agree across the GP lanes of a block); returns the number flagged.
-// scan holds kFlatPer * 32 + 1 ints.
-template <int GP>
-__device__ __forceinline__ int flat_ranks(const bool (&f)[kFlatPer], int (&pos)[kFlatPer], int* scan) {
+// scan holds KP * 32 + 1 ints.
+template <int GP, int KP = kFlatPer>
+__device__ __forceinline__ int flat_ranks(const bool (&f)[KP], int (&pos)[KP], int* scan) {
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, nw = blockDim.x >> 5;
     const bool lead = (lane & (GP - 1)) == 0;
     const uint32_t below = (1u << (lane & ~(GP - 1))) - 1u;   // lanes of earlier blocks
-    uint32_t bal[kFlatPer];
+    uint32_t bal[KP];
 #pragma unroll
-    for (int k = 0; k < kFlatPer; ++k) {
+    for (int k = 0; k < KP; ++k) {
         bal[k] = __ballot_sync(0xffffffffu, f[k] && lead);
         if (lane == 0) scan[k * nw + w] = __popc(bal[k]);
     }
     __syncthreads();
     if (w == 0) {
         // exclusive scan of the (chunk, warp) counts, chunk-major
-        const int E = kFlatPer * nw, per = (E + 31) >> 5;
+        const int E = KP * nw, per = (E + 31) >> 5;
         const int e0 = min(lane * per, E), e1 = min(e0 + per, E);
         int s = 0;
         for (int e = e0; e < e1; ++e) s += scan[e];
@@ -151,8 +151,8 @@ __device__ __forceinline__ int flat_ranks(const bool (&f)[kFlatPer], int (&pos)[
     }
     __syncthreads();
 #pragma unroll
-    for (int k = 0; k < kFlatPer; ++k) pos[k] = scan[k * nw + w] + __popc(bal[k] & below);
-    return scan[kFlatPer * nw];
+    for (int k = 0; k < KP; ++k) pos[k] = scan[k * nw + w] + __popc(bal[k] & below);
+    return scan[KP * nw];
 }
 
 }  // namespace eti

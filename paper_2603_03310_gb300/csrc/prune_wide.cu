@@ -1,13 +1,13 @@
-// prune_wide.cu -- the keep-set kernel for segments too long for the
-// register-resident flat layout, and for the given keep sets of a standalone
-// decode (Section 3.2).
+// prune_wide.cu -- the keep-set kernels for segments longer than the tile
+// kernel stages (more than 8192 block-heads), and for the given keep sets of
+// a standalone decode (Section 3.2).
 #include "keep_set.cuh"
 
 namespace eti {
 
 // ---------------------------------------------------------------------------
 // prune_finalize for segments of any size (and for the given keep sets), in
-// the flat kernel's layout: thread t owns query head h = t % GP of the blocks
+// a flat layout: thread t owns query head h = t % GP of the blocks
 // r * RB + t / GP + k * JS, k < kFlatPer, in rounds r of RB = JS * kFlatPer
 // blocks.  Every pass walks the rounds and re-reads the block stats
 // (L2-resident after the first pass), so loads are coalesced and nothing of

@@ -23,8 +23,10 @@
 // Then the normalised group score, the threshold, the B_min budget (radix
 // select, ties to the lower block index), compaction, and the kept-token
 // softmax normaliser (max, sum) that the decode pass uses.  This file holds
-// the flat kernel (a segment held in registers); longer segments and the
-// given keep sets of a standalone decode go to prune_wide.cu.
+// the scorer and the keep-set entry; the keep-set kernels are in
+// keep_tile.cu (segments of up to 8192 block-heads, rule mode) and
+// prune_wide.cu (longer segments, and the given keep sets of a standalone
+// decode).
 #include "common.cuh"
 #include "keep_set.cuh"
 
@@ -345,278 +347,6 @@ __global__ void __launch_bounds__(256) clear_words_kernel(uint32_t* w, int n) {
     for (int i = blockIdx.x * 256 + threadIdx.x; i < n; i += gridDim.x * 256) w[i] = 0u;
 }
 
-// ---------------------------------------------------------------------------
-// prune_finalize for segments of up to 16 * NT block-heads, one CTA of NT
-// threads per (sequence, kv head).  Flat layout: with GP the power of two
-// >= G, thread t owns query head h = t % GP of the blocks j = t / GP +
-// k * (NT / GP), k < kFlatPer, so the stats loads are coalesced, every
-// (block, head) term stays in registers from the load to the kept-token
-// normaliser, e^{m_b - M} is evaluated once, and the per-head reductions run
-// over lanes of equal h.  The GP lanes of a block end up with the same group
-// score, so they take the same keep decision; ranks in ascending block order
-// (budget ties, compaction) come from ballots over the head-0 lanes.
-template <int G, int NT>
-__global__ void __launch_bounds__(NT)
-prune_finalize_flat_kernel(const FinArgs a) {
-    constexpr int GP = FlatGP<G>::v;
-    constexpr int JS = NT / GP;                  // block stride between a thread's chunks
-    pdl_trigger();
-    pdl_wait();
-    extern __shared__ __align__(16) float ff_smem[];
-    float* sh_score = ff_smem;                   // [max_blocks] (budget select only)
-    __shared__ float red[4][2 * 32 * GP];
-    __shared__ int scan[2][kFlatPer * 32 + 1];
-    __shared__ int hist[256];
-    __shared__ int sel_digit, sel_rem;
-    __shared__ float arg_v[32];
-    __shared__ int arg_j[32];
-    const int seg = blockIdx.x;
-    const int b = seg / a.Hkv, kvh = seg - b * a.Hkv;
-    const int tid = threadIdx.x, lane = tid & 31;
-    const int h = lane & (GP - 1);
-    const int jt = tid / GP;
-    // chunk k holds no block below `bound` for any lane of this warp: the
-    // heavy passes skip it (a warp-uniform test)
-    const int jt0 = (tid & ~31) / GP;
-    auto live = [&](int k, int bound) { return jt0 + k * JS < bound; };
-    const int L = a.ctx_lens[b];
-    const float th = a.theta[b];
-    const bool bad_ctx = L < 0 || L > a.max_blocks * a.P;
-    const int nb = bad_ctx ? 0 : (L + a.P - 1) / a.P;
-    const long long segbase = (long long)seg * a.max_blocks;
-    const float4* st = a.stats + segbase * G;
-
-    const int bad = any_bad_page(a.block_table + (long long)b * a.max_blocks, tid, NT, nb, a.num_pages);
-    float m[kFlatPer], l1[kFlatPer], w[kFlatPer];   // w: u_b, then the block term I_b
-    int stale = 0;
-    float Mh[1] = {-kInf};
-#pragma unroll
-    for (int k = 0; k < kFlatPer; ++k) {
-        const int j = jt + k * JS;
-        m[k] = -kInf; l1[k] = 0.f; w[k] = 0.f;
-        if (!live(k, nb)) continue;
-        if (h < G && j < nb) {
-            const float4 s = st[(long long)j * G + h];
-            m[k] = s.x; l1[k] = s.y; w[k] = a.score_mode == 1 ? s.w : s.z;
-            stale |= (s.x != s.x);              // NaN max: the scoring pass gave up on this block
-            Mh[0] = fmaxf(Mh[0], s.x);
-        }
-    }
-    const bool bad_page = __syncthreads_or(bad) != 0;
-    const bool timed_out = __syncthreads_or(stale) != 0 && !bad_page;
-    bool drain = false;
-    if (timed_out) {
-        // rare: a block marked l - 1 = +inf had a copy in flight when the drain gave up
-        int d = 0;
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) {
-            const int j = jt + k * JS;
-            if (h < G && j < nb) d |= (m[k] != m[k]) && l1[k] == kInf;
-        }
-        drain = __syncthreads_or(d) != 0;
-    }
-    if (a.err && tid == 0) {
-        // err was cleared before this kernel; every kv head ORs in its bits
-        const uint32_t e = (bad_ctx ? ETI_ERRF_BAD_CTX : 0u) | (bad_page ? ETI_ERRF_BAD_PAGE : 0u) |
-                           (timed_out ? ETI_ERRF_TIMEOUT : 0u) | (drain ? ETI_ERRF_DRAIN : 0u);
-        if (e) atomicOr(a.err + b, e);
-    }
-    const int n = (bad_ctx || bad_page || timed_out) ? 0 : nb;
-    bool valid[kFlatPer];
-#pragma unroll
-    for (int k = 0; k < kFlatPer; ++k) valid[k] = h < G && jt + k * JS < n;
-
-    float M = -kInf, score[kFlatPer];
-#pragma unroll
-    for (int k = 0; k < kFlatPer; ++k) score[k] = -kInf;
-    if (n > 0) {
-        head_reduce<GP, 1, true>(Mh, red[0]);
-        M = Mh[0];
-        // Z - 1 = sum_b c_b l1_b + sum_{b: m_b < M} c_b + (#blocks at M - 1),
-        // c_b = e^{m_b - M}: the "1"s of the blocks at the max are counted, not
-        // summed, so log Z = log1p(Z - 1) keeps its relative precision when one
-        // token takes nearly all of the attention.
-        float zs[2] = {0.f, 0.f}, c[kFlatPer];
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k)
-            c[k] = 0.f;
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k)
-            if (live(k, n) && valid[k]) {
-                const bool top = !(m[k] < M);
-                c[k] = top ? 1.f : exp_le0(m[k] - M);
-                zs[0] += c[k] * l1[k] + (top ? 0.f : c[k]);
-                zs[1] += top ? 1.f : 0.f;
-            }
-        head_reduce<GP, 2, false>(zs, red[1]);
-        const float zm1 = zs[0] + (zs[1] - 1.f);
-        const float lZ = log1pf(zm1), iZ = 1.f / (1.f + zm1);
-        // I_b = e^{m_b - M}[(1 + l1_b)(log Z + M - m_b) - u_b] / Z; H = sum_b I_b
-        // (l1 becomes (1 + l1_b) e^{m_b - M}, the block's share of Z)
-        float Hs[1] = {0.f};
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k)
-            if (live(k, n) && valid[k]) {
-                if (a.score_mode == 1) w[k] = c[k] * w[k] * iZ;                 // E
-                else if (a.score_mode == 2) w[k] = c[k] * (1.f + l1[k]) * iZ;   // M
-                else w[k] = c[k] * ((1.f + l1[k]) * (lZ + M - m[k]) - w[k]) * iZ;
-                Hs[0] += w[k];
-                l1[k] = (1.f + l1[k]) * c[k];
-            }
-        head_reduce<GP, 1, false>(Hs, red[2]);
-        const float nH = Hs[0] > 0.f ? (float)n / Hs[0] : 0.f;
-        // group score: the largest normalised term over the heads of the block
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) {
-            if (!live(k, n)) continue;           // score[k] stays -inf
-            float s = valid[k] ? (Hs[0] > 0.f ? w[k] * nH : 1.f) : -kInf;
-#pragma unroll
-            for (int o = 1; o < GP; o <<= 1) s = fmaxf(s, __shfl_xor_sync(0xffffffffu, s, o));
-            score[k] = s;
-        }
-    }
-    if (a.block_score) {
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) {
-            const int j = jt + k * JS;
-            if (h == 0 && j < n) a.block_score[segbase + j] = score[k];
-        }
-        for (int j = n + tid; j < a.max_blocks; j += NT) a.block_score[segbase + j] = 0.f;
-    }
-
-    // B_min budget: the first k blocks by (score desc, index asc)
-    const int kb = min(max(a.B_min, 0), n);
-    bool keep[kFlatPer];
-#pragma unroll
-    for (int k = 0; k < kFlatPer; ++k) keep[k] = jt + k * JS < n && (score[k] >= th || kb >= n);
-    if (kb == 1 && n > 1) {
-        float bs = -kInf;
-        int bj = 0x7fffffff;
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) {
-            const int j = jt + k * JS;
-            if (j < n && (score[k] > bs || bj == 0x7fffffff)) { bs = score[k]; bj = j; }
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, bs, o);
-            const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
-            if (ov > bs || (ov == bs && oj < bj)) { bs = ov; bj = oj; }
-        }
-        if (lane == 0) { arg_v[tid >> 5] = bs; arg_j[tid >> 5] = bj; }
-        __syncthreads();
-        for (int u = 0; u < NT / 32; ++u)
-            if (arg_v[u] > bs || (arg_v[u] == bs && arg_j[u] < bj)) { bs = arg_v[u]; bj = arg_j[u]; }
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) keep[k] |= (jt + k * JS == bj);
-    } else if (kb > 1 && kb < n) {
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) {
-            const int j = jt + k * JS;
-            if (h == 0 && j < n) sh_score[j] = score[k];
-        }
-        __syncthreads();
-        uint32_t prefix = 0, mask = 0;
-        int need = kb;
-        for (int digit = 3; digit >= 0; --digit) {
-            const int sh = digit * 8;
-            for (int i = tid; i < 256; i += NT) hist[i] = 0;
-            __syncthreads();
-            for (int j0 = 0; j0 < n; j0 += NT) {      // the same trip count for every lane
-                const int j = j0 + tid;
-                const uint32_t key = j < n ? order_key(sh_score[j]) : 0u;
-                warp_hist_add(hist, (key >> sh) & 255, j < n && (key & mask) == prefix);
-            }
-            __syncthreads();
-            // bucket where the count from the top reaches `need`
-            if (tid < 32) {
-                int cnt8[8], s8 = 0;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) { cnt8[e] = hist[255 - (tid * 8 + e)]; s8 += cnt8[e]; }
-                int incl = s8;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const int y = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (tid >= o) incl += y;
-                }
-                int above = incl - s8;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    if (above < need && need <= above + cnt8[e]) {
-                        sel_digit = 255 - (tid * 8 + e);
-                        sel_rem = need - above;
-                    }
-                    above += cnt8[e];
-                }
-            }
-            __syncthreads();
-            prefix |= (uint32_t)sel_digit << sh;
-            mask |= 255u << sh;
-            need = sel_rem;
-            __syncthreads();
-        }
-        // keys above the k-th are in; of those equal to it, the lowest indices
-        bool eq[kFlatPer];
-        int eq_pos[kFlatPer];
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) {
-            const uint32_t key = order_key(score[k]);
-            eq[k] = jt + k * JS < n && key == prefix;
-            keep[k] |= jt + k * JS < n && key > prefix;
-        }
-        flat_ranks<GP>(eq, eq_pos, scan[0]);
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k) keep[k] |= eq[k] && eq_pos[k] < need;
-    }
-
-    // compaction (ascending block index)
-    int pos[kFlatPer];
-    const int total = flat_ranks<GP>(keep, pos, scan[1]);
-#pragma unroll
-    for (int k = 0; k < kFlatPer; ++k) {
-        const int j = jt + k * JS;
-        if (h == 0 && keep[k]) a.kept_idx[segbase + pos[k]] = j;
-        if (a.keep_mask && h == 0 && j < n) a.keep_mask[segbase + j] = keep[k] ? 1 : 0;
-    }
-    for (int i = total + tid; i < a.max_blocks; i += NT) a.kept_idx[segbase + i] = -1;
-    if (a.keep_mask)
-        for (int j = n + tid; j < a.max_blocks; j += NT) a.keep_mask[segbase + j] = 0;
-    if (tid == 0) a.kept_cnt[seg] = total;
-
-    // softmax normaliser over the kept tokens of each query head
-    if (a.kept_norm) {
-        float Mk[1] = {-kInf};
-#pragma unroll
-        for (int k = 0; k < kFlatPer; ++k)
-            if (valid[k] && keep[k]) Mk[0] = fmaxf(Mk[0], m[k]);
-        head_reduce<GP, 1, true>(Mk, red[3]);
-        float Lk[1] = {0.f};
-        if (Mk[0] == M) {
-#pragma unroll
-            for (int k = 0; k < kFlatPer; ++k)
-                if (valid[k] && keep[k]) Lk[0] += l1[k];
-        } else {
-            // the largest logit's block was pruned: rescale from the stats
-            // (a rolled loop: this path is rare and its code stays small)
-            uint32_t kk = 0;
-#pragma unroll
-            for (int k = 0; k < kFlatPer; ++k) kk |= (valid[k] && keep[k]) ? 1u << k : 0u;
-#pragma unroll 1
-            for (int k = 0; k < kFlatPer; ++k)
-                if ((kk >> k) & 1u) {
-                    const float4 s = st[(long long)(jt + k * JS) * G + h];
-                    Lk[0] += (1.f + s.y) * exp_le0(s.x - Mk[0]);
-                }
-        }
-        head_reduce<GP, 1, false>(Lk, red[0]);
-        if (tid < GP && h < G) {
-            float* kn = a.kept_norm + ((long long)b * a.Hq + kvh * a.g + h) * 2;
-            kn[0] = Mk[0];
-            kn[1] = Lk[0];
-        }
-    }
-}
-
 }  // namespace eti
 
 using namespace eti;
@@ -664,6 +394,8 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
 }
 
 cudaError_t eti_launch_prune_wide(const eti::FinArgs& a, int segs, int sms, cudaStream_t stream);
+bool eti_prune_tile_fits(int max_blocks, int g);
+cudaError_t eti_launch_prune_tile(const eti::FinArgs& a, cudaStream_t stream);
 
 int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, const int32_t* block_table,
                               long long num_pages, int B, int Hq, int Hkv, int P, int max_blocks,
@@ -693,46 +425,12 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
         if (eti_launch_pdl(clear_words_kernel, dim3((B + 255) / 256), dim3(256), 0, stream, err, B) != cudaSuccess)
             return ETI_ERR_CUDA;
     }
-    // the flat kernel holds a segment in registers: 16 block-heads a thread.
-    // Its work follows max_blocks whatever the segment's length, so it is
-    // taken when the segments run in one wave (at most four a SM, where it is
-    // latency-bound); more segments go to the segment kernel, whose work
-    // follows each segment's length (on 2048 segments of 4 to 512 blocks x 4
-    // heads: 23 against 41 us; on 512 segments of 64 to 512 blocks: 18.7
-    // against 16.6 us)
-    const int gp = a.g <= 1 ? 1 : a.g <= 2 ? 2 : a.g <= 4 ? 4 : 8;
-    const long long flat_need = ((long long)max_blocks * gp + kFlatPer - 1) / kFlatPer;
-    const bool seg_fits = (size_t)max_blocks * (gp + 1) * 4 <= kWideSmemMax / 2;
-    const int flat_nt = !given && theta && flat_need <= 512 && (grid <= 4 * sms || !seg_fits)
-                            ? (flat_need <= 128 ? 128 : flat_need <= 256 ? 256 : 512) : 0;
-#define ETI_FIN_FLAT(GG, NT)                                                                \
-    if (flat_nt == NT) {                                                                    \
-        auto k = prune_finalize_flat_kernel<GG, NT>;                                        \
-        const size_t smem = (size_t)max_blocks * 4;                                         \
-        if (smem > 48 * 1024) cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem); \
-        e = eti_launch_pdl(k, dim3(grid), dim3(NT), smem, stream, a);                       \
-        break;                                                                              \
-    }
-#define ETI_FIN_CASE(GG)                                                                    \
-    case GG: {                                                                              \
-        ETI_FIN_FLAT(GG, 128)                                                               \
-        ETI_FIN_FLAT(GG, 256)                                                               \
-        ETI_FIN_FLAT(GG, 512)                                                               \
-        e = eti_launch_prune_wide(a, grid, sms, stream);                                    \
-        break;                                                                              \
-    }
-    switch (a.g) {
-        ETI_FIN_CASE(1)
-        ETI_FIN_CASE(2)
-        ETI_FIN_CASE(3)
-        ETI_FIN_CASE(4)
-        ETI_FIN_CASE(5)
-        ETI_FIN_CASE(6)
-        ETI_FIN_CASE(7)
-        ETI_FIN_CASE(8)
-        default: return ETI_ERR_UNSUPPORTED;
-    }
-#undef ETI_FIN_CASE
-#undef ETI_FIN_FLAT
+    // segments of up to 8192 block-heads in the rule mode: the tile kernel
+    // (the stats staged in shared memory, work that follows each segment's
+    // length); the rest: prune_wide.cu
+    if (!given && theta && eti_prune_tile_fits(max_blocks, a.g))
+        e = eti_launch_prune_tile(a, stream);
+    else
+        e = eti_launch_prune_wide(a, grid, sms, stream);
     return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
 }

@@ -258,6 +258,9 @@ SHAPES = [
     (3, 24, 4, 64, 16, [129, 640, 2]),
     (2, 7, 7, 128, 16, [77, 400]),
     (2, 24, 3, 128, 32, [800, 95]),
+    # max_blocks * g of 8192: the keep-set tile kernel with eight warps a segment
+    (2, 64, 8, 128, 16, [16384, 5000]),
+    (3, 32, 8, 64, 16, [32768, 100, 20000]),
 ]
 
 

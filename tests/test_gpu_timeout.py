@@ -69,7 +69,7 @@ def _decode(eti, w, kv, o):
 
 
 def _workload(long_segments):
-    # flat keep-set kernel (max_blocks * g <= 8192) or the wide one
+    # the tile keep-set kernel (max_blocks * g <= 8192) or the wide one
     lens = [3000, 700, 1, 2500, 0] if not long_segments else [40000, 65536, 9000]
     return workloads.Workload("t", B=len(lens), Hq=32, Hkv=8, D=128, P=16, V=16, ctx=("list", lens),
                               seed=5, hi_frac=0.05)
