@@ -5,6 +5,11 @@ One step = one pass of the whole hot path over one batch:
   kept-token normaliser (eti_prune_blocks) -> GQA paged decode over the kept
   blocks (eti_paged_decode) -> entropy / entropic time / temperature /
   threshold / sample (eti_entropy_temp_sample).
+The step runs overlapped, as a serving loop would issue it: the sampling call
+on one stream and the attention half (score, keep set, decode) of each of two
+sub-batches (the batch's halves) on a stream of its own, all forked at the
+step's start and joined before its end; the same four calls over the whole
+batch on one stream give `ms_per_step_sequential`.
 The workload is the Llama-3-8B-shaped layer step (64 sequences, 32 query /
 8 kv heads, head_dim 128, page 16, context lengths uniform in [1024, 8192],
 vocabulary 128,256) with seeded synthetic inputs.
@@ -53,6 +58,7 @@ import workloads
 
 METRIC = "paged-decode tokens/s per layer-step"
 UNIT = "tokens/s"
+SUB_BATCHES = 2      # sub-batches of the overlapped step, each on its own stream
 
 
 def dist_env():
@@ -409,18 +415,57 @@ class StepRunner:
         self.theta = self.step.theta_next.clone()
         self.L = self.kv["ctx_lens"].cpu().numpy()
         self.total_blocks = int((-(-self.L // w.P)).sum()) * w.Hkv
+        # sub-batches of the overlapped step: contiguous runs of the batch whose
+        # calls write into views of the same outputs, each with its own decode
+        # workspace (two calls in flight must not share one)
+        nsplit = min(SUB_BATCHES, w.B)
+        bounds = [round(i * w.B / nsplit) for i in range(nsplit + 1)]
+        self.parts = []
+        for lo, hi in zip(bounds[:-1], bounds[1:]):
+            ws = torch.empty(eti.paged_decode_workspace_size(hi - lo, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, True),
+                             dtype=torch.uint8, device=device)
+            self.parts.append((lo, hi, (hi - lo, w.Hq, w.Hkv, w.D, w.P, w.max_blocks), ws))
 
-    def run(self, ev=None, offset=0, side=None):
-        """One step; with `ev` (5 events) an event between the calls.  With a
-        `side` stream the sampling call (which reads only the logits and the
-        per-sequence state) runs there, beside the attention half, and the
-        launching stream waits for it before the step ends."""
+    def attention_part(self, lo, hi, shape, ws, q=None, theta=None):
+        """Score, keep set and decode of sequences [lo, hi) on the current
+        stream (q and theta: the whole batch's, if not the runner's own)."""
+        eti, kv, st = self.eti, self.kv, self.step
+        q = (kv["q"] if q is None else q)[lo:hi]
+        theta = (self.theta if theta is None else theta)[lo:hi]
+        bt, cl = kv["block_table"][lo:hi], kv["ctx_lens"][lo:hi]
+        eti.eti_score_blocks(q, kv["k_cache"], bt, cl, kv["scale"], self.stats[lo:hi],
+                             token_scores=st.token_scores[lo:hi], num_pages=kv["num_pages"])
+        eti.eti_prune_blocks(self.stats[lo:hi], bt, cl, shape, theta, self.B_min,
+                             st.keep_mask[lo:hi], st.kept_idx[lo:hi], st.kept_cnt[lo:hi], st.err_attn[lo:hi],
+                             kept_norm=st.kept_norm[lo:hi], num_pages=kv["num_pages"])
+        eti.eti_paged_decode(q, kv["k_cache"], kv["v_cache"], bt, cl, kv["scale"], st.out[lo:hi],
+                             st.err_dec[lo:hi], ws, kept_idx=st.kept_idx[lo:hi], kept_cnt=st.kept_cnt[lo:hi],
+                             token_scores=st.token_scores[lo:hi], kept_norm=st.kept_norm[lo:hi],
+                             num_pages=kv["num_pages"])
+
+    def run(self, ev=None, offset=0, sched=None):
+        """One step; with `ev` (5 events) an event between the calls, all four
+        on the launching stream.  With `sched` = (side, subs) the step is
+        overlapped: the sampling call (which reads only the logits and the
+        per-sequence state) runs on `side`, and the attention half of each
+        sub-batch (score, keep set, decode) on its own stream of `subs`; all
+        fork at the step's start and the launching stream waits for them before
+        the step ends."""
         eti, kv, st, w = self.eti, self.kv, self.step, self.w
         s = self.stream
-        if side is not None:
+        if sched is not None:
+            side, subs = sched
             side.wait_stream(s)                  # fork
             st.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], self.lg["tau"],
                       self.lg["H_target"], params=self.prm, seed=w.seed, offset=offset, stream=side)
+            for part, sub in zip(self.parts, subs):
+                sub.wait_stream(s)
+                with torch.cuda.stream(sub):
+                    self.attention_part(*part)
+            for sub in subs[:len(self.parts)]:
+                s.wait_stream(sub)               # join
+            s.wait_stream(side)
+            return
         if ev is not None:
             ev[0].record(s)
         eti.eti_score_blocks(kv["q"], kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
@@ -438,11 +483,8 @@ class StepRunner:
                              num_pages=kv["num_pages"])
         if ev is not None:
             ev[3].record(s)
-        if side is None:
-            st.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], self.lg["tau"], self.lg["H_target"],
-                      params=self.prm, seed=w.seed, offset=offset)
-        else:
-            s.wait_stream(side)                  # join
+        st.sample(self.lg["logits"], self.lg["T_in"], self.lg["H_prev"], self.lg["tau"], self.lg["H_target"],
+                  params=self.prm, seed=w.seed, offset=offset)
         if ev is not None:
             ev[4].record(s)
 
@@ -496,26 +538,26 @@ def dense_decode_ms(r, flush_l2, reps=20):
     return ms
 
 
-def timed_steps(r, flush_l2, steps, offset0, side=None):
+def timed_steps(r, flush_l2, steps, offset0, sched=None):
     """Mean CUDA-event time (ms) of `steps` steps, L2 flushed before each."""
     evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
     for i in range(steps):
         flush_l2()
         evs[i][0].record(r.stream)
-        r.run(offset=offset0 + i, side=side)
+        r.run(offset=offset0 + i, sched=sched)
         evs[i][1].record(r.stream)
     torch.cuda.synchronize()
     return statistics.mean(e[0].elapsed_time(e[1]) for e in evs)
 
 
-def workload_summary(r, flush_l2, peak, steps, warmup, side, offset0=0):
+def workload_summary(r, flush_l2, peak, steps, warmup, sched, offset0=0):
     """Step time, throughput, kept fraction and per-kernel times / fractions of
     the HBM peak for one workload (same timing rules as the main line)."""
     w = r.w
     for i in range(warmup):
         flush_l2()
-        r.run(offset=offset0 + i, side=side)
-    ms = timed_steps(r, flush_l2, steps, offset0 + warmup, side)
+        r.run(offset=offset0 + i, sched=sched)
+    ms = timed_steps(r, flush_l2, steps, offset0 + warmup, sched)
     ms_seq = timed_steps(r, flush_l2, min(steps, 50), offset0 + warmup + steps)
     per = kernel_pass(r, flush_l2, min(steps, 50), offset0 + warmup + steps)
     kept = r.kept()
@@ -568,8 +610,11 @@ def run_gpu(args):
         w = w.scaled(B=args.batch)   # a reduced case of the same shape (for profiling)
     prm = eti.ctrl_params()
     stream = torch.cuda.current_stream()
-    side = torch.cuda.Stream(device=device)      # the sampling call runs beside the attention half
+    # the overlapped step: the sampling call on one stream, each sub-batch's
+    # attention half on another
+    sched = (torch.cuda.Stream(device=device), [torch.cuda.Stream(device=device) for _ in range(SUB_BATCHES)])
     r = StepRunner(eti, w, device, prm, stream)
+    nparts = len(r.parts)
     L2 = torch.cuda.get_device_properties(device).L2_cache_size
     flush_w = torch.empty(max(2 * L2, 256 << 20), dtype=torch.uint8, device=device)
     flush_r = torch.ones(max(2 * L2, 256 << 20) // 4, dtype=torch.int32, device=device)
@@ -588,7 +633,7 @@ def run_gpu(args):
 
     for i in range(args.warmup):
         flush_l2()
-        r.run(offset=i, side=side)
+        r.run(offset=i, sched=sched)
     torch.cuda.synchronize()
     kept = r.kept()
     total_blocks = r.total_blocks
@@ -610,7 +655,7 @@ def run_gpu(args):
         for i in range(args.steps):
             flush_l2()
             evs[i][0].record(stream)
-            r.run(offset=off + i, side=side)
+            r.run(offset=off + i, sched=sched)
             evs[i][1].record(stream)
         torch.cuda.synchronize()
         wall = time.perf_counter() - t0
@@ -626,7 +671,7 @@ def run_gpu(args):
             while time.perf_counter() - t1 < args.clock_seconds:
                 for _ in range(50):
                     flush_l2()
-                    r.run(offset=off + ncp, side=side)
+                    r.run(offset=off + ncp, sched=sched)
                     ncp += 1
                 torch.cuda.synchronize()
             e1.record(stream)
@@ -726,7 +771,7 @@ def run_gpu(args):
             res = []
             for f in fracs:
                 ro = StepRunner(eti, ow, device, prm, stream, H_target_frac=f)
-                s = workload_summary(ro, flush_l2, peak, ksteps, 5, side)
+                s = workload_summary(ro, flush_l2, peak, ksteps, 5, sched)
                 if f is not None:
                     s["H_target"] = f"{f} log V"
                 res.append(s)
@@ -741,9 +786,10 @@ def run_gpu(args):
         "data": "synthetic (seeded; Llama-3-8B-shaped layer step)",
         "ms_per_step_sequential": round(seq_ms, 5),
         "config": {"workload": main_desc,
-                   "streams": "the sampling call on a second stream beside the attention half "
-                              "(forked at the step's start, joined before its end event); "
-                              "ms_per_step_sequential: the four calls on one stream",
+                   "streams": f"the sampling call on one stream and the attention half (score, keep set, "
+                              f"decode) of each of {nparts} sub-batches (contiguous halves of the batch) "
+                              f"on its own, all forked at the step's start and joined before its end event; "
+                              f"ms_per_step_sequential: the four calls over the whole batch on one stream",
                    "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write, then 2x L2 read)",
                    "parallelism": f"replicas x{world} (independent batches)", "B_min": 1,
                    "theta": "theta_next of the step's own entropy (defaults)",
@@ -757,10 +803,11 @@ def run_gpu(args):
         "sampling": sampling,
         "attention_tbs": round((abytes["score"] + abytes["decode"]) / (attn_ms / 1e3) / 1e12, 3),
         "dense_baseline": dense,
-        "gpu_launches": 7 * args.steps,
-        "launches_per_step": {"score_blocks": 1, "clear_words (keep-set error words)": 1,
-                              "prune_finalize": 1, "decode_plan": 1, "paged_decode": 1,
-                              "ets_clear (sampling tickets)": 1, "entropy_sample": 1},
+        "gpu_launches": (5 * nparts + 2) * args.steps,
+        "launches_per_step": {"score_blocks": nparts, "clear_words (keep-set error words)": nparts,
+                              "prune_finalize": nparts, "decode_plan": nparts,
+                              "paged_decode": nparts, "ets_clear (sampling tickets)": 1,
+                              "entropy_sample": 1},
         "e2e": e2e,
         "estimators": est,
         "keep_sweep": sweep,
@@ -810,14 +857,16 @@ def run_e2e(eti, r, args, device):
 
     # The small inputs go up first; the logits (the bulk of the bytes) then go
     # up on a second stream, where the sampling call follows them and its
-    # results come down, all while the attention half runs on the first; the
-    # attention output comes down on the second stream once both are done.
+    # results come down, all while the attention half runs (each sub-batch's
+    # on a stream of its own, as in the device-resident step); the attention
+    # output comes down on the second stream once both are done.
     # The whole step (copies and calls, both streams) is captured once in a CUDA
     # graph and replayed every step, as a serving loop would; the sampling
     # offset lives in device memory (the call advances it), so every replay
     # draws fresh numbers.  If the capture is refused the same body runs eagerly.
     main = torch.cuda.current_stream()
     copy = torch.cuda.Stream(device=device)
+    subs = [torch.cuda.Stream(device=device) for _ in r.parts]
     ev_out = torch.cuda.Event()
     stages = ("start", "logits_up_start", "logits_up_end", "small_up_end", "attention_end", "out_down_end",
               "sample_end", "results_down_end", "end")
@@ -840,16 +889,12 @@ def run_e2e(eti, r, args, device):
             rec("sample_end", copy)
             h_res.copy_(d_io[qb + 4 * row:], non_blocking=True)
             rec("results_down_end", copy)
-        eti.eti_score_blocks(d_q, kv["k_cache"], kv["block_table"], kv["ctx_lens"], kv["scale"],
-                             r.stats, token_scores=step.token_scores, num_pages=kv["num_pages"])
-        eti.eti_prune_blocks(r.stats, kv["block_table"], kv["ctx_lens"], r.shape, th, r.B_min,
-                             step.keep_mask, step.kept_idx, step.kept_cnt, step.err_attn,
-                             kept_norm=step.kept_norm, num_pages=kv["num_pages"])
-        eti.eti_paged_decode(d_q, kv["k_cache"], kv["v_cache"], kv["block_table"], kv["ctx_lens"],
-                             kv["scale"], step.out, step.err_dec, step.ws_dec,
-                             kept_idx=step.kept_idx, kept_cnt=step.kept_cnt,
-                             token_scores=step.token_scores, kept_norm=step.kept_norm,
-                             num_pages=kv["num_pages"])
+        for part, sub in zip(r.parts, subs):
+            sub.wait_stream(cur)
+            with torch.cuda.stream(sub):
+                r.attention_part(*part, q=d_q, theta=th)
+        for sub in subs:
+            cur.wait_stream(sub)
         ev_out.record(cur)
         rec("attention_end", cur)
         with torch.cuda.stream(copy):
