@@ -394,7 +394,7 @@ int eti_launch_score_blocks(const uint16_t* q, const uint16_t* k_cache, const in
 }
 
 cudaError_t eti_launch_prune_wide(const eti::FinArgs& a, int segs, int sms, cudaStream_t stream);
-bool eti_prune_tile_fits(int max_blocks, int g);
+bool eti_prune_tile_fits(int max_blocks, int g, int B_min, int segs, int sms);
 cudaError_t eti_launch_prune_tile(const eti::FinArgs& a, cudaStream_t stream);
 
 int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, const int32_t* block_table,
@@ -425,12 +425,19 @@ int eti_launch_prune_finalize(const float4* stats, const int32_t* ctx_lens, cons
         if (eti_launch_pdl(clear_words_kernel, dim3((B + 255) / 256), dim3(256), 0, stream, err, B) != cudaSuccess)
             return ETI_ERR_CUDA;
     }
-    // segments of up to 8192 block-heads in the rule mode: the tile kernel
-    // (the stats staged in shared memory, work that follows each segment's
-    // length); the rest: prune_wide.cu
-    if (!given && theta && eti_prune_tile_fits(max_blocks, a.g))
+    // the rule mode with segments of up to 8192 block-heads, or up to 32768
+    // with B_min <= 1 and few segments (a cluster of CTAs a segment): the
+    // tile kernel (the stats staged in shared memory, work that follows each
+    // segment's length); the rest, and a cluster launch the device refuses:
+    // prune_wide.cu
+    if (!given && theta && eti_prune_tile_fits(max_blocks, a.g, B_min, grid, sms)) {
         e = eti_launch_prune_tile(a, stream);
-    else
+        if (e != cudaSuccess && (long long)max_blocks * a.g > 8192) {
+            (void)cudaGetLastError();
+            e = eti_launch_prune_wide(a, grid, sms, stream);
+        }
+    } else {
         e = eti_launch_prune_wide(a, grid, sms, stream);
+    }
     return e == cudaSuccess ? ETI_OK : ETI_ERR_CUDA;
 }

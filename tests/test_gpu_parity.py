@@ -261,6 +261,10 @@ SHAPES = [
     # max_blocks * g of 8192: the keep-set tile kernel with eight warps a segment
     (2, 64, 8, 128, 16, [16384, 5000]),
     (3, 32, 8, 64, 16, [32768, 100, 20000]),
+    # 16384 and 32768: clusters of four and eight CTAs a segment (B_min <= 1;
+    # larger budgets go to the wide kernel)
+    (2, 32, 8, 64, 16, [65536, 3000]),
+    (2, 64, 8, 64, 16, [65536, 777]),
 ]
 
 
