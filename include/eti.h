@@ -222,7 +222,7 @@ int eti_entropy_temp_sample(const float* logits, int B, int V, int64_t ld,
  *    threads) race on the array: serialise them.
  *  - A problem whose scratch (eti_entropy_temp_sample_workspace_size(B, V))
  *    exceeds the array returns ETI_ERR_TOO_LARGE and enqueues nothing; at
- *    152 SMs the limit is about 14,500 sequences, whatever V is.
+ *    152 SMs the limit is about 16,600 sequences, whatever V is.
  */
 size_t eti_entropy_temp_sample_noalloc_max_bytes(void);
 
