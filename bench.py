@@ -392,6 +392,14 @@ def pool_for(w, device) -> int | None:
     return min(w.pool, 1 << max(10, cap.bit_length() - 1))
 
 
+def sub_batches(B: int, n: int) -> list[tuple[int, int]]:
+    """Contiguous runs [lo, hi) that cover sequences 0 .. B-1 in order, as
+    even as the count allows, never empty (fewer runs than n when B < n)."""
+    n = max(1, min(n, B))
+    bounds = [round(i * B / n) for i in range(n + 1)]
+    return list(zip(bounds[:-1], bounds[1:]))
+
+
 class StepRunner:
     """One workload's inputs, buffers and the four calls of the step (score
     -> keep set -> decode over the kept blocks -> entropy / sample)."""
@@ -418,10 +426,8 @@ class StepRunner:
         # sub-batches of the overlapped step: contiguous runs of the batch whose
         # calls write into views of the same outputs, each with its own decode
         # workspace (two calls in flight must not share one)
-        nsplit = min(SUB_BATCHES, w.B)
-        bounds = [round(i * w.B / nsplit) for i in range(nsplit + 1)]
         self.parts = []
-        for lo, hi in zip(bounds[:-1], bounds[1:]):
+        for lo, hi in sub_batches(w.B, SUB_BATCHES):
             ws = torch.empty(eti.paged_decode_workspace_size(hi - lo, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, True),
                              dtype=torch.uint8, device=device)
             self.parts.append((lo, hi, (hi - lo, w.Hq, w.Hkv, w.D, w.P, w.max_blocks), ws))

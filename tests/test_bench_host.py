@@ -198,3 +198,17 @@ def test_kept_attention_mass_matches_the_oracle(oracle_lib):
     # keeping every block keeps all of the attention
     full = bench.kept_attention_mass(stats, torch.ones_like(keep), kv["ctx_lens"], w.P)
     assert full["mean"] == pytest.approx(1.0, abs=1e-6) and full["min"] == pytest.approx(1.0, abs=1e-6)
+
+
+def test_sub_batches_cover_the_batch_in_order():
+    """The overlapped step's sub-batches: contiguous, in order, disjoint,
+    covering every sequence once, none empty, sizes within one of each other."""
+    for B in (1, 2, 3, 4, 7, 8, 64, 65, 128, 256, 8191):
+        for n in (1, 2, 3, 4, 8):
+            runs = bench.sub_batches(B, n)
+            assert len(runs) == min(n, B)
+            assert runs[0][0] == 0 and runs[-1][1] == B
+            assert all(a[1] == b[0] for a, b in zip(runs, runs[1:]))
+            sizes = [hi - lo for lo, hi in runs]
+            assert min(sizes) >= 1 and max(sizes) - min(sizes) <= 1
+
