@@ -491,9 +491,9 @@ static cudaError_t launch_tile_shape(const FinArgs& a, cudaStream_t stream) {
 // Four warps a CTA up to 4096 block-heads (fewer leave the longest
 // segments' chains exposed, more add per-warp work: on the Llama-3-8B-shaped
 // step 2/4/8/16 warps took 18.9/16.0/16.4/21.1 us), eight above, and above
-// 8192 a cluster of CTAs a segment.  Returns cudaErrorInvalidValue for a
-// shape the caller must send elsewhere (and a cluster launch the device
-// refuses returns its error: the caller falls back).
+// 8192 a cluster of CTAs a segment.  The caller sends only the shapes that
+// eti_prune_tile_fits accepts; a cluster launch the device refuses returns
+// its error, and the caller falls back to the wide kernel.
 cudaError_t eti_launch_prune_tile(const FinArgs& a, cudaStream_t stream) {
     switch (a.g) {
         case 1: return launch_tile_shape<1>(a, stream);
