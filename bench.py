@@ -51,6 +51,12 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+# The overlapped step runs on several streams at once (the sampling call and
+# one per sub-batch, the copy stream of the end-to-end step); with the driver's
+# default of 8 hardware work queues, two of them could share a queue and run
+# one after the other (a per-process draw).  Before CUDA starts:
+os.environ.setdefault("CUDA_DEVICE_MAX_CONNECTIONS", "32")
+
 import numpy as np
 import torch
 
@@ -392,11 +398,23 @@ def pool_for(w, device) -> int | None:
     return min(w.pool, 1 << max(10, cap.bit_length() - 1))
 
 
-def sub_batches(B: int, n: int) -> list[tuple[int, int]]:
-    """Contiguous runs [lo, hi) that cover sequences 0 .. B-1 in order, as
-    even as the count allows, never empty (fewer runs than n when B < n)."""
+def sub_batches(B: int, n: int, weights=None) -> list[tuple[int, int]]:
+    """Contiguous runs [lo, hi) that cover sequences 0 .. B-1 in order, never
+    empty (fewer runs than n when B < n): as even in count as possible, or,
+    with per-sequence `weights` (the blocks each reads), cut where the
+    running weight crosses each i/n of the total."""
     n = max(1, min(n, B))
-    bounds = [round(i * B / n) for i in range(n + 1)]
+    if weights is None:
+        bounds = [round(i * B / n) for i in range(n + 1)]
+    else:
+        cum = np.concatenate([[0.0], np.cumsum(np.asarray(weights, dtype=np.float64))])
+        bounds = [0]
+        for i in range(1, n):
+            k = int(np.searchsorted(cum, cum[-1] * i / n))            # first prefix >= the target
+            if k > 0 and abs(cum[k - 1] - cum[-1] * i / n) <= abs(cum[k] - cum[-1] * i / n):
+                k -= 1
+            bounds.append(min(max(k, bounds[-1] + 1), B - (n - i)))   # non-empty runs
+        bounds.append(B)
     return list(zip(bounds[:-1], bounds[1:]))
 
 
@@ -427,7 +445,7 @@ class StepRunner:
         # calls write into views of the same outputs, each with its own decode
         # workspace (two calls in flight must not share one)
         self.parts = []
-        for lo, hi in sub_batches(w.B, SUB_BATCHES):
+        for lo, hi in sub_batches(w.B, SUB_BATCHES, weights=-(-self.L // w.P)):
             ws = torch.empty(eti.paged_decode_workspace_size(hi - lo, w.Hq, w.Hkv, w.D, w.P, w.max_blocks, True),
                              dtype=torch.uint8, device=device)
             self.parts.append((lo, hi, (hi - lo, w.Hq, w.Hkv, w.D, w.P, w.max_blocks), ws))

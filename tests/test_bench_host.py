@@ -212,3 +212,24 @@ def test_sub_batches_cover_the_batch_in_order():
             sizes = [hi - lo for lo, hi in runs]
             assert min(sizes) >= 1 and max(sizes) - min(sizes) <= 1
 
+
+def test_sub_batches_by_weight_balance_the_work():
+    """With per-sequence weights the cuts fall where the running weight
+    crosses each share of the total (the best cut in the sequence order),
+    the runs stay contiguous and non-empty."""
+    rng = np.random.default_rng(0)
+    for B in (2, 3, 7, 64, 256):
+        wts = rng.integers(1, 512, size=B)
+        for n in (1, 2, 3, 4):
+            runs = bench.sub_batches(B, n, weights=wts)
+            assert len(runs) == min(n, B)
+            assert runs[0][0] == 0 and runs[-1][1] == B
+            assert all(a[1] == b[0] and a[0] < a[1] for a, b in zip(runs, runs[1:]))
+            if n == 2 and B > 2:
+                cut = runs[0][1]
+                tot = wts.sum()
+                best = min(abs(wts[:k].sum() - tot / 2) for k in range(1, B))
+                assert abs(wts[:cut].sum() - tot / 2) == best
+    assert bench.sub_batches(4, 2, weights=[1, 1, 1, 100]) == [(0, 3), (3, 4)]
+    assert bench.sub_batches(4, 2, weights=[100, 1, 1, 1]) == [(0, 1), (1, 4)]
+
