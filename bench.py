@@ -635,8 +635,10 @@ def run_gpu(args):
     prm = eti.ctrl_params()
     stream = torch.cuda.current_stream()
     # the overlapped step: the sampling call on one stream, each sub-batch's
-    # attention half on another
-    sched = (torch.cuda.Stream(device=device), [torch.cuda.Stream(device=device) for _ in range(SUB_BATCHES)])
+    # attention half on another, of higher priority (the attention half is
+    # the step's critical path; the sampling call fills the SMs it leaves)
+    sched = (torch.cuda.Stream(device=device, priority=0),
+             [torch.cuda.Stream(device=device, priority=-1) for _ in range(SUB_BATCHES)])
     r = StepRunner(eti, w, device, prm, stream)
     nparts = len(r.parts)
     L2 = torch.cuda.get_device_properties(device).L2_cache_size
