@@ -813,9 +813,10 @@ def run_gpu(args):
         "ms_per_step_sequential": round(seq_ms, 5),
         "config": {"workload": main_desc,
                    "streams": f"the sampling call on one stream and the attention half (score, keep set, "
-                              f"decode) of each of {nparts} sub-batches (contiguous halves of the batch) "
-                              f"on its own, all forked at the step's start and joined before its end event; "
-                              f"ms_per_step_sequential: the four calls over the whole batch on one stream",
+                              f"decode) of each of {nparts} sub-batches (contiguous runs of the batch with "
+                              f"about equal blocks) on its own, of higher priority, all forked at the step's "
+                              f"start and joined before its end event; ms_per_step_sequential: the four "
+                              f"calls over the whole batch on one stream",
                    "global_batch": w.B * world, "l2": "flushed before every step (2x L2 write, then 2x L2 read)",
                    "parallelism": f"replicas x{world} (independent batches)", "B_min": 1,
                    "theta": "theta_next of the step's own entropy (defaults)",
